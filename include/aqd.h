@@ -1,0 +1,201 @@
+/*
+ * aqd.h -- C ABI of libaqd: integer-only quantized convolution for GB300 (sm_103a).
+ *
+ * Implements the inference path of AQD (Chen et al., "AQD: Towards Accurate Quantized
+ * Object Detection", arXiv 2007.06919, Sec. 3.2): convolution on low-bit integer codes
+ * (Eq. 4) followed by a fused integer epilogue -- the folded batch-norm bias (Eq. 6,
+ * optionally one parameter set per FPN level for multi-level BN, Sec. 3.2.2 / Fig. 3),
+ * the dyadically rescaled skip add (Eq. 7 with F of Eq. 8), and the fixed-point rescale,
+ * round and clip that produce the next layer's k-bit codes (Eq. 2). No floating point
+ * value crosses a layer boundary.
+ *
+ * Conventions for every entry point
+ *   - Pointers inside aqd_tensor / parameter structs are DEVICE pointers owned by the
+ *     caller; the structs themselves live in host memory and are read before return.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream). Work is enqueued on it;
+ *     no entry point synchronizes except aqd_device_status.
+ *   - The library allocates no device memory. Errors come back as aqd_status; argument
+ *     errors are detected before any launch and launch nothing. C++ exceptions never
+ *     cross this boundary. aqd_last_error() gives a message for the calling thread.
+ *   - Device-side failures (a bounded wait that timed out, a failed device check) are
+ *     latched in a device status word that aqd_device_status() reads and clears.
+ *
+ * Tensor layout (NHWC, one "row" = the C channels of one pixel)
+ *   bits 2, 4, 8 (unsigned codes, Eq. 2 range [0, 2^k - 1]):
+ *     a row is a run of 32-bit little-endian words; word w holds channels [w*q, (w+1)*q)
+ *     with q = 32/bits, and channel i of its word sits at bit 8*(i%4) + bits*(i/4).
+ *     bits 8 is plain bytes. bits 2 and 4 need C % 32 == 0.
+ *   bits 3: each group of 32 channels takes 12 bytes = 3 words; words 0 and 1 hold the
+ *     low 2 bits of channels 0..15 and 16..31 in the 2-bit layout, word 2 holds bit 2 of
+ *     channel i at bit 8*(i%4) + i/4. Needs C % 32 == 0.
+ *   bits 32: one int32 per channel (accumulator-domain values, e.g. detection-head
+ *     outputs whose scale is passed on to the next stage, Sec. 3.2.1).
+ *   Rows are contiguous: pixel (n, h, w) starts at byte ((n*H + h)*W + w) * row_bytes.
+ *   Code tensors must be 16-byte aligned.
+ *
+ * Arithmetic of one output element (all integer; rhu(v, R) = floor((v + 2^(R-1)) / 2^R),
+ * rhu(v, 0) = v; sat32 saturates to int32):
+ *   acc = sum_{r,s,c} x[n, ho*S - P + r, wo*S - P + s, c] * w[co, r, s, c]   (Eq. 4;
+ *         taps outside the image read code 0, the zero point of Eq. 2)
+ *   t   = acc + bias[l][co]                                                   (Eq. 6)
+ *   with a skip tensor s (Eq. 7, F(m, n) = c / 2^d of Eq. 8):
+ *     scale_main = 0 (skip coarser): t = t + rhu(s * c[l][co], d[l][co])
+ *     scale_main = 1 (main coarser): t = rhu(sat32(t) * c[l][co], d[l][co]) + s
+ *   u   = sat32(t)
+ *   out = u                                            for 32-bit outputs
+ *   out = min(max(rhu(u * M0[l][co], 31 + shift[l][co]), 0), 2^k - 1)   for k-bit codes
+ *         (Eq. 2 applied to the BN output; the clip at 0 is the ReLU)
+ * Weights: signed integers w, either k-bit two's complement (AQD_W_TWOS) or Eq. 3's
+ * unsigned eta_w standing for 2*eta_w - (2^k - 1) (AQD_W_ODD, the odd grid of Eq. 4).
+ */
+#ifndef AQD_H
+#define AQD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef void* aqd_stream_t; /* a cudaStream_t */
+
+typedef enum {
+  AQD_OK = 0,
+  AQD_ERR_INVALID = 1,      /* bad argument; nothing launched */
+  AQD_ERR_UNSUPPORTED = 2,  /* valid but outside what the kernels implement */
+  AQD_ERR_CUDA = 3,         /* a CUDA runtime call failed */
+  AQD_ERR_TIMEOUT = 4,      /* a bounded device-side wait expired (device status) */
+  AQD_ERR_DEVICE_CHECK = 5  /* a device-side consistency check failed (device status) */
+} aqd_status;
+
+enum { AQD_W_TWOS = 0, AQD_W_ODD = 1 };
+
+typedef struct {
+  int32_t n, h, w, c; /* logical NHWC shape */
+  int32_t bits;       /* 2, 3, 4, 8: packed unsigned codes; 32: int32 values */
+  void* data;         /* device pointer, layout above */
+} aqd_tensor;
+
+/* Per-(level, output channel) requant tables, each [levels][cout] row-major (Eq. 6, the
+ * multi-level BN of Sec. 3.2.2 keeps one row per FPN level over shared weights).
+ * m0/shift may be NULL when the output is 32-bit; bias may be NULL (all zero).
+ * shift must lie in [-31, 31] (total right shift 31 + shift in [0, 62]). */
+typedef struct {
+  const int32_t* m0;
+  const int8_t* shift;
+  const int32_t* bias;
+  int32_t levels;
+} aqd_requant_params;
+
+/* Skip-add rescale of Eq. 7/8, tables [levels][cout]: c any int32, d in [0, 62].
+ * upsample = 2 reads the skip at (h/2, w/2): the nearest 2x interpolation of the FPN
+ * top-down path (Sec. 3.2.3 occasion 3 with Sec. 3.2.4). */
+typedef struct {
+  const int32_t* c;
+  const int8_t* d;
+  int32_t upsample;   /* 1 or 2 */
+  int32_t scale_main; /* 0: the skip is rescaled; 1: the main branch is rescaled */
+} aqd_skip_params;
+
+/* Prepared weights: written once by aqd_conv_prepare_weights, read by every conv call. */
+typedef struct {
+  const void* data; /* device buffer of aqd_conv_weights_bytes() bytes, 256-byte aligned */
+  int32_t cout, kh, kw, cin;
+  int32_t w_bits;   /* 2, 3, 4 or 8 */
+  int32_t w_format; /* AQD_W_TWOS or AQD_W_ODD */
+} aqd_conv_weights;
+
+/* One image group of a grouped convolution (e.g. one FPN level). */
+typedef struct {
+  aqd_tensor x;    /* input codes */
+  aqd_tensor y;    /* output: codes or int32 */
+  aqd_tensor skip; /* skip operand; skip.data == NULL means no skip for this job */
+  int32_t level;   /* row of the requant / skip tables */
+} aqd_conv_job;
+
+/* ---- host helpers ---------------------------------------------------------------- */
+
+/* Bytes of one packed row of c channels at `bits`, or -1 if the layout does not exist. */
+int64_t aqd_row_bytes(int32_t c, int32_t bits);
+
+/* Eq. 8: the dyadic approximation m0 * 2^-(31 + shift) of `real` with |m0| < 2^31 and
+ * 31 + shift in [0, 62] that minimizes the absolute error (largest shift whose
+ * round-half-up m0 still fits). real = 0 gives (0, 0). Host only; no device work. */
+aqd_status aqd_quantize_multiplier(double real, int32_t* m0, int8_t* shift);
+
+const char* aqd_status_string(aqd_status s);
+const char* aqd_last_error(void);
+
+/* Reads and clears the device status word of the current device (synchronizes the
+ * stream). *code receives AQD_OK or the first latched AQD_ERR_TIMEOUT /
+ * AQD_ERR_DEVICE_CHECK. */
+aqd_status aqd_device_status(aqd_stream_t stream, int32_t* code);
+
+/* Diagnostics: force the convolution kernel (0 = automatic choice, 1 = tensor-core
+ * kernel when the shape allows it, 2 = CUDA-core kernel); returns the previous setting,
+ * or -1 for an unknown value. aqd_last_conv_path() reports the kernel the calling
+ * thread's last successful conv call used (1 tensor core, 2 CUDA core, 0 none yet). */
+int32_t aqd_set_conv_path(int32_t path);
+int32_t aqd_last_conv_path(void);
+
+/* ---- codes <-> int32 ----------------------------------------------------------- */
+
+/* Packs rows x c int32 codes (device) into the k-bit layout (low k bits of each value;
+ * signed weights therefore pack as two's complement). bits 2/3/4/8. */
+aqd_status aqd_pack_codes(const int32_t* codes, int64_t rows, int32_t c, int32_t bits,
+                          void* out, aqd_stream_t stream);
+/* Inverse of aqd_pack_codes; is_signed sign-extends two's-complement fields. */
+aqd_status aqd_unpack_codes(const void* packed, int64_t rows, int32_t c, int32_t bits,
+                            int32_t is_signed, int32_t* out, aqd_stream_t stream);
+
+/* ---- convolution (Eq. 4 + fused epilogue) ----------------------------------------- */
+
+/* Size of the prepared-weights buffer for a [cout][kh][kw][cin] kernel. */
+size_t aqd_conv_weights_bytes(int32_t cout, int32_t kh, int32_t kw, int32_t cin);
+
+/* Converts packed signed weights [cout][kh][kw][cin] (rows packed along cin in the
+ * w_bits layout) into the prepared layout at w->data (the struct's shape fields must be
+ * filled in). Done once per model load; conv calls then read the prepared form. */
+aqd_status aqd_conv_prepare_weights(const void* w_packed, const aqd_conv_weights* w,
+                                    void* w_prepared, size_t bytes, aqd_stream_t stream);
+
+/* One convolution y = epilogue(conv(x, w)) at the given level of the tables.
+ * skip may be NULL (no skip; sp ignored). y->bits selects the output: 2/3/4/8 codes or
+ * 32 (int32, rq->m0/shift unused). rq may be NULL only for 32-bit outputs (no bias). */
+aqd_status aqd_conv_int(const aqd_tensor* x, const aqd_conv_weights* w, int32_t stride,
+                        int32_t pad, int32_t level, const aqd_requant_params* rq,
+                        const aqd_tensor* skip, const aqd_skip_params* sp, aqd_tensor* y,
+                        aqd_stream_t stream);
+
+/* The same convolution over up to 8 jobs with shared weights in ONE launch: the shared
+ * detector head applied to every FPN level, each with its own level's BN row. All jobs
+ * share x->c, y->bits, skip presence and the weights; spatial sizes and batch differ. */
+aqd_status aqd_conv_int_grouped(const aqd_conv_job* jobs, int32_t njobs,
+                                const aqd_conv_weights* w, int32_t stride, int32_t pad,
+                                const aqd_requant_params* rq, const aqd_skip_params* sp,
+                                aqd_stream_t stream);
+
+/* ---- elementwise ------------------------------------------------------------------ */
+
+/* y = requant(sat32(acc + bias)) per channel at `level`: Eq. 6 + Eq. 2 on an int32
+ * accumulator tensor. y->bits 2/3/4/8 (or 32: sat32(acc + bias)). */
+aqd_status aqd_requant(const aqd_tensor* acc, const aqd_requant_params* rq, int32_t level,
+                       aqd_tensor* y, aqd_stream_t stream);
+
+/* Eq. 7 on two tensors: a plays the accumulator (codes or int32), b the skip (codes or
+ * int32, half size when sp->upsample == 2). rq NULL: 32-bit output sat32(result) with no
+ * bias; otherwise bias is added to a first and y->bits selects the output as above. */
+aqd_status aqd_residual_add_int(const aqd_tensor* a, const aqd_tensor* b,
+                                const aqd_skip_params* sp, const aqd_requant_params* rq,
+                                int32_t level, aqd_tensor* y, aqd_stream_t stream);
+
+/* Sec. 3.2.4: k x k max-pooling (stride, zero-or-more padding < k) directly on codes;
+ * padded taps are ignored. y has x's bits. */
+aqd_status aqd_maxpool_codes(const aqd_tensor* x, int32_t k, int32_t stride, int32_t pad,
+                             aqd_tensor* y, aqd_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* AQD_H */

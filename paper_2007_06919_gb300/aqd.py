@@ -1,0 +1,344 @@
+"""Thin ctypes binding of libaqd (include/aqd.h), with the same entry-point names.
+
+Only argument marshalling happens here: every step of the integer convolution path runs
+in libaqd's CUDA kernels. PyTorch supplies device memory and the current stream. There is
+no CPU fallback: if the library or a GPU is missing the calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import torch
+
+from . import build as _build
+
+W_TWOS = 0
+W_ODD = 1
+
+STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported", 3: "CUDA error", 4: "device wait timed out",
+          5: "device check failed"}
+
+
+class AqdError(RuntimeError):
+    def __init__(self, status: int, func: str, msg: str):
+        super().__init__(f"{func}: {STATUS.get(status, status)}: {msg}")
+        self.status = status
+
+
+class _Tensor(ctypes.Structure):
+    _fields_ = [("n", ctypes.c_int32), ("h", ctypes.c_int32), ("w", ctypes.c_int32), ("c", ctypes.c_int32),
+                ("bits", ctypes.c_int32), ("data", ctypes.c_void_p)]
+
+
+class _Requant(ctypes.Structure):
+    _fields_ = [("m0", ctypes.c_void_p), ("shift", ctypes.c_void_p), ("bias", ctypes.c_void_p),
+                ("levels", ctypes.c_int32)]
+
+
+class _Skip(ctypes.Structure):
+    _fields_ = [("c", ctypes.c_void_p), ("d", ctypes.c_void_p), ("upsample", ctypes.c_int32),
+                ("scale_main", ctypes.c_int32)]
+
+
+class _Weights(ctypes.Structure):
+    _fields_ = [("data", ctypes.c_void_p), ("cout", ctypes.c_int32), ("kh", ctypes.c_int32),
+                ("kw", ctypes.c_int32), ("cin", ctypes.c_int32), ("w_bits", ctypes.c_int32),
+                ("w_format", ctypes.c_int32)]
+
+
+class _Job(ctypes.Structure):
+    _fields_ = [("x", _Tensor), ("y", _Tensor), ("skip", _Tensor), ("level", ctypes.c_int32)]
+
+
+EXPORTS = ["aqd_row_bytes", "aqd_quantize_multiplier", "aqd_status_string", "aqd_last_error",
+           "aqd_device_status", "aqd_set_conv_path", "aqd_last_conv_path", "aqd_pack_codes",
+           "aqd_unpack_codes", "aqd_conv_weights_bytes", "aqd_conv_prepare_weights", "aqd_conv_int",
+           "aqd_conv_int_grouped", "aqd_requant", "aqd_residual_add_int", "aqd_maxpool_codes"]
+
+_lib = None
+
+
+def lib_path() -> str:
+    return _build.LIB
+
+
+def load(build_if_missing: bool = True):
+    """Loads libaqd.so (building it in-tree first if it is missing)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = _build.LIB
+    if not os.path.exists(path):
+        if not build_if_missing:
+            raise FileNotFoundError(f"{path} is not built")
+        _build.build()
+    L = ctypes.CDLL(path)
+    c_int, i32, i64, vp = ctypes.c_int, ctypes.c_int32, ctypes.c_int64, ctypes.c_void_p
+    L.aqd_row_bytes.restype = i64
+    L.aqd_row_bytes.argtypes = [i32, i32]
+    L.aqd_quantize_multiplier.argtypes = [ctypes.c_double, ctypes.POINTER(i32), ctypes.POINTER(ctypes.c_int8)]
+    L.aqd_status_string.restype = ctypes.c_char_p
+    L.aqd_status_string.argtypes = [c_int]
+    L.aqd_last_error.restype = ctypes.c_char_p
+    L.aqd_device_status.argtypes = [vp, ctypes.POINTER(i32)]
+    L.aqd_set_conv_path.restype = i32
+    L.aqd_set_conv_path.argtypes = [i32]
+    L.aqd_last_conv_path.restype = i32
+    L.aqd_pack_codes.argtypes = [vp, i64, i32, i32, vp, vp]
+    L.aqd_unpack_codes.argtypes = [vp, i64, i32, i32, i32, vp, vp]
+    L.aqd_conv_weights_bytes.restype = ctypes.c_size_t
+    L.aqd_conv_weights_bytes.argtypes = [i32, i32, i32, i32]
+    L.aqd_conv_prepare_weights.argtypes = [vp, ctypes.POINTER(_Weights), vp, ctypes.c_size_t, vp]
+    L.aqd_conv_int.argtypes = [ctypes.POINTER(_Tensor), ctypes.POINTER(_Weights), i32, i32, i32,
+                               ctypes.POINTER(_Requant), ctypes.POINTER(_Tensor), ctypes.POINTER(_Skip),
+                               ctypes.POINTER(_Tensor), vp]
+    L.aqd_conv_int_grouped.argtypes = [ctypes.POINTER(_Job), i32, ctypes.POINTER(_Weights), i32, i32,
+                                       ctypes.POINTER(_Requant), ctypes.POINTER(_Skip), vp]
+    L.aqd_requant.argtypes = [ctypes.POINTER(_Tensor), ctypes.POINTER(_Requant), i32, ctypes.POINTER(_Tensor), vp]
+    L.aqd_residual_add_int.argtypes = [ctypes.POINTER(_Tensor), ctypes.POINTER(_Tensor), ctypes.POINTER(_Skip),
+                                       ctypes.POINTER(_Requant), i32, ctypes.POINTER(_Tensor), vp]
+    L.aqd_maxpool_codes.argtypes = [ctypes.POINTER(_Tensor), i32, i32, i32, ctypes.POINTER(_Tensor), vp]
+    for name in ("aqd_quantize_multiplier", "aqd_device_status", "aqd_pack_codes", "aqd_unpack_codes",
+                 "aqd_conv_prepare_weights", "aqd_conv_int", "aqd_conv_int_grouped", "aqd_requant",
+                 "aqd_residual_add_int", "aqd_maxpool_codes"):
+        getattr(L, name).restype = c_int
+    _lib = L
+    return L
+
+
+def _check(st: int, func: str):
+    if st != 0:
+        msg = load().aqd_last_error().decode(errors="replace")
+        raise AqdError(st, func, msg)
+
+
+def _stream(stream=None) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream
+
+
+def _ptr(t: torch.Tensor | None):
+    if t is None:
+        return None
+    assert t.is_cuda and t.is_contiguous(), "device tensors must be contiguous CUDA tensors"
+    return t.data_ptr()
+
+
+# ------------------------------------------------------------------ tensors
+
+
+def row_bytes(c: int, bits: int) -> int:
+    return int(load().aqd_row_bytes(c, bits))
+
+
+@dataclass
+class DTensor:
+    """A packed NHWC code tensor (or int32 tensor) in device memory."""
+    data: torch.Tensor  # uint8 [n, h, w, row_bytes] (any contiguous byte buffer of that size)
+    n: int
+    h: int
+    w: int
+    c: int
+    bits: int
+
+    @classmethod
+    def empty(cls, n, h, w, c, bits, device="cuda"):
+        rb = row_bytes(c, bits)
+        if rb < 0:
+            raise ValueError(f"no packed layout for C={c} at {bits} bits")
+        return cls(torch.empty((n, h, w, rb), dtype=torch.uint8, device=device), n, h, w, c, bits)
+
+    @classmethod
+    def from_codes(cls, codes: torch.Tensor, bits: int) -> "DTensor":
+        """codes: int32 CUDA tensor [n, h, w, c]."""
+        n, h, w, c = codes.shape
+        if bits == 32:
+            data = codes.to(torch.int32).contiguous().view(torch.uint8).reshape(n, h, w, 4 * c)
+            return cls(data, n, h, w, c, 32)
+        out = cls.empty(n, h, w, c, bits, device=codes.device)
+        pack_codes(codes.reshape(-1, c), bits, out=out.data)
+        return out
+
+    def codes(self, signed: bool = False) -> torch.Tensor:
+        if self.bits == 32:
+            return self.data.contiguous().view(torch.int32).reshape(self.n, self.h, self.w, self.c)
+        return unpack_codes(self.data.reshape(-1, row_bytes(self.c, self.bits)), self.c, self.bits,
+                            signed).reshape(self.n, self.h, self.w, self.c)
+
+    def ct(self) -> _Tensor:
+        assert self.data.numel() * self.data.element_size() == self.n * self.h * self.w * row_bytes(self.c, self.bits)
+        return _Tensor(self.n, self.h, self.w, self.c, self.bits, _ptr(self.data))
+
+
+def pack_codes(codes: torch.Tensor, bits: int, out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """codes: int32 CUDA [rows, c] -> packed uint8 [rows, row_bytes]."""
+    codes = codes.to(torch.int32).contiguous()
+    c = codes.shape[-1]
+    rows = codes.numel() // c
+    rb = row_bytes(c, bits)
+    if out is None:
+        out = torch.empty((rows, rb), dtype=torch.uint8, device=codes.device)
+    _check(load().aqd_pack_codes(_ptr(codes), rows, c, bits, _ptr(out), _stream(stream)), "aqd_pack_codes")
+    return out
+
+
+def unpack_codes(packed: torch.Tensor, c: int, bits: int, signed: bool = False, stream=None) -> torch.Tensor:
+    packed = packed.contiguous()
+    rb = row_bytes(c, bits)
+    rows = packed.numel() // rb
+    out = torch.empty((rows, c), dtype=torch.int32, device=packed.device)
+    _check(load().aqd_unpack_codes(_ptr(packed), rows, c, bits, int(signed), _ptr(out), _stream(stream)),
+           "aqd_unpack_codes")
+    return out
+
+
+# ------------------------------------------------------------------ parameters
+
+
+@dataclass
+class RequantParams:
+    m0: torch.Tensor | None      # int32 [levels, cout]
+    shift: torch.Tensor | None   # int8  [levels, cout]
+    bias: torch.Tensor | None    # int32 [levels, cout]
+    levels: int
+
+    @classmethod
+    def from_numpy(cls, m0, shift, bias, device="cuda"):
+        def t(a, dt):
+            return None if a is None else torch.as_tensor(a).to(dt).contiguous().to(device)
+        ref = m0 if m0 is not None else bias
+        return cls(t(m0, torch.int32), t(shift, torch.int8), t(bias, torch.int32), int(ref.shape[0]))
+
+    def c(self) -> _Requant:
+        return _Requant(_ptr(self.m0), _ptr(self.shift), _ptr(self.bias), self.levels)
+
+
+@dataclass
+class SkipParams:
+    c: torch.Tensor     # int32 [levels, cout]
+    d: torch.Tensor     # int8  [levels, cout]
+    upsample: int = 1
+    scale_main: int = 0
+
+    @classmethod
+    def from_numpy(cls, c, d, upsample=1, scale_main=0, device="cuda"):
+        return cls(torch.as_tensor(c).to(torch.int32).contiguous().to(device),
+                   torch.as_tensor(d).to(torch.int8).contiguous().to(device), upsample, scale_main)
+
+    def cs(self) -> _Skip:
+        return _Skip(_ptr(self.c), _ptr(self.d), self.upsample, self.scale_main)
+
+
+def quantize_multiplier(real: float) -> tuple[int, int]:
+    m0 = ctypes.c_int32()
+    sh = ctypes.c_int8()
+    _check(load().aqd_quantize_multiplier(float(real), ctypes.byref(m0), ctypes.byref(sh)), "aqd_quantize_multiplier")
+    return int(m0.value), int(sh.value)
+
+
+class ConvWeights:
+    """Prepared weights of one conv layer ([cout, kh, kw, cin] signed integers)."""
+
+    def __init__(self, w_codes: torch.Tensor, w_bits: int, w_format: int = W_TWOS, stream=None):
+        cout, kh, kw, cin = w_codes.shape
+        packed = pack_codes(w_codes.reshape(-1, cin), w_bits, stream=stream)
+        self._prepare(packed, cout, kh, kw, cin, w_bits, w_format, stream)
+
+    @classmethod
+    def from_packed(cls, packed: torch.Tensor, cout: int, kh: int, kw: int, cin: int, w_bits: int,
+                    w_format: int = W_TWOS, stream=None) -> "ConvWeights":
+        """packed: uint8 CUDA rows [cout*kh*kw, row_bytes(cin, w_bits)]."""
+        self = cls.__new__(cls)
+        self._prepare(packed.contiguous(), cout, kh, kw, cin, w_bits, w_format, stream)
+        return self
+
+    def _prepare(self, packed, cout, kh, kw, cin, w_bits, w_format, stream):
+        L = load()
+        nbytes = int(L.aqd_conv_weights_bytes(cout, kh, kw, cin))
+        if nbytes == 0:
+            raise ValueError("unsupported weight shape")
+        self.buf = torch.zeros(nbytes + 256, dtype=torch.uint8, device=packed.device)
+        off = (-self.buf.data_ptr()) % 256
+        self.prepared = self.buf[off:off + nbytes]
+        self.desc = _Weights(_ptr(self.prepared), cout, kh, kw, cin, w_bits, w_format)
+        _check(L.aqd_conv_prepare_weights(_ptr(packed), ctypes.byref(self.desc), _ptr(self.prepared), nbytes,
+                                          _stream(stream)), "aqd_conv_prepare_weights")
+        self._packed = packed  # kept alive until the stream has consumed it
+        self.cout, self.kh, self.kw, self.cin = cout, kh, kw, cin
+
+
+def conv_out_hw(h, w, kh, kw, stride, pad):
+    return (h + 2 * pad - kh) // stride + 1, (w + 2 * pad - kw) // stride + 1
+
+
+def conv_int(x: DTensor, w: ConvWeights, stride: int, pad: int, y: DTensor, *, level: int = 0,
+             rq: RequantParams | None = None, skip: DTensor | None = None, sp: SkipParams | None = None,
+             stream=None) -> DTensor:
+    xc, yc = x.ct(), y.ct()
+    rqc = rq.c() if rq is not None else None
+    skc = skip.ct() if skip is not None else None
+    spc = sp.cs() if sp is not None else None
+    _check(load().aqd_conv_int(ctypes.byref(xc), ctypes.byref(w.desc), stride, pad, level,
+                               ctypes.byref(rqc) if rqc is not None else None,
+                               ctypes.byref(skc) if skc is not None else None,
+                               ctypes.byref(spc) if spc is not None else None, ctypes.byref(yc), _stream(stream)),
+           "aqd_conv_int")
+    return y
+
+
+def conv_int_grouped(jobs, w: ConvWeights, stride: int, pad: int, *, rq: RequantParams | None = None,
+                     sp: SkipParams | None = None, stream=None):
+    """jobs: list of (x: DTensor, y: DTensor, skip: DTensor | None, level: int)."""
+    arr = (_Job * len(jobs))()
+    for i, (x, y, skip, level) in enumerate(jobs):
+        arr[i].x = x.ct()
+        arr[i].y = y.ct()
+        arr[i].skip = skip.ct() if skip is not None else _Tensor(0, 0, 0, 0, 0, None)
+        arr[i].level = level
+    rqc = rq.c() if rq is not None else None
+    spc = sp.cs() if sp is not None else None
+    _check(load().aqd_conv_int_grouped(arr, len(jobs), ctypes.byref(w.desc), stride, pad,
+                                       ctypes.byref(rqc) if rqc is not None else None,
+                                       ctypes.byref(spc) if spc is not None else None, _stream(stream)),
+           "aqd_conv_int_grouped")
+
+
+def requant(acc: DTensor, rq: RequantParams, y: DTensor, *, level: int = 0, stream=None) -> DTensor:
+    ac, yc, rqc = acc.ct(), y.ct(), rq.c()
+    _check(load().aqd_requant(ctypes.byref(ac), ctypes.byref(rqc), level, ctypes.byref(yc), _stream(stream)),
+           "aqd_requant")
+    return y
+
+
+def residual_add_int(a: DTensor, b: DTensor, sp: SkipParams, y: DTensor, *, rq: RequantParams | None = None,
+                     level: int = 0, stream=None) -> DTensor:
+    ac, bc, yc, spc = a.ct(), b.ct(), y.ct(), sp.cs()
+    rqc = rq.c() if rq is not None else None
+    _check(load().aqd_residual_add_int(ctypes.byref(ac), ctypes.byref(bc), ctypes.byref(spc),
+                                       ctypes.byref(rqc) if rqc is not None else None, level, ctypes.byref(yc),
+                                       _stream(stream)), "aqd_residual_add_int")
+    return y
+
+
+def maxpool_codes(x: DTensor, k: int, stride: int, pad: int, y: DTensor, stream=None) -> DTensor:
+    xc, yc = x.ct(), y.ct()
+    _check(load().aqd_maxpool_codes(ctypes.byref(xc), k, stride, pad, ctypes.byref(yc), _stream(stream)),
+           "aqd_maxpool_codes")
+    return y
+
+
+def device_status(stream=None) -> int:
+    code = ctypes.c_int32()
+    _check(load().aqd_device_status(_stream(stream), ctypes.byref(code)), "aqd_device_status")
+    return int(code.value)
+
+
+def set_conv_path(path: int) -> int:
+    return int(load().aqd_set_conv_path(path))
+
+
+def last_conv_path() -> int:
+    return int(load().aqd_last_conv_path())

@@ -1,0 +1,374 @@
+// aqd_api.cu -- the C ABI of libaqd (declared in include/aqd.h): argument validation,
+// kernel selection and launch. Every argument error is reported before any launch.
+#include <cuda_runtime.h>
+
+#include <climits>
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <string>
+
+#include "../../include/aqd.h"
+#include "common.cuh"
+#include "kernels.h"
+
+namespace aqd {
+
+static thread_local std::string g_last_error;
+static thread_local int32_t g_last_path = 0;
+static int32_t g_forced_path = 0;  // 0 auto, 1 tensor core, 2 direct
+
+__device__ uint32_t g_status_word;
+
+static aqd_status fail(aqd_status s, const std::string& msg) {
+  g_last_error = msg;
+  return s;
+}
+
+// Device address of the status word, looked up once per device.
+static uint32_t* status_ptr(std::string* err) {
+  static std::mutex mu;
+  static uint32_t* ptrs[64] = {nullptr};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    *err = "cudaGetDevice failed";
+    return nullptr;
+  }
+  std::lock_guard<std::mutex> lk(mu);
+  if (!ptrs[dev]) {
+    void* p = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&p, g_status_word);
+    if (e != cudaSuccess) {
+      *err = std::string("cudaGetSymbolAddress(status): ") + cudaGetErrorString(e);
+      return nullptr;
+    }
+    ptrs[dev] = static_cast<uint32_t*>(p);
+  }
+  return ptrs[dev];
+}
+
+WeightGeom weight_geom(int32_t cout, int32_t kh, int32_t kw, int32_t cin) {
+  WeightGeom g{};
+  g.cout = cout; g.kh = kh; g.kw = kw; g.cin = cin;
+  g.k_total = kh * kw * cin;
+  g.k_pad = (g.k_total + 127) / 128 * 128;
+  g.bn = cout <= 256 ? (cout + 15) / 16 * 16 : 256;
+  g.cout_pad = (cout + g.bn - 1) / g.bn * g.bn;
+  g.e4m3_bytes = (size_t)g.cout_pad * g.k_pad;
+  g.i16_offset = (g.e4m3_bytes + 255) / 256 * 256;
+  g.total_bytes = g.i16_offset + 2 * (size_t)cout * g.k_total;
+  return g;
+}
+
+static bool code_bits(int b) { return b == 2 || b == 3 || b == 4 || b == 8; }
+static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+static bool check_tensor(const aqd_tensor* t, bool allow32, const char* name, std::string* err) {
+  if (!t) { *err = std::string(name) + " is NULL"; return false; }
+  if (!t->data) { *err = std::string(name) + "->data is NULL"; return false; }
+  if (t->n <= 0 || t->h <= 0 || t->w <= 0 || t->c <= 0) { *err = std::string(name) + " has a non-positive dimension"; return false; }
+  if (!(code_bits(t->bits) || (allow32 && t->bits == 32))) { *err = std::string(name) + " has unsupported bits"; return false; }
+  if (row_bytes_of(t->c, t->bits) < 0) { *err = std::string(name) + ": channels must be a multiple of 32 at 2/3/4 bits"; return false; }
+  if (!aligned16(t->data)) { *err = std::string(name) + "->data must be 16-byte aligned"; return false; }
+  if ((int64_t)t->n * t->h * t->w >= (int64_t)INT_MAX) { *err = std::string(name) + " has too many pixels"; return false; }
+  return true;
+}
+
+static int64_t max_abs_weight(int w_bits, int w_format) {
+  return w_format == AQD_W_TWOS ? (1LL << (w_bits - 1)) : ((1LL << w_bits) - 1);
+}
+
+extern "C" {
+
+int64_t aqd_row_bytes(int32_t c, int32_t bits) { return row_bytes_of(c, bits); }
+
+const char* aqd_status_string(aqd_status s) {
+  switch (s) {
+    case AQD_OK: return "ok";
+    case AQD_ERR_INVALID: return "invalid argument";
+    case AQD_ERR_UNSUPPORTED: return "unsupported";
+    case AQD_ERR_CUDA: return "CUDA error";
+    case AQD_ERR_TIMEOUT: return "device wait timed out";
+    case AQD_ERR_DEVICE_CHECK: return "device check failed";
+  }
+  return "unknown status";
+}
+
+const char* aqd_last_error(void) { return g_last_error.c_str(); }
+
+// Eq. 8 with |c| < 2^31 and d = 31 + shift in [0, 62]: the largest d whose rounded c fits.
+aqd_status aqd_quantize_multiplier(double real, int32_t* m0, int8_t* shift) {
+  if (!m0 || !shift) return fail(AQD_ERR_INVALID, "null output pointer");
+  if (!std::isfinite(real)) return fail(AQD_ERR_INVALID, "real must be finite");
+  if (real == 0.0) { *m0 = 0; *shift = 0; return AQD_OK; }
+  const double mag = std::fabs(real);
+  int e = 0;
+  std::frexp(mag, &e);  // mag = f * 2^e, f in [0.5, 1)
+  // c = round(mag * 2^d) < 2^31 needs d <= 31 - e (and one less if rounding reaches 2^31)
+  int d = 31 - e;
+  if (d > 62) d = 62;
+  for (; d >= 0; --d) {
+    const double c = std::floor(std::ldexp(mag, d) + 0.5);
+    if (c < 2147483648.0) {
+      *m0 = (int32_t)(real < 0 ? -c : c);
+      *shift = (int8_t)(d - 31);
+      return AQD_OK;
+    }
+  }
+  return fail(AQD_ERR_INVALID, "|real| too large for a 31-bit multiplier");
+}
+
+aqd_status aqd_device_status(aqd_stream_t stream, int32_t* code) {
+  if (!code) return fail(AQD_ERR_INVALID, "code is NULL");
+  std::string err;
+  uint32_t* sp = status_ptr(&err);
+  if (!sp) return fail(AQD_ERR_CUDA, err);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint32_t v = 0;
+  cudaError_t e = cudaMemcpyAsync(&v, sp, sizeof(v), cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e == cudaSuccess && v != 0) {
+    e = cudaMemsetAsync(sp, 0, sizeof(uint32_t), st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  }
+  if (e != cudaSuccess) return fail(AQD_ERR_CUDA, std::string("device status: ") + cudaGetErrorString(e));
+  *code = (int32_t)v;
+  return AQD_OK;
+}
+
+int32_t aqd_set_conv_path(int32_t path) {
+  if (path < 0 || path > 2) return -1;
+  const int32_t old = g_forced_path;
+  g_forced_path = path;
+  return old;
+}
+
+int32_t aqd_last_conv_path(void) { return g_last_path; }
+
+aqd_status aqd_pack_codes(const int32_t* codes, int64_t rows, int32_t c, int32_t bits, void* out,
+                          aqd_stream_t stream) {
+  if (!code_bits(bits)) return fail(AQD_ERR_INVALID, "bits must be 2, 3, 4 or 8");
+  if (row_bytes_of(c, bits) < 0) return fail(AQD_ERR_INVALID, "channels must be a multiple of 32 at 2/3/4 bits");
+  if (rows < 0) return fail(AQD_ERR_INVALID, "rows < 0");
+  if (rows == 0) return AQD_OK;
+  if (!codes || !out) return fail(AQD_ERR_INVALID, "null pointer");
+  if (bits != 8 && !aligned16(out)) return fail(AQD_ERR_INVALID, "out must be 16-byte aligned");
+  std::string err;
+  int st = launch_pack(codes, rows, c, bits, static_cast<uint8_t*>(out), static_cast<cudaStream_t>(stream), &err);
+  return st ? fail((aqd_status)st, err) : AQD_OK;
+}
+
+aqd_status aqd_unpack_codes(const void* packed, int64_t rows, int32_t c, int32_t bits, int32_t is_signed,
+                            int32_t* out, aqd_stream_t stream) {
+  if (!code_bits(bits)) return fail(AQD_ERR_INVALID, "bits must be 2, 3, 4 or 8");
+  if (row_bytes_of(c, bits) < 0) return fail(AQD_ERR_INVALID, "channels must be a multiple of 32 at 2/3/4 bits");
+  if (rows < 0) return fail(AQD_ERR_INVALID, "rows < 0");
+  if (rows == 0) return AQD_OK;
+  if (!packed || !out) return fail(AQD_ERR_INVALID, "null pointer");
+  if (bits != 8 && !aligned16(packed)) return fail(AQD_ERR_INVALID, "packed must be 16-byte aligned");
+  std::string err;
+  int st = launch_unpack(static_cast<const uint8_t*>(packed), rows, c, bits, is_signed, out,
+                         static_cast<cudaStream_t>(stream), &err);
+  return st ? fail((aqd_status)st, err) : AQD_OK;
+}
+
+size_t aqd_conv_weights_bytes(int32_t cout, int32_t kh, int32_t kw, int32_t cin) {
+  if (cout <= 0 || kh <= 0 || kw <= 0 || cin <= 0) return 0;
+  if ((int64_t)kh * kw * cin > (1 << 24)) return 0;
+  return weight_geom(cout, kh, kw, cin).total_bytes;
+}
+
+static bool check_weights(const aqd_conv_weights* w, std::string* err) {
+  if (!w) { *err = "weights descriptor is NULL"; return false; }
+  if (w->cout <= 0 || w->kh <= 0 || w->kw <= 0 || w->cin <= 0) { *err = "weights have a non-positive dimension"; return false; }
+  if (!code_bits(w->w_bits)) { *err = "w_bits must be 2, 3, 4 or 8"; return false; }
+  if (w->w_format != AQD_W_TWOS && w->w_format != AQD_W_ODD) { *err = "unknown w_format"; return false; }
+  if (row_bytes_of(w->cin, w->w_bits) < 0) { *err = "weight rows: cin must be a multiple of 32 at 2/3/4 bits"; return false; }
+  if ((int64_t)w->kh * w->kw * w->cin > (1 << 24)) { *err = "kernel too large"; return false; }
+  return true;
+}
+
+aqd_status aqd_conv_prepare_weights(const void* w_packed, const aqd_conv_weights* w, void* w_prepared,
+                                    size_t bytes, aqd_stream_t stream) {
+  std::string err;
+  if (!check_weights(w, &err)) return fail(AQD_ERR_INVALID, err);
+  if (!w_packed || !w_prepared) return fail(AQD_ERR_INVALID, "null pointer");
+  if ((reinterpret_cast<uintptr_t>(w_prepared) & 255) != 0) return fail(AQD_ERR_INVALID, "w_prepared must be 256-byte aligned");
+  const WeightGeom g = weight_geom(w->cout, w->kh, w->kw, w->cin);
+  if (bytes < g.total_bytes) return fail(AQD_ERR_INVALID, "w_prepared buffer too small");
+  int st = launch_prepare_weights(static_cast<const uint8_t*>(w_packed), w->w_bits, w->w_format, g,
+                                  static_cast<uint8_t*>(w_prepared), static_cast<cudaStream_t>(stream), &err);
+  return st ? fail((aqd_status)st, err) : AQD_OK;
+}
+
+aqd_status aqd_conv_int_grouped(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
+                                int32_t stride, int32_t pad, const aqd_requant_params* rq,
+                                const aqd_skip_params* sp, aqd_stream_t stream) {
+  std::string err;
+  if (!jobs || njobs <= 0 || njobs > kMaxJobs) return fail(AQD_ERR_INVALID, "njobs must be 1..8");
+  if (!check_weights(w, &err)) return fail(AQD_ERR_INVALID, err);
+  if (!w->data || (reinterpret_cast<uintptr_t>(w->data) & 255) != 0)
+    return fail(AQD_ERR_INVALID, "w->data must be a 256-byte aligned prepared-weights buffer");
+  if (stride <= 0 || pad < 0) return fail(AQD_ERR_INVALID, "stride must be > 0 and pad >= 0");
+  const int out_bits = jobs[0].y.bits;
+  const bool has_skip = jobs[0].skip.data != nullptr;
+  if (!(code_bits(out_bits) || out_bits == 32)) return fail(AQD_ERR_INVALID, "y.bits must be 2, 3, 4, 8 or 32");
+  if (out_bits != 32 && (!rq || !rq->m0 || !rq->shift)) return fail(AQD_ERR_INVALID, "code outputs need rq->m0 and rq->shift");
+  if (rq && rq->levels <= 0) return fail(AQD_ERR_INVALID, "rq->levels must be > 0");
+  if (has_skip) {
+    if (!sp || !sp->c || !sp->d) return fail(AQD_ERR_INVALID, "a skip needs sp->c and sp->d");
+    if (sp->upsample != 1 && sp->upsample != 2) return fail(AQD_ERR_INVALID, "sp->upsample must be 1 or 2");
+    if (sp->scale_main != 0 && sp->scale_main != 1) return fail(AQD_ERR_INVALID, "sp->scale_main must be 0 or 1");
+    if (!rq) return fail(AQD_ERR_INVALID, "a skip needs rq (its level count indexes sp's tables)");
+  }
+  ConvArgs a{};
+  a.njobs = njobs;
+  a.cin = w->cin; a.cout = w->cout; a.kh = w->kh; a.kw = w->kw; a.stride = stride; a.pad = pad;
+  a.x_bits = jobs[0].x.bits;
+  a.out_bits = out_bits;
+  a.skip_bits = has_skip ? jobs[0].skip.bits : 0;
+  for (int j = 0; j < njobs; ++j) {
+    const aqd_conv_job& jb = jobs[j];
+    const std::string nm = "jobs[" + std::to_string(j) + "]";
+    if (!check_tensor(&jb.x, false, (nm + ".x").c_str(), &err)) return fail(AQD_ERR_INVALID, err);
+    if (!check_tensor(&jb.y, true, (nm + ".y").c_str(), &err)) return fail(AQD_ERR_INVALID, err);
+    if (jb.x.c != w->cin) return fail(AQD_ERR_INVALID, nm + ".x.c != weights cin");
+    if (jb.x.bits != a.x_bits || jb.y.bits != out_bits) return fail(AQD_ERR_INVALID, nm + ": all jobs must share x.bits and y.bits");
+    const int ho = (jb.x.h + 2 * pad - w->kh) / stride + 1;
+    const int wo = (jb.x.w + 2 * pad - w->kw) / stride + 1;
+    if (jb.x.h + 2 * pad < w->kh || jb.x.w + 2 * pad < w->kw || ho <= 0 || wo <= 0)
+      return fail(AQD_ERR_INVALID, nm + ": kernel larger than the padded input");
+    if (jb.y.n != jb.x.n || jb.y.h != ho || jb.y.w != wo || jb.y.c != w->cout)
+      return fail(AQD_ERR_INVALID, nm + ".y shape does not match the convolution output");
+    if (rq && (jb.level < 0 || jb.level >= rq->levels)) return fail(AQD_ERR_INVALID, nm + ".level out of range");
+    if (!rq && jb.level != 0) return fail(AQD_ERR_INVALID, nm + ".level must be 0 without rq");
+    if ((jb.skip.data != nullptr) != has_skip) return fail(AQD_ERR_INVALID, "all jobs must agree on having a skip");
+    ConvJobDev& d = a.jobs[j];
+    d.x = static_cast<const uint8_t*>(jb.x.data);
+    d.y = static_cast<uint8_t*>(jb.y.data);
+    d.n = jb.x.n; d.h = jb.x.h; d.w = jb.x.w; d.ho = ho; d.wo = wo;
+    d.level = jb.level;
+    d.m_total = jb.x.n * ho * wo;
+    if (has_skip) {
+      if (!check_tensor(&jb.skip, true, (nm + ".skip").c_str(), &err)) return fail(AQD_ERR_INVALID, err);
+      if (jb.skip.bits != a.skip_bits) return fail(AQD_ERR_INVALID, "all skips must share bits");
+      const int up = sp->upsample;
+      if (jb.skip.n != jb.x.n || jb.skip.c != w->cout || jb.skip.h < (ho + up - 1) / up || jb.skip.w < (wo + up - 1) / up)
+        return fail(AQD_ERR_INVALID, nm + ".skip shape does not cover the output");
+      d.skip = static_cast<const uint8_t*>(jb.skip.data);
+      d.skip_h = jb.skip.h; d.skip_w = jb.skip.w;
+    }
+  }
+  a.x_row_bytes = row_bytes_of(a.cin, a.x_bits);
+  a.y_row_bytes = row_bytes_of(a.cout, out_bits);
+  a.skip_row_bytes = has_skip ? row_bytes_of(a.cout, a.skip_bits) : 0;
+  a.m0 = rq ? rq->m0 : nullptr;
+  a.shift = rq ? rq->shift : nullptr;
+  a.bias = rq ? rq->bias : nullptr;
+  a.has_skip = has_skip;
+  if (has_skip) { a.skip_c = sp->c; a.skip_d = sp->d; a.upsample = sp->upsample; a.scale_main = sp->scale_main; }
+  else { a.upsample = 1; }
+  const WeightGeom g = weight_geom(w->cout, w->kh, w->kw, w->cin);
+  a.w_e4m3 = static_cast<const uint8_t*>(w->data);
+  a.w_i16 = reinterpret_cast<const int16_t*>(static_cast<const uint8_t*>(w->data) + g.i16_offset);
+  a.cout_pad = g.cout_pad; a.k_total = g.k_total; a.k_pad = g.k_pad; a.bn = g.bn;
+  a.status = status_ptr(&err);
+  if (!a.status) return fail(AQD_ERR_CUDA, err);
+
+  // kernel choice: tensor cores when the FP32 sum is exact, else CUDA cores (int32)
+  const int64_t max_a = (1LL << a.x_bits) - 1;
+  const int64_t max_w = max_abs_weight(w->w_bits, w->w_format);
+  const int64_t bound = (int64_t)g.k_total * max_a * max_w;
+  const bool tc_ok = a.x_bits <= 4 && max_w <= 15 && (a.cin % 32) == 0 && bound < (1LL << 24);
+  const bool direct_ok = bound < (1LL << 31);
+  int path = tc_ok ? 1 : 2;
+  if (g_forced_path == 1 && tc_ok) path = 1;
+  if (g_forced_path == 2) path = 2;
+  if (path == 2 && !direct_ok) return fail(AQD_ERR_UNSUPPORTED, "accumulator bound exceeds int32");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int rc = path == 1 ? launch_conv_tc(a, st, &err) : launch_conv_direct(a, st, &err);
+  if (rc) return fail((aqd_status)rc, err);
+  g_last_path = path;
+  return AQD_OK;
+}
+
+aqd_status aqd_conv_int(const aqd_tensor* x, const aqd_conv_weights* w, int32_t stride, int32_t pad,
+                        int32_t level, const aqd_requant_params* rq, const aqd_tensor* skip,
+                        const aqd_skip_params* sp, aqd_tensor* y, aqd_stream_t stream) {
+  if (!x || !y) return fail(AQD_ERR_INVALID, "x and y must not be NULL");
+  aqd_conv_job job{};
+  job.x = *x;
+  job.y = *y;
+  if (skip) {
+    job.skip = *skip;
+    if (!skip->data) return fail(AQD_ERR_INVALID, "skip->data is NULL");
+  }
+  job.level = level;
+  return aqd_conv_int_grouped(&job, 1, w, stride, pad, rq, sp, stream);
+}
+
+static aqd_status elementwise(const aqd_tensor* a, const aqd_tensor* b, const aqd_skip_params* sp,
+                              const aqd_requant_params* rq, int32_t level, aqd_tensor* y, aqd_stream_t stream) {
+  std::string err;
+  if (!check_tensor(a, true, "a", &err)) return fail(AQD_ERR_INVALID, err);
+  if (!check_tensor(y, true, "y", &err)) return fail(AQD_ERR_INVALID, err);
+  if (y->n != a->n || y->h != a->h || y->w != a->w || y->c != a->c) return fail(AQD_ERR_INVALID, "y shape must equal a's");
+  if (y->bits != 32 && (!rq || !rq->m0 || !rq->shift)) return fail(AQD_ERR_INVALID, "code outputs need rq->m0 and rq->shift");
+  if (rq && (rq->levels <= 0 || level < 0 || level >= rq->levels)) return fail(AQD_ERR_INVALID, "level out of range");
+  if (!rq && level != 0) return fail(AQD_ERR_INVALID, "level must be 0 without rq");
+  EltArgs e{};
+  e.a = static_cast<const uint8_t*>(a->data); e.a_bits = a->bits; e.a_row_bytes = row_bytes_of(a->c, a->bits);
+  e.y = static_cast<uint8_t*>(y->data); e.y_bits = y->bits; e.y_row_bytes = row_bytes_of(y->c, y->bits);
+  e.n = a->n; e.h = a->h; e.w = a->w; e.c = a->c; e.level = level;
+  e.m0 = rq ? rq->m0 : nullptr; e.shift = rq ? rq->shift : nullptr; e.bias = rq ? rq->bias : nullptr;
+  e.upsample = 1;
+  if (b) {
+    if (!check_tensor(b, true, "b", &err)) return fail(AQD_ERR_INVALID, err);
+    if (!sp || !sp->c || !sp->d) return fail(AQD_ERR_INVALID, "sp with c and d is required");
+    if (sp->upsample != 1 && sp->upsample != 2) return fail(AQD_ERR_INVALID, "sp->upsample must be 1 or 2");
+    if (sp->scale_main != 0 && sp->scale_main != 1) return fail(AQD_ERR_INVALID, "sp->scale_main must be 0 or 1");
+    const int up = sp->upsample;
+    if (b->n != a->n || b->c != a->c || b->h < (a->h + up - 1) / up || b->w < (a->w + up - 1) / up)
+      return fail(AQD_ERR_INVALID, "b shape does not cover a");
+    e.b = static_cast<const uint8_t*>(b->data); e.b_bits = b->bits; e.b_row_bytes = row_bytes_of(b->c, b->bits);
+    e.b_h = b->h; e.b_w = b->w;
+    e.skip_c = sp->c; e.skip_d = sp->d; e.upsample = up; e.scale_main = sp->scale_main; e.has_skip = 1;
+  }
+  int st = launch_elementwise(e, static_cast<cudaStream_t>(stream), &err);
+  return st ? fail((aqd_status)st, err) : AQD_OK;
+}
+
+aqd_status aqd_requant(const aqd_tensor* acc, const aqd_requant_params* rq, int32_t level, aqd_tensor* y,
+                       aqd_stream_t stream) {
+  if (!acc || acc->bits != 32) return fail(AQD_ERR_INVALID, "acc must be an int32 tensor");
+  if (!rq) return fail(AQD_ERR_INVALID, "rq is NULL");
+  return elementwise(acc, nullptr, nullptr, rq, level, y, stream);
+}
+
+aqd_status aqd_residual_add_int(const aqd_tensor* a, const aqd_tensor* b, const aqd_skip_params* sp,
+                                const aqd_requant_params* rq, int32_t level, aqd_tensor* y, aqd_stream_t stream) {
+  if (!b) return fail(AQD_ERR_INVALID, "b is NULL");
+  return elementwise(a, b, sp, rq, level, y, stream);
+}
+
+aqd_status aqd_maxpool_codes(const aqd_tensor* x, int32_t k, int32_t stride, int32_t pad, aqd_tensor* y,
+                             aqd_stream_t stream) {
+  std::string err;
+  if (!check_tensor(x, false, "x", &err)) return fail(AQD_ERR_INVALID, err);
+  if (!check_tensor(y, false, "y", &err)) return fail(AQD_ERR_INVALID, err);
+  if (k <= 0 || stride <= 0 || pad < 0 || pad >= k) return fail(AQD_ERR_INVALID, "need k > 0, stride > 0, 0 <= pad < k");
+  const int ho = (x->h + 2 * pad - k) / stride + 1, wo = (x->w + 2 * pad - k) / stride + 1;
+  if (x->h + 2 * pad < k || x->w + 2 * pad < k) return fail(AQD_ERR_INVALID, "window larger than the padded input");
+  if (y->n != x->n || y->h != ho || y->w != wo || y->c != x->c || y->bits != x->bits)
+    return fail(AQD_ERR_INVALID, "y shape does not match the pooled output");
+  PoolArgs p{};
+  p.x = static_cast<const uint8_t*>(x->data); p.y = static_cast<uint8_t*>(y->data);
+  p.n = x->n; p.h = x->h; p.w = x->w; p.c = x->c; p.bits = x->bits; p.ho = ho; p.wo = wo;
+  p.k = k; p.stride = stride; p.pad = pad; p.row_bytes = row_bytes_of(x->c, x->bits);
+  int st = launch_maxpool(p, static_cast<cudaStream_t>(stream), &err);
+  return st ? fail((aqd_status)st, err) : AQD_OK;
+}
+
+}  // extern "C"
+}  // namespace aqd

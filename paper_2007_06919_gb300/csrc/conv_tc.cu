@@ -1,0 +1,613 @@
+// conv_tc.cu -- AQD's integer convolution (Eq. 4) as a persistent tcgen05 implicit GEMM
+// on sm_103a, with the integer epilogue (Eq. 6 bias, Eq. 7/8 skip, Eq. 2 rescale + clip)
+// fused after the TMEM accumulator.
+//
+// Exact integer arithmetic on the FP8 tensor pipe. sm_103a has no integer tcgen05 MMA
+// (kind::i8), so codes are embedded in E4M3 bit patterns: the raw byte n (0..15) of an
+// E4M3 value is exactly n * 2^-9 (0..7 subnormal, 8..15 exponent field 1), and a signed
+// weight |w| <= 15 is the same byte with the sign bit set. Every product is an integer
+// times 2^-18, and the FP32 accumulator holds the exact integer sum times 2^-18 as long as
+// K * max|x| * max|w| < 2^24, which the host checks before choosing this kernel.
+//
+// Per CTA (one per SM, persistent over tiles of 128 output pixels x BN channels):
+//   warps 0-3  epilogue: tcgen05.ld of the accumulator, integer epilogue, bit-pack, store
+//   warp  4    TMEM allocation + one thread issuing tcgen05.mma (kind::f8f6f4, M=128)
+//   warp  5    one thread loading prepared weights with TMA (cp.async.bulk.tensor, SW128)
+//   warps 6-9  activation producers: im2col gather of packed k-bit codes with cp.async
+//              (zero-fill = the padding code 0), unpack to E4M3 bytes, store into the
+//              128B-swizzled K-major operand layout, signal an mbarrier
+// Stages of 128 K-bytes (one 128B swizzle atom) circulate between producers and the MMA
+// thread; two TMEM accumulators let the epilogue of tile i overlap the MMAs of tile i+1.
+// Every wait is bounded: on expiry the CTA latches kStatusTimeout and unwinds.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cstdio>
+#include <mutex>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace aqd {
+namespace tc {
+
+constexpr int BM = 128;            // output pixels per tile (= TMEM lanes)
+constexpr int BK = 128;            // K bytes per stage
+constexpr int kWarpMma = 4;
+constexpr int kWarpTma = 5;
+constexpr int kWarpProd0 = 6;
+constexpr int kProdWarps = 4;
+constexpr int kThreads = (kWarpProd0 + kProdWarps) * 32;  // 320
+constexpr int kMaxStages = 8;
+constexpr int kDepth = 3;          // cp.async chunks in flight per producer thread
+constexpr uint64_t kTimeoutNs = 1000000000ull;  // 1 s per wait
+
+struct Params {
+  ConvJobDev jobs[kMaxJobs];
+  int32_t njobs, total_tiles, n_tiles, num_kchunks;
+  int32_t cin, cout, kh, kw, stride, pad, k_total;
+  int32_t out_bits, skip_bits;
+  int64_t x_row_bytes, y_row_bytes, skip_row_bytes;
+  const int32_t* m0;
+  const int8_t* shift;
+  const int32_t* bias;
+  const int32_t* skip_c;
+  const int8_t* skip_d;
+  int32_t upsample, scale_main, has_skip;
+  int32_t bn, stages, stg_stride, tmem_cols;
+  uint32_t off_b, off_stg, off_epi, off_bar;
+  uint32_t* status;
+};
+
+// ---------------------------------------------------------------- PTX wrappers
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ uint64_t globaltimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count));
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  uint64_t st;
+  asm volatile("mbarrier.arrive.shared::cta.b64 %0, [%1];" : "=l"(st) : "r"(bar) : "memory");
+  (void)st;
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  uint64_t st;
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 %0, [%1], %2;"
+               : "=l"(st) : "r"(bar), "r"(bytes) : "memory");
+  (void)st;
+}
+__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
+  return ok != 0;
+}
+
+// Bounded wait: false if the deadline passed or another role aborted.
+__device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+  if (mbar_try(bar, parity)) return true;
+  uint64_t deadline = 0;
+  for (uint32_t spin = 1;; ++spin) {
+    if (mbar_try(bar, parity)) return true;
+    if ((spin & 63) == 0) {
+      if (*abort_flag) return false;
+      uint64_t now = globaltimer();
+      if (deadline == 0) deadline = now + kTimeoutNs;
+      else if (now > deadline) return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void fail(volatile int* abort_flag, uint32_t* status) {
+  *abort_flag = 1;
+  atomicCAS(status, 0u, (uint32_t)kStatusTimeout);
+}
+
+__device__ __forceinline__ void fence_proxy_async() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void fence_barrier_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void named_bar(int id, int n) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+
+template <int kBytes>
+__device__ __forceinline__ void cp_async(uint32_t dst, const void* src, bool ok) {
+  const uint32_t n = ok ? kBytes : 0;  // 0 source bytes = zero fill
+  if constexpr (kBytes == 16)
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(n) : "memory");
+  else if constexpr (kBytes == 8)
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;" ::"r"(dst), "l"(src), "r"(n) : "memory");
+  else
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(dst), "l"(src), "r"(n) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];"
+      ::"r"(dst), "l"((uint64_t)map), "r"(x), "r"(y), "r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// SW128 K-major shared-memory matrix descriptor (tcgen05 format): start address >> 4,
+// leading byte offset 16 (unused for swizzled K-major), stride byte offset 1024 between
+// 8-row groups, descriptor version 1, swizzle mode 2 = 128B.
+__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
+  uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)1 << 16;
+  d |= (uint64_t)(1024 >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+// Instruction descriptor, kind::f8f6f4: D=F32, A=B=E4M3, both K-major, N>>3, M>>4.
+__device__ __forceinline__ uint32_t idesc_e4m3(int n) {
+  return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_e4m3(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}"
+      ::"r"(d_tmem), "l"(a), "l"(b), "r"(idesc), "r"(acc) : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
+               ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
+// ---------------------------------------------------------------- tile bookkeeping
+
+struct TileInfo {
+  int job, mt, nt;
+};
+__device__ __forceinline__ TileInfo tile_info(const Params& p, int t) {
+  int j = 0;
+#pragma unroll 1
+  while (j + 1 < p.njobs && t >= p.jobs[j + 1].tile_begin) ++j;
+  int local = t - p.jobs[j].tile_begin;
+  TileInfo ti;
+  ti.job = j;
+  ti.mt = local / p.n_tiles;
+  ti.nt = local - ti.mt * p.n_tiles;
+  return ti;
+}
+
+// ---------------------------------------------------------------- the kernel
+
+template <int kXBits>
+__global__ void __launch_bounds__(kThreads, 1)
+conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ Params p) {
+  constexpr int kGB = 4 * kXBits;  // bytes of one 32-channel input group
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t s_a = sbase;
+  const uint32_t s_b = sbase + p.off_b;
+  uint8_t* stg = smem + p.off_stg;
+  EpiChan* epi = reinterpret_cast<EpiChan*>(smem + p.off_epi);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + p.off_bar);
+  // barrier slots: full[0..S), empty[0..S), tfull[2], tempty[2], final
+  const int S = p.stages;
+  const uint32_t b_full = smem_u32(bars);
+  const uint32_t b_empty = b_full + 8 * S;
+  const uint32_t b_tfull = b_empty + 8 * S;
+  const uint32_t b_tempty = b_tfull + 16;
+  const uint32_t b_final = b_tempty + 16;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * S + 5);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x / 32;
+  const int lane = threadIdx.x % 32;
+  const int BN = p.bn;
+  const uint32_t stage_b_bytes = (uint32_t)BN * BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(b_full + 8 * s, kProdWarps * 32 + 1);
+      mbar_init(b_empty + 8 * s, 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(b_tfull + 8 * b, 1);
+      mbar_init(b_tempty + 8 * b, 4 * 32);
+    }
+    mbar_init(b_final, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == kWarpMma) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
+                 ::"r"(smem_u32(tmem_slot)), "r"(p.tmem_cols) : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  if (warp == kWarpTma && lane == 0)
+    asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmap_w) : "memory");
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int nk = p.num_kchunks;
+  const int first_tile = blockIdx.x;
+  const int tile_stride = gridDim.x;
+
+  if (warp == kWarpMma) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      const uint32_t idesc = idesc_e4m3(BN);
+      uint32_t it = 0, lt = 0;
+      bool ok = true;
+      for (int t = first_tile; t < p.total_tiles && ok; t += tile_stride, ++lt) {
+        const uint32_t buf = lt & 1;
+        if (!mbar_wait(b_tempty + 8 * buf, ((lt >> 1) & 1) ^ 1, abort_flag)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + buf * (uint32_t)BN;
+        for (int q = 0; q < nk; ++q, ++it) {
+          const uint32_t s = it % S, ph = (it / S) & 1;
+          if (!mbar_wait(b_full + 8 * s, ph, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t a0 = s_a + s * (BM * BK);
+          const uint32_t b0 = s_b + s * stage_b_bytes;
+#pragma unroll
+          for (int kk = 0; kk < BK / 32; ++kk)
+            mma_e4m3(d_tmem, sdesc_sw128(a0 + 32 * kk), sdesc_sw128(b0 + 32 * kk), idesc,
+                     (q > 0 || kk > 0) ? 1u : 0u);
+          mma_commit(b_empty + 8 * s);
+        }
+        if (ok) mma_commit(b_tfull + 8 * buf);
+      }
+      if (!ok) fail(abort_flag, p.status);
+      // drain: every MMA issued above has completed once this barrier flips
+      mma_commit(b_final);
+      if (!mbar_wait(b_final, 0, abort_flag)) fail(abort_flag, p.status);
+    }
+  } else if (warp == kWarpTma) {
+    // ------------------------------------------------------------ weight loader (TMA)
+    if (lane == 0) {
+      uint32_t it = 0;
+      bool ok = true;
+      for (int t = first_tile; t < p.total_tiles && ok; t += tile_stride) {
+        const TileInfo ti = tile_info(p, t);
+        for (int q = 0; q < nk; ++q, ++it) {
+          const uint32_t s = it % S, ph = (it / S) & 1;
+          if (!mbar_wait(b_empty + 8 * s, ph ^ 1, abort_flag)) { ok = false; break; }
+          mbar_arrive_expect_tx(b_full + 8 * s, stage_b_bytes);
+          tma_load_2d(s_b + s * stage_b_bytes, &tmap_w, q * BK, ti.nt * BN, b_full + 8 * s);
+        }
+      }
+      if (!ok) fail(abort_flag, p.status);
+    }
+  } else if (warp >= kWarpProd0) {
+    // ------------------------------------------------------------ activation producers
+    const int row = threadIdx.x - kWarpProd0 * 32;  // 0..127: tile row owned by this thread
+    const uint32_t stg_row = smem_u32(stg) + row * p.stg_stride;
+    const uint32_t stg_slot_bytes = (uint32_t)BM * p.stg_stride;
+    int my_tiles = 0;
+    for (int t = first_tile; t < p.total_tiles; t += tile_stride) ++my_tiles;
+    const int total_chunks = my_tiles * nk;
+
+    // issue cursor
+    int i_tile = first_tile, i_q = 0, issued = 0;
+    const uint8_t* xbase = nullptr;
+    int hb = 0, wb = 0, H = 1, W = 1;
+    bool rvalid = false;
+    int tr = 0, ts = 0, tc0 = 0;  // tap state of the next 32-channel group
+    const uint8_t* xdummy = p.jobs[0].x;
+
+    auto issue = [&]() {
+      if (i_q == 0) {
+        const TileInfo ti = tile_info(p, i_tile);
+        const ConvJobDev& jb = p.jobs[ti.job];
+        const int m = ti.mt * BM + row;
+        rvalid = m < jb.m_total;
+        const int mm = rvalid ? m : 0;
+        const int hw = jb.ho * jb.wo;
+        const int img = mm / hw;
+        const int rem = mm - img * hw;
+        const int ho = rem / jb.wo, wo = rem - (rem / jb.wo) * jb.wo;
+        hb = ho * p.stride - p.pad;
+        wb = wo * p.stride - p.pad;
+        H = jb.h;
+        W = jb.w;
+        xbase = jb.x + (int64_t)img * jb.h * jb.w * p.x_row_bytes;
+        tr = 0; ts = 0; tc0 = 0;
+      }
+      const uint32_t slot = stg_row + (uint32_t)(issued % kDepth) * stg_slot_bytes;
+#pragma unroll
+      for (int g = 0; g < BK / 32; ++g) {
+        const int k0 = i_q * BK + 32 * g;
+        bool ok = false;
+        const uint8_t* src = xdummy;
+        if (k0 < p.k_total) {
+          const int hi = hb + tr, wi = wb + ts;
+          ok = rvalid && hi >= 0 && hi < H && wi >= 0 && wi < W;
+          if (ok) src = xbase + ((int64_t)hi * W + wi) * p.x_row_bytes + (tc0 >> 5) * kGB;
+          tc0 += 32;
+          if (tc0 == p.cin) { tc0 = 0; if (++ts == p.kw) { ts = 0; ++tr; } }
+        }
+        const uint32_t dst = slot + g * kGB;
+        if constexpr (kGB == 8) {
+          cp_async<8>(dst, src, ok);
+        } else if constexpr (kGB == 16) {
+          cp_async<16>(dst, src, ok);
+        } else {  // 12 bytes: three 4-byte copies
+          cp_async<4>(dst, src, ok);
+          cp_async<4>(dst + 4, src + 4, ok);
+          cp_async<4>(dst + 8, src + 8, ok);
+        }
+      }
+      ++issued;
+      if (++i_q == nk) { i_q = 0; i_tile += tile_stride; }
+    };
+
+    for (int d = 0; d < kDepth; ++d) {
+      if (issued < total_chunks) issue();
+      cp_async_commit();
+    }
+    bool ok = true;
+    for (int c = 0; c < total_chunks; ++c) {
+      cp_async_wait<kDepth - 1>();
+      const uint32_t s = c % S, ph = (c / S) & 1;
+      if (!mbar_wait(b_empty + 8 * s, ph ^ 1, abort_flag)) { ok = false; break; }
+      // unpack this thread's row: 4 groups of 32 codes -> 128 E4M3 bytes (raw byte = code)
+      const uint8_t* src = stg + (size_t)(c % kDepth) * BM * p.stg_stride + (size_t)row * p.stg_stride;
+      uint32_t words[4 * kXBits];
+#pragma unroll
+      for (int i = 0; i < kXBits; ++i) {
+        const uint4 v = reinterpret_cast<const uint4*>(src)[i];
+        words[4 * i + 0] = v.x; words[4 * i + 1] = v.y; words[4 * i + 2] = v.z; words[4 * i + 3] = v.w;
+      }
+      uint8_t* arow = smem + (size_t)s * (BM * BK) + (size_t)row * BK;
+#pragma unroll
+      for (int g = 0; g < 4; ++g) {
+        uint32_t o[8];
+        unpack_group_bytes<kXBits>(words + g * kXBits, o);
+        const int j0 = (2 * g) ^ (row & 7), j1 = (2 * g + 1) ^ (row & 7);
+        *reinterpret_cast<uint4*>(arow + 16 * j0) = make_uint4(o[0], o[1], o[2], o[3]);
+        *reinterpret_cast<uint4*>(arow + 16 * j1) = make_uint4(o[4], o[5], o[6], o[7]);
+      }
+      fence_proxy_async();
+      mbar_arrive(b_full + 8 * s);
+      if (issued < total_chunks) issue();
+      cp_async_commit();
+    }
+    cp_async_wait<0>();
+    if (!ok) fail(abort_flag, p.status);
+  } else {
+    // ------------------------------------------------------------ epilogue (warps 0-3)
+    const int e = threadIdx.x;  // tile row = TMEM lane
+    const uint32_t lane_base = tmem_base + ((uint32_t)(warp * 32) << 16);
+    uint32_t lt = 0;
+    bool ok = true;
+    const int out_bits = p.out_bits;
+    for (int t = first_tile; t < p.total_tiles; t += tile_stride, ++lt) {
+      const TileInfo ti = tile_info(p, t);
+      const ConvJobDev& jb = p.jobs[ti.job];
+      named_bar(1, 128);
+      for (int col = e; col < 256; col += 128) {
+        const int ch = ti.nt * BN + col;
+        EpiChan ec{};
+        if (col < BN && ch < p.cout) {
+          const int64_t idx = (int64_t)jb.level * p.cout + ch;
+          ec.bias = p.bias ? p.bias[idx] : 0;
+          if (out_bits != 32) { ec.m0 = p.m0[idx]; ec.r = (int8_t)(31 + p.shift[idx]); }
+          if (p.has_skip) { ec.c = p.skip_c[idx]; ec.d = p.skip_d[idx]; }
+        }
+        epi[col] = ec;
+      }
+      named_bar(1, 128);
+      const uint32_t buf = lt & 1;
+      if (!mbar_wait(b_tfull + 8 * buf, (lt >> 1) & 1, abort_flag)) { ok = false; break; }
+      tc_fence_after();
+
+      const int m = ti.mt * BM + e;
+      const bool valid = m < jb.m_total;
+      const int mm = valid ? m : 0;
+      const int hw = jb.ho * jb.wo;
+      const int img = mm / hw;
+      const int rem = mm - img * hw;
+      const int ho = rem / jb.wo, wo = rem - (rem / jb.wo) * jb.wo;
+      uint8_t* yrow = jb.y + (int64_t)mm * p.y_row_bytes;
+      const uint8_t* srow = nullptr;
+      if (p.has_skip) {
+        const int sh = ho / p.upsample, sw = wo / p.upsample;
+        srow = jb.skip + (((int64_t)img * jb.skip_h + sh) * jb.skip_w + sw) * p.skip_row_bytes;
+      }
+      const uint32_t tcol = buf * (uint32_t)BN;
+      for (int g0 = 0; g0 < BN; g0 += 32) {
+        const int ncols = (BN - g0) < 32 ? (BN - g0) : 32;  // warp-uniform
+        uint32_t v[32];
+        uint32_t r16[16];
+        __syncwarp();
+        tmem_ld16(lane_base + tcol + g0, r16);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = r16[i];
+        if (ncols == 32) tmem_ld16(lane_base + tcol + g0 + 16, r16);
+        tmem_wait_ld();
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[16 + i] = (ncols == 32) ? r16[i] : 0u;
+        if (valid) {
+        const int ch0 = ti.nt * BN + g0;
+        int32_t sk[32];
+        if (p.has_skip) {
+          if (p.skip_bits == 32) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) sk[i] = (i < ncols && ch0 + i < p.cout) ? reinterpret_cast<const int32_t*>(srow)[ch0 + i] : 0;
+          } else {
+            unpack_group_vals(srow + (ch0 >> 5) * group_bytes(p.skip_bits), p.skip_bits, false, sk);
+          }
+        }
+        int32_t out[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const float f = __uint_as_float(v[i]) * 262144.0f;  // exact integer (x 2^18)
+          const int64_t acc = (int64_t)__float2int_rn(f);
+          const EpiChan ec = epi[g0 + i];
+          out[i] = p.has_skip ? epilogue<true>(acc, sk[i], ec, p.scale_main, out_bits)
+                              : epilogue<false>(acc, 0, ec, p.scale_main, out_bits);
+        }
+        if (out_bits == 32) {
+          int32_t* yr = reinterpret_cast<int32_t*>(yrow);
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (i < ncols && ch0 + i < p.cout) yr[ch0 + i] = out[i];
+        } else {
+          uint32_t gw[8];
+          pack_group_vals(out, out_bits, gw);
+          store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
+        }
+        }  // valid
+      }
+      __syncwarp();
+      tc_fence_before();
+      mbar_arrive(b_tempty + 8 * buf);
+    }
+    if (!ok) fail(abort_flag, p.status);
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kWarpMma) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;"
+                 ::"r"(tmem_base), "r"(p.tmem_cols) : "memory");
+  }
+}
+
+// ---------------------------------------------------------------- host side
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn get_encode_fn(std::string* err) {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  static cudaError_t st = cudaSuccess;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    st = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q);
+    if (st == cudaSuccess && q == cudaDriverEntryPointSuccess) fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  });
+  if (!fn && err) *err = "cuTensorMapEncodeTiled entry point unavailable";
+  return fn;
+}
+
+template <int kXBits>
+static int launch_bits(const Params& prm, const CUtensorMap& map, int grid, size_t smem,
+                       cudaStream_t stream, std::string* err) {
+  auto kern = conv_tc_kernel<kXBits>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) { *err = std::string("cudaFuncSetAttribute: ") + cudaGetErrorString(e); return 3; }
+  kern<<<grid, kThreads, smem, stream>>>(map, prm);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) { *err = std::string("conv_tc launch: ") + cudaGetErrorString(e); return 3; }
+  return 0;
+}
+
+}  // namespace tc
+
+int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
+  using namespace tc;
+  Params prm{};
+  const int BN = a.bn;
+  prm.njobs = a.njobs;
+  prm.n_tiles = a.cout_pad / BN;
+  int tiles = 0;
+  for (int j = 0; j < a.njobs; ++j) {
+    prm.jobs[j] = a.jobs[j];
+    prm.jobs[j].tile_begin = tiles;
+    tiles += ((a.jobs[j].m_total + BM - 1) / BM) * prm.n_tiles;
+  }
+  prm.total_tiles = tiles;
+  if (tiles == 0) return 0;
+  prm.num_kchunks = a.k_pad / BK;
+  prm.cin = a.cin; prm.cout = a.cout; prm.kh = a.kh; prm.kw = a.kw;
+  prm.stride = a.stride; prm.pad = a.pad; prm.k_total = a.k_total;
+  prm.out_bits = a.out_bits; prm.skip_bits = a.skip_bits;
+  prm.x_row_bytes = a.x_row_bytes; prm.y_row_bytes = a.y_row_bytes; prm.skip_row_bytes = a.skip_row_bytes;
+  prm.m0 = a.m0; prm.shift = a.shift; prm.bias = a.bias;
+  prm.skip_c = a.skip_c; prm.skip_d = a.skip_d;
+  prm.upsample = a.upsample; prm.scale_main = a.scale_main; prm.has_skip = a.has_skip;
+  prm.bn = BN;
+  prm.status = a.status;
+  // shared memory plan
+  const int stg_stride = (a.x_bits == 2) ? 48 : 80;  // conflict-free 16-byte row reads
+  const size_t stage_bytes = (size_t)BM * BK + (size_t)BN * BK;
+  const size_t stg_bytes = (size_t)kDepth * BM * stg_stride;
+  const size_t epi_bytes = 256 * sizeof(EpiChan);
+  const size_t bar_bytes = 8 * (2 * kMaxStages + 5) + 16;
+  const size_t budget = 232448 - 1024;  // max dynamic smem per block minus alignment slack
+  const size_t fixed = stg_bytes + epi_bytes + bar_bytes;
+  int stages = (int)((budget - fixed) / stage_bytes);
+  if (stages > kMaxStages) stages = kMaxStages;
+  if (stages < 2) { *err = "conv_tc: shared memory plan does not fit"; return 2; }
+  prm.stages = stages;
+  prm.stg_stride = stg_stride;
+  prm.off_b = (uint32_t)(stages * BM * BK);
+  prm.off_stg = prm.off_b + (uint32_t)(stages * BN * BK);
+  prm.off_epi = prm.off_stg + (uint32_t)stg_bytes;
+  prm.off_bar = prm.off_epi + (uint32_t)epi_bytes;
+  const size_t smem = 1024 + prm.off_bar + bar_bytes;
+  int cols = 32;
+  while (cols < 2 * BN) cols *= 2;
+  prm.tmem_cols = cols;
+
+  EncodeTiledFn enc = get_encode_fn(err);
+  if (!enc) return 3;
+  CUtensorMap map;
+  cuuint64_t gdim[2] = {(cuuint64_t)a.k_pad, (cuuint64_t)a.cout_pad};
+  cuuint64_t gstride[1] = {(cuuint64_t)a.k_pad};
+  cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)BN};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(&map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)a.w_e4m3, gdim, gstride, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) { *err = "cuTensorMapEncodeTiled failed: " + std::to_string((int)r); return 3; }
+
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int grid = tiles < sms ? tiles : sms;
+  switch (a.x_bits) {
+    case 2: return launch_bits<2>(prm, map, grid, smem, stream, err);
+    case 3: return launch_bits<3>(prm, map, grid, smem, stream, err);
+    case 4: return launch_bits<4>(prm, map, grid, smem, stream, err);
+    default: *err = "conv_tc: activation bits must be 2, 3 or 4"; return 2;
+  }
+}
+
+}  // namespace aqd

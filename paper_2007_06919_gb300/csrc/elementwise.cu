@@ -1,0 +1,242 @@
+// elementwise.cu -- the element-wise parts of AQD's integer inference path:
+//   * requant (Eq. 6 bias + Eq. 2 fixed-point rescale and clip) of an int32 tensor,
+//   * the integer skip add of Eq. 7 with Eq. 8's dyadic factor (optionally reading the
+//     skip through a nearest 2x upsample, the FPN top-down add),
+//   * max-pooling directly on codes (Sec. 3.2.4),
+//   * code packing / unpacking and the one-time weight preparation.
+// One thread handles one pixel's 32-channel group, so loads and stores are whole
+// packed groups (8/12/16/32 bytes, or 128 bytes of int32).
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace aqd {
+namespace elt {
+
+constexpr int kThreads = 256;
+
+__device__ __forceinline__ void load_vals(const uint8_t* row, int bits, int c, int ch0, bool is_signed,
+                                          int32_t v[32]) {
+  if (bits == 32 && (c % 32) == 0) {
+    const int4* p = reinterpret_cast<const int4*>(row + 4 * (int64_t)ch0);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const int4 x = p[q];
+      v[4 * q] = x.x; v[4 * q + 1] = x.y; v[4 * q + 2] = x.z; v[4 * q + 3] = x.w;
+    }
+  } else if (bits != 32 && (bits != 8 || (c % 32) == 0)) {
+    unpack_group_vals(row + (ch0 >> 5) * group_bytes(bits), bits, is_signed, v);
+  } else {
+#pragma unroll 4
+    for (int i = 0; i < 32; ++i) v[i] = (ch0 + i < c) ? read_code(row, ch0 + i, bits, is_signed) : 0;
+  }
+}
+
+__device__ __forceinline__ void store_vals(uint8_t* row, int bits, int c, int ch0, const int32_t v[32]) {
+  if (bits == 32) {
+    int32_t* p = reinterpret_cast<int32_t*>(row) + ch0;
+    if ((c % 32) == 0) {
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        reinterpret_cast<int4*>(p)[q] = make_int4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+    } else {
+      for (int i = 0; i < 32; ++i)
+        if (ch0 + i < c) p[i] = v[i];
+    }
+  } else if (bits == 8 && (c % 32) != 0) {
+    for (int i = 0; i < 32; ++i)
+      if (ch0 + i < c) row[ch0 + i] = (uint8_t)v[i];
+  } else {
+    uint32_t g[8];
+    pack_group_vals(v, bits, g);
+    store_group(row + (ch0 >> 5) * group_bytes(bits), g, bits);
+  }
+}
+
+template <bool kHasSkip>
+__global__ void __launch_bounds__(kThreads) eltwise_kernel(const EltArgs a) {
+  const int groups = (a.c + 31) / 32;
+  const int64_t total = (int64_t)a.n * a.h * a.w * groups;
+  const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  if (t >= total) return;
+  const int64_t pix = t / groups;
+  const int ch0 = (int)(t - pix * groups) * 32;
+  int32_t av[32];
+  load_vals(a.a + pix * a.a_row_bytes, a.a_bits, a.c, ch0, a.a_bits == 32, av);
+  int32_t sv[32];
+  if (kHasSkip) {
+    const int64_t hw = (int64_t)a.h * a.w;
+    const int64_t img = pix / hw;
+    const int64_t rem = pix - img * hw;
+    const int hh = (int)(rem / a.w), ww = (int)(rem - (rem / a.w) * a.w);
+    const int64_t sp = (img * a.b_h + hh / a.upsample) * a.b_w + ww / a.upsample;
+    load_vals(a.b + sp * a.b_row_bytes, a.b_bits, a.c, ch0, a.b_bits == 32, sv);
+  }
+  int32_t out[32];
+#pragma unroll 4
+  for (int i = 0; i < 32; ++i) {
+    const int ch = ch0 + i;
+    EpiChan ec{};
+    if (ch < a.c) {
+      const int64_t idx = (int64_t)a.level * a.c + ch;
+      ec.bias = a.bias ? a.bias[idx] : 0;
+      if (a.y_bits != 32) { ec.m0 = a.m0[idx]; ec.r = (int8_t)(31 + a.shift[idx]); }
+      if (kHasSkip) { ec.c = a.skip_c[idx]; ec.d = a.skip_d[idx]; }
+    }
+    out[i] = epilogue<kHasSkip>(av[i], kHasSkip ? sv[i] : 0, ec, a.scale_main, a.y_bits);
+  }
+  store_vals(a.y + pix * a.y_row_bytes, a.y_bits, a.c, ch0, out);
+}
+
+__global__ void __launch_bounds__(kThreads) maxpool_kernel(const PoolArgs a) {
+  const int groups = (a.c + 31) / 32;
+  const int64_t total = (int64_t)a.n * a.ho * a.wo * groups;
+  const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  if (t >= total) return;
+  const int64_t pix = t / groups;
+  const int ch0 = (int)(t - pix * groups) * 32;
+  const int64_t hw = (int64_t)a.ho * a.wo;
+  const int64_t img = pix / hw;
+  const int64_t rem = pix - img * hw;
+  const int oh = (int)(rem / a.wo), ow = (int)(rem - (rem / a.wo) * a.wo);
+  int32_t best[32];
+#pragma unroll
+  for (int i = 0; i < 32; ++i) best[i] = 0;  // codes are >= 0; every window holds a tap
+  for (int r = 0; r < a.k; ++r) {
+    const int hi = oh * a.stride - a.pad + r;
+    if (hi < 0 || hi >= a.h) continue;
+    for (int s = 0; s < a.k; ++s) {
+      const int wi = ow * a.stride - a.pad + s;
+      if (wi < 0 || wi >= a.w) continue;
+      int32_t v[32];
+      load_vals(a.x + ((img * a.h + hi) * a.w + wi) * a.row_bytes, a.bits, a.c, ch0, false, v);
+#pragma unroll
+      for (int i = 0; i < 32; ++i) best[i] = max(best[i], v[i]);
+    }
+  }
+  store_vals(a.y + pix * a.row_bytes, a.bits, a.c, ch0, best);
+}
+
+__global__ void __launch_bounds__(kThreads)
+pack_kernel(const int32_t* codes, int64_t rows, int c, int bits, int64_t row_bytes, uint8_t* out) {
+  const int groups = (c + 31) / 32;
+  const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  if (t >= rows * groups) return;
+  const int64_t r = t / groups;
+  const int ch0 = (int)(t - r * groups) * 32;
+  int32_t v[32];
+#pragma unroll 4
+  for (int i = 0; i < 32; ++i) v[i] = (ch0 + i < c) ? codes[r * c + ch0 + i] : 0;
+  if (bits == 8) {
+    for (int i = 0; i < 32; ++i)
+      if (ch0 + i < c) out[r * row_bytes + ch0 + i] = (uint8_t)(v[i] & 0xFF);
+    return;
+  }
+  uint32_t g[8];
+  pack_group_vals(v, bits, g);
+  store_group(out + r * row_bytes + (ch0 >> 5) * group_bytes(bits), g, bits);
+}
+
+__global__ void __launch_bounds__(kThreads)
+unpack_kernel(const uint8_t* packed, int64_t rows, int c, int bits, int64_t row_bytes, int is_signed,
+              int32_t* out) {
+  const int groups = (c + 31) / 32;
+  const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  if (t >= rows * groups) return;
+  const int64_t r = t / groups;
+  const int ch0 = (int)(t - r * groups) * 32;
+  int32_t v[32];
+  load_vals(packed + r * row_bytes, bits, c, ch0, is_signed != 0, v);
+  for (int i = 0; i < 32; ++i)
+    if (ch0 + i < c) out[r * c + ch0 + i] = v[i];
+}
+
+// Prepared weights: E4M3 sign-magnitude bytes [cout_pad][k_pad] (zero padded; only when
+// every |w| <= 15) followed by int16 [cout][k_total].
+__global__ void __launch_bounds__(kThreads)
+prepare_weights_kernel(const uint8_t* wp, int w_bits, int w_format, WeightGeom g, int64_t w_row_bytes,
+                       int make_e4m3, uint8_t* out) {
+  const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  const int64_t n_e4 = (int64_t)g.cout_pad * g.k_pad;
+  const int64_t n_i16 = (int64_t)g.cout * g.k_total;
+  if (t >= n_e4 + n_i16) return;
+  int64_t co, k;
+  if (t < n_e4) { co = t / g.k_pad; k = t - co * g.k_pad; }
+  else { co = (t - n_e4) / g.k_total; k = (t - n_e4) - co * g.k_total; }
+  int32_t w = 0;
+  if (co < g.cout && k < g.k_total) {
+    const int64_t tap = k / g.cin;
+    const int ch = (int)(k - tap * g.cin);
+    const uint8_t* row = wp + (co * g.kh * g.kw + tap) * w_row_bytes;
+    if (w_format == 0) {
+      w = read_code(row, ch, w_bits, true);
+    } else {  // Eq. 3 odd grid: eta -> 2 eta - (2^k - 1)
+      w = 2 * read_code(row, ch, w_bits, false) - ((1 << w_bits) - 1);
+    }
+  }
+  if (t < n_e4) {
+    if (make_e4m3) {
+      const uint32_t mag = (uint32_t)(w < 0 ? -w : w);
+      out[t] = (uint8_t)((w < 0 ? 0x80u : 0u) | (mag & 0x0Fu));
+    } else {
+      out[t] = 0;
+    }
+  } else {
+    reinterpret_cast<int16_t*>(out + g.i16_offset)[t - n_e4] = (int16_t)w;
+  }
+}
+
+inline unsigned blocks_for(int64_t n) { return (unsigned)((n + kThreads - 1) / kThreads); }
+
+}  // namespace elt
+
+static int check_launch(const char* what, std::string* err) {
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) { *err = std::string(what) + ": " + cudaGetErrorString(e); return 3; }
+  return 0;
+}
+
+int launch_elementwise(const EltArgs& a, cudaStream_t stream, std::string* err) {
+  const int64_t total = (int64_t)a.n * a.h * a.w * ((a.c + 31) / 32);
+  if (total == 0) return 0;
+  if (a.has_skip) elt::eltwise_kernel<true><<<elt::blocks_for(total), elt::kThreads, 0, stream>>>(a);
+  else elt::eltwise_kernel<false><<<elt::blocks_for(total), elt::kThreads, 0, stream>>>(a);
+  return check_launch("eltwise launch", err);
+}
+
+int launch_maxpool(const PoolArgs& a, cudaStream_t stream, std::string* err) {
+  const int64_t total = (int64_t)a.n * a.ho * a.wo * ((a.c + 31) / 32);
+  if (total == 0) return 0;
+  elt::maxpool_kernel<<<elt::blocks_for(total), elt::kThreads, 0, stream>>>(a);
+  return check_launch("maxpool launch", err);
+}
+
+int launch_pack(const int32_t* codes, int64_t rows, int32_t c, int32_t bits, uint8_t* out,
+                cudaStream_t stream, std::string* err) {
+  const int64_t total = rows * ((c + 31) / 32);
+  if (total == 0) return 0;
+  elt::pack_kernel<<<elt::blocks_for(total), elt::kThreads, 0, stream>>>(codes, rows, c, bits,
+                                                                          row_bytes_of(c, bits), out);
+  return check_launch("pack launch", err);
+}
+
+int launch_unpack(const uint8_t* packed, int64_t rows, int32_t c, int32_t bits, int32_t is_signed,
+                  int32_t* out, cudaStream_t stream, std::string* err) {
+  const int64_t total = rows * ((c + 31) / 32);
+  if (total == 0) return 0;
+  elt::unpack_kernel<<<elt::blocks_for(total), elt::kThreads, 0, stream>>>(packed, rows, c, bits,
+                                                                            row_bytes_of(c, bits), is_signed, out);
+  return check_launch("unpack launch", err);
+}
+
+int launch_prepare_weights(const uint8_t* w_packed, int32_t w_bits, int32_t w_format, const WeightGeom& g,
+                           uint8_t* out, cudaStream_t stream, std::string* err) {
+  const int64_t total = (int64_t)g.cout_pad * g.k_pad + (int64_t)g.cout * g.k_total;
+  const int max_abs = (w_format == 0) ? (1 << (w_bits - 1)) : ((1 << w_bits) - 1);
+  elt::prepare_weights_kernel<<<elt::blocks_for(total), elt::kThreads, 0, stream>>>(
+      w_packed, w_bits, w_format, g, row_bytes_of(g.cin, w_bits), max_abs <= 15 ? 1 : 0, out);
+  return check_launch("prepare_weights launch", err);
+}
+
+}  // namespace aqd

@@ -1,0 +1,91 @@
+// kernels.h -- internal interface between the C-ABI layer (aqd_api.cu) and the kernels.
+#pragma once
+#include <cuda_runtime.h>
+
+#include <cstdint>
+#include <string>
+
+namespace aqd {
+
+constexpr int kMaxJobs = 8;
+
+struct ConvJobDev {
+  const uint8_t* x;
+  uint8_t* y;
+  const uint8_t* skip;
+  int32_t n, h, w;        // input
+  int32_t ho, wo;         // output
+  int32_t skip_h, skip_w;
+  int32_t level;
+  int32_t m_total;        // n * ho * wo
+  int32_t tile_begin;     // first global tile index of this job
+};
+
+struct ConvArgs {
+  ConvJobDev jobs[kMaxJobs];
+  int32_t njobs;
+  int32_t cin, cout, kh, kw, stride, pad;
+  int32_t x_bits, out_bits, skip_bits;
+  int64_t x_row_bytes, y_row_bytes, skip_row_bytes;
+  const int32_t* m0;
+  const int8_t* shift;
+  const int32_t* bias;
+  const int32_t* skip_c;
+  const int8_t* skip_d;
+  int32_t upsample, scale_main, has_skip;
+  // prepared weights
+  const uint8_t* w_e4m3;  // [cout_pad][k_pad] E4M3 sign-magnitude bytes (|w| <= 15)
+  const int16_t* w_i16;   // [cout][k_total] signed integers
+  int32_t cout_pad, k_total, k_pad, bn;
+  uint32_t* status;       // device status word
+};
+
+// Prepared-weight geometry shared by the API and the weight-prep kernel.
+struct WeightGeom {
+  int32_t cout, kh, kw, cin;
+  int32_t k_total, k_pad, bn, cout_pad;
+  size_t e4m3_bytes, i16_offset, total_bytes;
+};
+WeightGeom weight_geom(int32_t cout, int32_t kh, int32_t kw, int32_t cin);
+
+// 0 on success, else an aqd_status value; *err gets a message.
+int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err);
+int launch_conv_direct(const ConvArgs& a, cudaStream_t stream, std::string* err);
+int launch_prepare_weights(const uint8_t* w_packed, int32_t w_bits, int32_t w_format,
+                           const WeightGeom& g, uint8_t* out, cudaStream_t stream,
+                           std::string* err);
+int launch_pack(const int32_t* codes, int64_t rows, int32_t c, int32_t bits, uint8_t* out,
+                cudaStream_t stream, std::string* err);
+int launch_unpack(const uint8_t* packed, int64_t rows, int32_t c, int32_t bits,
+                  int32_t is_signed, int32_t* out, cudaStream_t stream, std::string* err);
+
+struct EltArgs {
+  const uint8_t* a;
+  int32_t a_bits;
+  int64_t a_row_bytes;
+  const uint8_t* b;       // skip (may be null)
+  int32_t b_bits;
+  int64_t b_row_bytes;
+  int32_t b_h, b_w;
+  uint8_t* y;
+  int32_t y_bits;
+  int64_t y_row_bytes;
+  int32_t n, h, w, c;
+  const int32_t* m0;
+  const int8_t* shift;
+  const int32_t* bias;
+  const int32_t* skip_c;
+  const int8_t* skip_d;
+  int32_t upsample, scale_main, has_skip, level;
+};
+int launch_elementwise(const EltArgs& a, cudaStream_t stream, std::string* err);
+
+struct PoolArgs {
+  const uint8_t* x;
+  uint8_t* y;
+  int32_t n, h, w, c, bits, ho, wo, k, stride, pad;
+  int64_t row_bytes;
+};
+int launch_maxpool(const PoolArgs& a, cudaStream_t stream, std::string* err);
+
+}  // namespace aqd

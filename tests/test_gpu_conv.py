@@ -1,0 +1,153 @@
+"""GPU parity of the integer convolution (Eq. 4 + fused Eq. 6/7/2 epilogue) against the
+CPU oracle: bit-exact on every output byte, through the C ABI, for both kernels."""
+import numpy as np
+import pytest
+
+from gpu_util import assert_same, conv_pair, weights
+from paper_2007_06919_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+TC, DIRECT = 1, 2
+
+
+def _params(rng, levels, cout, out_bits, calib_std=None):
+    return synth.requant_params(rng, levels, cout, calib_std=calib_std, out_bits=out_bits)
+
+
+def test_library_uses_the_gpu():
+    import torch
+    assert torch.cuda.is_available()
+    cap = torch.cuda.get_device_capability()
+    assert cap[0] >= 10, cap
+
+
+@pytest.mark.parametrize("path", [TC, DIRECT])
+def test_config0_bit_exact(path):
+    wl = synth.config0()
+    cv = wl.convs[0]
+    got, want, used = conv_pair(wl.inputs[0], 2, cv.w, 2, m0=cv.m0, shift=cv.shift, bias=cv.bias,
+                                out_bits=2, path=path)
+    assert used == path
+    assert_same(got, want, 64, 2, "config0")
+
+
+@pytest.mark.parametrize("path", [TC, DIRECT])
+def test_config0_calibrated_bit_exact(path):
+    """Same shape with shifts drawn so codes spread over 0..3 (not all clipped)."""
+    rng = np.random.default_rng(100)
+    x = synth.act_codes(rng, (1, 32, 32, 64), 2)
+    w = synth.weight_codes(rng, (64, 3, 3, 64), 2)
+    m0, sh, b = _params(rng, 1, 64, 2, calib_std=37.0)
+    got, want, _ = conv_pair(x, 2, w, 2, m0=m0, shift=sh, bias=b, out_bits=2, path=path)
+    assert len(np.unique(got)) > 8
+    assert_same(got, want, 64, 2, "config0 calibrated")
+
+
+# (x_bits, w_bits, w_format, n, h, w, cin, cout, k, stride, pad, out_bits)
+CASES = [
+    (2, 2, 0, 2, 13, 17, 64, 64, 3, 1, 1, 2),      # ragged M (442 rows), K = 576
+    (4, 4, 0, 1, 9, 23, 128, 128, 3, 1, 1, 4),     # 4-bit, ragged
+    (3, 3, 0, 2, 7, 11, 96, 64, 3, 1, 1, 3),       # 3-bit, cin 96: a 128-byte chunk spans taps
+    (2, 2, 1, 1, 10, 10, 32, 32, 3, 1, 1, 2),      # Eq. 3 odd weights, cin 32 (K = 288 -> 384)
+    (4, 4, 1, 1, 6, 9, 64, 64, 3, 1, 1, 4),        # odd 4-bit weights: |w| up to 15
+    (4, 4, 0, 2, 15, 14, 64, 128, 3, 2, 1, 4),     # stride 2
+    (4, 4, 0, 2, 16, 12, 512, 128, 1, 1, 0, 4),    # 1x1 512 -> 128
+    (4, 4, 0, 1, 8, 8, 128, 512, 1, 1, 0, 4),      # 1x1 128 -> 512: two N tiles
+    (4, 2, 0, 1, 19, 21, 32, 64, 7, 2, 3, 4),      # 7x7 stride 2
+    (2, 2, 0, 2, 11, 9, 256, 80, 3, 1, 1, 32),     # int32 output, 80 channels (N tile 80)
+    (2, 2, 0, 2, 5, 7, 256, 4, 3, 1, 1, 32),       # int32 output, 4 channels (N tile 16)
+    (2, 2, 0, 1, 1, 1, 64, 64, 3, 1, 1, 2),        # 1x1 image: every tap but the centre pads
+    (4, 4, 0, 1, 3, 300, 64, 32, 1, 1, 0, 8),      # 8-bit output codes
+    (3, 4, 0, 1, 33, 5, 32, 96, 3, 1, 0, 3),       # no padding, cout 96
+]
+
+
+@pytest.mark.parametrize("case", CASES, ids=[str(i) for i in range(len(CASES))])
+@pytest.mark.parametrize("path", [TC, DIRECT])
+def test_conv_shapes_bit_exact(case, path):
+    xb, wb, fmt, n, h, wd, cin, cout, k, stride, pad, ob = case
+    rng = np.random.default_rng(hash(case) % 2 ** 32)
+    x = synth.act_codes(rng, (n, h, wd, cin), xb)
+    if fmt == 0:
+        w = rng.integers(-(1 << (wb - 1)), 1 << (wb - 1), size=(cout, k, k, cin)).astype(np.int32)
+    else:
+        w = rng.integers(0, 1 << wb, size=(cout, k, k, cin)).astype(np.int32)
+    std = np.sqrt(k * k * cin * np.mean(np.arange(1 << xb) ** 2) * (1 << (2 * wb - 2)) / 3)
+    m0, sh, b = _params(rng, 1, cout, ob if ob != 32 else 4, calib_std=std)
+    got, want, used = conv_pair(x, xb, w, wb, w_format=fmt, stride=stride, pad=pad, out_bits=ob,
+                                m0=m0, shift=sh, bias=b, path=path)
+    assert used == path
+    assert_same(got, want, cout, ob, f"case {case}")
+
+
+@pytest.mark.parametrize("path", [TC, DIRECT])
+@pytest.mark.parametrize("skip_bits,upsample,mirror", [(4, 1, 0), (4, 1, 1), (32, 1, 0), (2, 2, 0), (32, 2, 1),
+                                                        (8, 1, 0)])
+def test_conv_with_skip_bit_exact(path, skip_bits, upsample, mirror):
+    """Eq. 7 fused into the epilogue: identity / downsample (int32) / FPN (upsample 2) skips,
+    both directions of the rescale."""
+    rng = np.random.default_rng(7 + skip_bits + 10 * upsample + 100 * mirror)
+    n, h, wd, cin, cout = 2, 14, 11, 128, 64
+    x = synth.act_codes(rng, (n, h, wd, cin), 4)
+    w = synth.weight_codes(rng, (cout, 3, 3, cin), 4, "normal2")
+    m0, sh, b = _params(rng, 1, cout, 4, calib_std=300.0)
+    sh_ = (h + upsample - 1) // upsample, (wd + upsample - 1) // upsample
+    if skip_bits == 32:
+        skip = rng.integers(-5000, 5000, size=(n, sh_[0], sh_[1], cout)).astype(np.int32)
+    else:
+        skip = synth.act_codes(rng, (n, sh_[0], sh_[1], cout), skip_bits)
+    c, d = synth.skip_params(rng, 1, cout, sh)
+    got, want, _ = conv_pair(x, 4, w, 4, out_bits=4, m0=m0, shift=sh, bias=b, skip=skip, skip_bits=skip_bits,
+                             skip_c=c, skip_d=d, upsample=upsample, scale_main=mirror, path=path)
+    assert_same(got, want, cout, 4, "skip")
+
+
+@pytest.mark.parametrize("x_bits,w_lim", [(4, 8), (3, 4), (2, 2)])
+def test_tensor_core_sum_is_exact_at_the_bound(x_bits, w_lim):
+    """Adversarial accumulation: every code at its maximum and weights of one sign, with
+    K as large as the exact-FP32 bound K * max|x| * max|w| < 2^24 lets the tensor-core
+    kernel take; int32 outputs must equal the oracle's int64 sums exactly."""
+    amax = (1 << x_bits) - 1
+    cin = 32 * ((((1 << 24) - 1) // (9 * amax * w_lim)) // 32)
+    cin = min(cin, 65536)
+    rng = np.random.default_rng(x_bits)
+    x = np.full((1, 5, 6, cin), amax, np.int32)
+    x[0, 2, 3, ::3] = rng.integers(0, amax + 1, size=x[0, 2, 3, ::3].shape)
+    w = np.full((32, 3, 3, cin), -w_lim, np.int32)
+    w[1::2] = w_lim - 1 if w_lim - 1 > 0 else 1     # odd channels positive
+    w[5, :, :, ::2] = 1                              # mixed signs inside one sum
+    got, want, used = conv_pair(x, x_bits, w, 4 if w_lim == 8 else (3 if w_lim == 4 else 2), pad=1,
+                                out_bits=32, bias=np.zeros((1, 32), np.int32), path=TC)
+    assert used == TC
+    assert_same(got, want, 32, 32, "exactness")
+    assert np.abs(want.view(np.int32)).max() > (1 << 21)
+
+
+def test_paths_agree_on_config1_conv2():
+    """3x3 128->128 4-bit of the bottleneck at full size on both kernels and the oracle."""
+    wl = synth.config1()
+    cv = wl.convs[1]
+    rng = np.random.default_rng(5)
+    x = synth.act_codes(rng, (2, 100, 152, 128), 4, "halfnormal4")
+    wp = weights(cv.w, 4)
+    outs = [conv_pair(x, 4, cv.w, 4, m0=cv.m0, shift=cv.shift, bias=cv.bias, out_bits=4, path=p, wprep=wp)
+            for p in (TC, DIRECT)]
+    assert_same(outs[0][0], outs[0][1], 128, 4, "tc")
+    assert_same(outs[1][0], outs[1][1], 128, 4, "direct")
+
+
+def test_invalid_skip_shape_is_rejected_before_launch():
+    import torch
+    from paper_2007_06919_gb300 import aqd
+    rng = np.random.default_rng(0)
+    W, _ = weights(synth.weight_codes(rng, (32, 3, 3, 32), 2), 2)
+    X = aqd.DTensor.empty(1, 8, 8, 32, 2)
+    Y = aqd.DTensor.empty(1, 8, 8, 32, 2)
+    S = aqd.DTensor.empty(1, 3, 8, 32, 2)  # too few rows for the output
+    rq = aqd.RequantParams.from_numpy(np.ones((1, 32)), np.zeros((1, 32)), np.zeros((1, 32)))
+    sp = aqd.SkipParams.from_numpy(np.ones((1, 32)), np.zeros((1, 32)))
+    with pytest.raises(aqd.AqdError) as e:
+        aqd.conv_int(X, W, 1, 1, Y, rq=rq, skip=S, sp=sp)
+    assert e.value.status == 1
+    torch.cuda.synchronize()

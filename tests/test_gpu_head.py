@@ -1,0 +1,136 @@
+"""GPU parity at the workloads' full sizes: the ResNet-50 C3 bottleneck (4-bit, identity
+skip), the shared RetinaNet head tower over the five FPN levels with multi-level BN tables
+(2-bit, grouped launch), and the 2/3/4/8-bit sweep of that tower at batch 16."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_util import assert_same, dev, to_device, weights
+from paper_2007_06919_gb300 import aqd, synth
+
+pytestmark = pytest.mark.gpu
+
+
+def _ref_conv(xt, wp, cv, level=0, skip=None):
+    return oracle.conv_int(xt, wp, cv.w_bits, 0, cv.kh, cv.kw, cv.stride, cv.pad, cv.cout, level=level,
+                           m0=cv.m0, shift=cv.shift, bias=cv.bias,
+                           levels=(cv.m0 if cv.m0 is not None else cv.bias).shape[0], skip=skip,
+                           skip_c=cv.skip_c, skip_d=cv.skip_d, out_bits=cv.out_bits)
+
+
+def _rq(cv):
+    return aqd.RequantParams.from_numpy(cv.m0, cv.shift, cv.bias)
+
+
+def test_config1_bottleneck_chain_bit_exact():
+    """1x1 512->128, 3x3 128->128, 1x1 128->512 + identity skip (Eq. 7), all at
+    2 x 100 x 152, 4-bit: each stage is compared; the GPU chain feeds itself and the
+    oracle chain feeds itself."""
+    wl = synth.config1()
+    x = wl.inputs[0]
+    xt = oracle.CodeTensor.from_codes(x, 4)
+    ref = xt
+    cur = to_device(xt)
+    for i, cv in enumerate(wl.convs):
+        W, wp = weights(cv.w, 4)
+        skip_ref = xt if cv.skip_c is not None else None
+        ref = _ref_conv(ref, wp, cv, skip=skip_ref)
+        Y = aqd.DTensor.empty(ref.n, ref.h, ref.w, cv.cout, 4)
+        sp = aqd.SkipParams.from_numpy(cv.skip_c, cv.skip_d) if cv.skip_c is not None else None
+        aqd.conv_int(cur, W, cv.stride, cv.pad, Y, rq=_rq(cv), skip=to_device(xt) if sp else None, sp=sp)
+        assert aqd.last_conv_path() == 1
+        torch.cuda.synchronize()
+        assert_same(Y.data.cpu().numpy().reshape(ref.packed.shape), ref.packed, cv.cout, 4, f"stage {i}")
+        cur = Y
+    assert aqd.device_status() == 0
+    assert len(np.unique(ref.codes())) > 3
+
+
+def _tower_levels_gpu(inputs, convs, bits, grouped=True):
+    """Runs the 4-layer tower + cls/box on every level; returns per-level outputs."""
+    nl = len(inputs)
+    xs = [to_device(oracle.CodeTensor.from_codes(x, bits)) for x in inputs]
+    for cv in convs[:4]:
+        W, _ = weights(cv.w, bits)
+        ys = [aqd.DTensor.empty(x.n, x.h, x.w, 256, bits) for x in xs]
+        if grouped:
+            aqd.conv_int_grouped([(xs[l], ys[l], None, l) for l in range(nl)], W, 1, 1, rq=_rq(cv))
+        else:
+            for l in range(nl):
+                aqd.conv_int(xs[l], W, 1, 1, ys[l], level=l, rq=_rq(cv))
+        xs = ys
+    heads = []
+    for cv in convs[4:]:
+        W, _ = weights(cv.w, bits)
+        ys = [aqd.DTensor.empty(x.n, x.h, x.w, cv.cout, 32) for x in xs]
+        aqd.conv_int_grouped([(xs[l], ys[l], None, l) for l in range(nl)], W, 1, 1,
+                             rq=aqd.RequantParams.from_numpy(None, None, cv.bias))
+        heads.append(ys)
+    torch.cuda.synchronize()
+    return xs, heads
+
+
+def _tower_levels_ref(inputs, convs, bits):
+    xs = [oracle.CodeTensor.from_codes(x, bits) for x in inputs]
+    for cv in convs[:4]:
+        wp = oracle.pack(cv.w.reshape(-1, cv.cin), bits)
+        xs = [_ref_conv(xs[l], wp, cv, level=l) for l in range(len(xs))]
+    heads = []
+    for cv in convs[4:]:
+        wp = oracle.pack(cv.w.reshape(-1, cv.cin), bits)
+        heads.append([_ref_conv(xs[l], wp, cv, level=l) for l in range(len(xs))])
+    return xs, heads
+
+
+@pytest.mark.parametrize("calibrated", [False, True])
+def test_head_tower_full_size_bit_exact(calibrated):
+    """The whole detector head at 800x1333 (levels 100x168 .. 7x11), batch 2, 2-bit:
+    4 grouped tower layers + cls (80) + box (4) int32 heads, every output compared."""
+    wl = synth.config2(calibrated=calibrated)
+    g_tower, g_heads = _tower_levels_gpu(wl.inputs, wl.convs, 2)
+    r_tower, r_heads = _tower_levels_ref(wl.inputs, wl.convs, 2)
+    for l in range(5):
+        assert_same(g_tower[l].data.cpu().numpy().reshape(r_tower[l].packed.shape), r_tower[l].packed, 256, 2,
+                    f"tower level {l}")
+        for hi, cout in enumerate((80, 4)):
+            assert_same(g_heads[hi][l].data.cpu().numpy().reshape(r_heads[hi][l].packed.shape),
+                        r_heads[hi][l].packed, cout, 32, f"head {cout} level {l}")
+    assert aqd.device_status() == 0
+    if calibrated:
+        assert len(np.unique(r_tower[0].codes())) == 4
+
+
+def test_grouped_launch_equals_per_level_launches():
+    wl = synth.head_tower(9, 2, 2, levels=[(20, 34), (10, 17), (5, 9), (3, 5), (2, 3)], calibrated=True)
+    a, ah = _tower_levels_gpu(wl.inputs, wl.convs, 2, grouped=True)
+    b, bh = _tower_levels_gpu(wl.inputs, wl.convs, 2, grouped=False)
+    for l in range(5):
+        assert torch.equal(a[l].data, b[l].data)
+        assert torch.equal(ah[0][l].data, bh[0][l].data)
+
+
+@pytest.mark.parametrize("bits", [2, 3, 4, 8])
+def test_bitwidth_sweep_batch16_sampled(bits):
+    """First tower layer of the batch-16 head for each bit width, all five levels in one
+    grouped launch; the oracle computes 600 sampled pixels per level (all channels)."""
+    wl = synth.config4(bits)
+    cv = wl.convs[0]
+    W, wp = weights(cv.w, bits)
+    xts = [oracle.CodeTensor.from_codes(x, bits) for x in wl.inputs]
+    xs = [to_device(t) for t in xts]
+    ys = [aqd.DTensor.empty(x.n, x.h, x.w, 256, bits) for x in xs]
+    aqd.conv_int_grouped([(xs[l], ys[l], None, l) for l in range(5)], W, 1, 1, rq=_rq(cv))
+    assert aqd.last_conv_path() == (1 if bits <= 4 else 2)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(bits)
+    for l in range(5):
+        t = xts[l]
+        total = t.n * t.h * t.w
+        pix = synth.sample_pixels(rng, total, 600)
+        want = oracle.conv_int_pixels(t, wp, bits, 0, 3, 3, 1, 1, 256, pix, level=l, m0=cv.m0, shift=cv.shift,
+                                      bias=cv.bias, levels=5, out_bits=bits)
+        got = oracle.unpack(ys[l].data.cpu().numpy().reshape(total, -1)[pix], 256, bits)
+        bad = np.argwhere(got != want)
+        assert bad.size == 0, f"level {l}: {len(bad)} mismatches, first {bad[:3].tolist()}"
+    assert aqd.device_status() == 0

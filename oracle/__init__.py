@@ -70,6 +70,18 @@ def lib():
                                       ctypes.c_int32, ctypes.c_void_p]
         _lib.aqd_ref_unpack.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32,
                                         ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p]
+        i32, i64, vp = ctypes.c_int32, ctypes.c_int64, ctypes.c_void_p
+        T, R, S = ctypes.POINTER(_Tensor), ctypes.POINTER(_Requant), ctypes.POINTER(_Residual)
+        _lib.aqd_ref_conv_int.argtypes = [T, vp, i32, i32, i32, i32, i32, i32, i32, i32, R, S, i32, T]
+        _lib.aqd_ref_conv_int_pixels.argtypes = [T, vp, i32, i32, i32, i32, i32, i32, i32, i32, R, S, i32,
+                                                 i32, i32, vp, i64, vp]
+        _lib.aqd_ref_requant_tensor.argtypes = [T, R, i32, i32, T]
+        _lib.aqd_ref_residual_add_int.argtypes = [T, T, vp, vp, i32, i32, R, i32, i32, T]
+        _lib.aqd_ref_maxpool_codes.argtypes = [T, i32, i32, i32, T]
+        for fn in ("aqd_ref_pack", "aqd_ref_unpack", "aqd_ref_quantize_multiplier", "aqd_ref_conv_int",
+                   "aqd_ref_conv_int_pixels", "aqd_ref_requant_tensor", "aqd_ref_residual_add_int",
+                   "aqd_ref_maxpool_codes"):
+            getattr(_lib, fn).restype = ctypes.c_int
     return _lib
 
 

@@ -10,10 +10,12 @@
 // K * max|x| * max|w| < 2^24, which the host checks before choosing this kernel.
 //
 // Per CTA (one per SM, persistent over tiles of 128 output pixels x BN channels):
-//   warps 0-3  epilogue: tcgen05.ld of the accumulator, integer epilogue, bit-pack, store
-//   warp  4    TMEM allocation + one thread issuing tcgen05.mma (kind::f8f6f4, M=128)
-//   warp  5    one thread loading prepared weights with TMA (cp.async.bulk.tensor, SW128)
-//   warps 6-9  activation producers: im2col gather of packed k-bit codes with cp.async
+//   warps 0..E-1  epilogue (E = 4 or 8): tcgen05.ld of the accumulator, integer epilogue,
+//              bit-pack, store (warp w reads TMEM lanes 32*(w%4)..; with 8 warps each takes
+//              every other 32-column group)
+//   warp  E    TMEM allocation + one thread issuing tcgen05.mma (kind::f8f6f4, M=128)
+//   warp  E+1  one thread loading prepared weights with TMA (cp.async.bulk.tensor, SW128)
+//   warps E+2..E+5 activation producers: im2col gather of packed k-bit codes with cp.async
 //              (zero-fill = the padding code 0), unpack to E4M3 bytes, store into the
 //              128B-swizzled K-major operand layout, signal an mbarrier
 // Stages of 128 K-bytes (one 128B swizzle atom) circulate between producers and the MMA
@@ -33,11 +35,17 @@ namespace tc {
 
 constexpr int BM = 128;            // output pixels per tile (= TMEM lanes)
 constexpr int BK = 128;            // K bytes per stage
-constexpr int kWarpMma = 4;
-constexpr int kWarpTma = 5;
-constexpr int kWarpProd0 = 6;
+#ifndef AQD_EPI_WARPS
+#define AQD_EPI_WARPS 4
+#endif
+constexpr int kEpiWarps = AQD_EPI_WARPS;  // 4 or 8
+static_assert(kEpiWarps == 4 || kEpiWarps == 8, "epilogue warps");
+constexpr int kEpiThreads = kEpiWarps * 32;
+constexpr int kWarpMma = kEpiWarps;
+constexpr int kWarpTma = kEpiWarps + 1;
+constexpr int kWarpProd0 = kEpiWarps + 2;
 constexpr int kProdWarps = 4;
-constexpr int kThreads = (kWarpProd0 + kProdWarps) * 32;  // 320
+constexpr int kThreads = (kWarpProd0 + kProdWarps) * 32;
 constexpr int kMaxStages = 8;
 constexpr int kDepth = 3;          // cp.async chunks in flight per producer thread
 constexpr uint64_t kTimeoutNs = 1000000000ull;  // 1 s per wait
@@ -122,6 +130,22 @@ __device__ __forceinline__ void fence_barrier_init() {
 __device__ __forceinline__ void named_bar(int id, int n) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
 }
+// named barrier that also returns the AND of `pred` over the participating threads
+__device__ __forceinline__ int named_bar_and(int id, int n, int pred) {
+  int r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.b32 p, %3, 0;\n\t"
+      "bar.red.and.pred q, %1, %2, p;\n\t"
+      "selp.b32 %0, 1, 0, q;\n\t}"
+      : "=r"(r) : "r"(id), "r"(n), "r"(pred) : "memory");
+  return r;
+}
+__device__ __forceinline__ int32_t add_sat(int32_t a, int32_t b) {
+  int32_t r;
+  asm("add.sat.s32 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
 
 template <int kBytes>
 __device__ __forceinline__ void cp_async(uint32_t dst, const void* src, bool ok) {
@@ -204,6 +228,52 @@ __device__ __forceinline__ TileInfo tile_info(const Params& p, int t) {
   return ti;
 }
 
+// ---------------------------------------------------------------- epilogue, general case
+
+// Eq. 6 -> Eq. 7 -> Eq. 2 in int64 for 32 accumulators of one row (any shift, any skip).
+// Kept out of line: the common cases take the 32-bit fast path in the kernel body.
+__device__ __noinline__ void general_epilogue(const Params& p, const uint32_t* v, const EpiChan* ep,
+                                              const uint8_t* srow, int ch0, int ncols, int32_t* out) {
+  int32_t sk[32];
+  if (p.has_skip) {
+    if (p.skip_bits == 32) {
+      for (int i = 0; i < 32; ++i)
+        sk[i] = (i < ncols && ch0 + i < p.cout) ? reinterpret_cast<const int32_t*>(srow)[ch0 + i] : 0;
+    } else {
+      unpack_group_vals(srow + (ch0 >> 5) * group_bytes(p.skip_bits), p.skip_bits, false, sk);
+    }
+  }
+  for (int i = 0; i < 32; ++i) {
+    const int64_t acc = (int64_t)__float2int_rn(__uint_as_float(v[i]) * 262144.0f);  // exact
+    const EpiChan ec = ep[i];
+    out[i] = p.has_skip ? epilogue<true>(acc, sk[i], ec, p.scale_main, p.out_bits)
+                        : epilogue<false>(acc, 0, ec, p.scale_main, p.out_bits);
+  }
+}
+
+// Fast requant of 32 accumulators of one row into one packed group (no skip, R >= 33):
+// u = sat32(acc + bias), y = clamp((mulhi(u, M0) + 2^(R-33)) >> (R-32), 0, 2^k - 1),
+// each code OR-ed straight into its word of the packed layout.
+template <int kOut>
+__device__ __forceinline__ void fast_requant_group(const uint32_t* v, const int4* f, int qmax, uint32_t gw[8]) {
+#pragma unroll
+  for (int w = 0; w < 8; ++w) gw[w] = 0u;
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    const int4 c = f[i];
+    const int32_t acc = __float2int_rn(__uint_as_float(v[i]) * 262144.0f);  // exact integer
+    const int32_t u = add_sat(acc, c.x);
+    const uint32_t y = (uint32_t)min(max((__mulhi(u, c.y) + c.z) >> c.w, 0), qmax);
+    if constexpr (kOut == 3) {
+      gw[i / 16] |= (y & 3u) << (8 * (i % 4) + 2 * ((i % 16) / 4));
+      gw[2] |= (y >> 2) << (8 * (i % 4) + i / 4);
+    } else {
+      constexpr int q = 32 / kOut;
+      gw[i / q] |= y << (8 * (i % 4) + kOut * ((i % q) / 4));
+    }
+  }
+}
+
 // ---------------------------------------------------------------- the kernel
 
 template <int kXBits>
@@ -240,7 +310,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(b_tfull + 8 * b, 1);
-      mbar_init(b_tempty + 8 * b, 4 * 32);
+      mbar_init(b_tempty + 8 * b, kEpiThreads);
     }
     mbar_init(b_final, 1);
     *abort_flag = 0;
@@ -383,10 +453,21 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       // unpack this thread's row: 4 groups of 32 codes -> 128 E4M3 bytes (raw byte = code)
       const uint8_t* src = stg + (size_t)(c % kDepth) * BM * p.stg_stride + (size_t)row * p.stg_stride;
       uint32_t words[4 * kXBits];
+      if constexpr (kXBits == 2) {  // 8-byte reads: stride 40 keeps 16 lanes conflict-free
 #pragma unroll
-      for (int i = 0; i < kXBits; ++i) {
-        const uint4 v = reinterpret_cast<const uint4*>(src)[i];
-        words[4 * i + 0] = v.x; words[4 * i + 1] = v.y; words[4 * i + 2] = v.z; words[4 * i + 3] = v.w;
+        for (int i = 0; i < 4; ++i) {
+          const uint2 v = reinterpret_cast<const uint2*>(src)[i];
+          words[2 * i] = v.x; words[2 * i + 1] = v.y;
+        }
+      } else if constexpr (kXBits == 3) {  // 4-byte reads: stride 52 (13 words, odd)
+#pragma unroll
+        for (int i = 0; i < 12; ++i) words[i] = reinterpret_cast<const uint32_t*>(src)[i];
+      } else {  // 16-byte reads: stride 80 keeps 8 lanes conflict-free
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const uint4 v = reinterpret_cast<const uint4*>(src)[i];
+          words[4 * i + 0] = v.x; words[4 * i + 1] = v.y; words[4 * i + 2] = v.z; words[4 * i + 3] = v.w;
+        }
       }
       uint8_t* arow = smem + (size_t)s * (BM * BK) + (size_t)row * BK;
 #pragma unroll
@@ -405,28 +486,47 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
     cp_async_wait<0>();
     if (!ok) fail(abort_flag, p.status);
   } else {
-    // ------------------------------------------------------------ epilogue (warps 0-3)
-    const int e = threadIdx.x;  // tile row = TMEM lane
-    const uint32_t lane_base = tmem_base + ((uint32_t)(warp * 32) << 16);
+    // ------------------------------------------------------------ epilogue (warps 0..E-1)
+    const int quarter = warp & 3;   // TMEM lane quarter this warp may read
+    const int half = warp >> 2;     // this warp takes every other 32-column group
+    const int e = quarter * 32 + lane;  // tile row = TMEM lane
+    const int et = threadIdx.x;         // 0 .. kEpiThreads-1
+    const uint32_t lane_base = tmem_base + ((uint32_t)(quarter * 32) << 16);
+    const int4* epf = reinterpret_cast<const int4*>(epi + 256);  // fast-path table after epi[256]
     uint32_t lt = 0;
     bool ok = true;
     const int out_bits = p.out_bits;
+    const int qmax = (1 << (out_bits & 15)) - 1;
     for (int t = first_tile; t < p.total_tiles; t += tile_stride, ++lt) {
       const TileInfo ti = tile_info(p, t);
       const ConvJobDev& jb = p.jobs[ti.job];
-      named_bar(1, 128);
-      for (int col = e; col < 256; col += 128) {
+      named_bar(1, kEpiThreads);
+      // Per-column constants of this tile's level. Fast path when the total requant shift
+      // R = 31 + shift is >= 33: y = (mulhi(u, M0) + 2^(R-33)) >> (R-32) equals
+      // rhu(u * M0, R) exactly (the low product word cannot carry into the result).
+      int fast = 1;
+      for (int col = et; col < 256; col += kEpiThreads) {
         const int ch = ti.nt * BN + col;
         EpiChan ec{};
+        int4 ef = make_int4(0, 0, 0, 1);
         if (col < BN && ch < p.cout) {
           const int64_t idx = (int64_t)jb.level * p.cout + ch;
           ec.bias = p.bias ? p.bias[idx] : 0;
-          if (out_bits != 32) { ec.m0 = p.m0[idx]; ec.r = (int8_t)(31 + p.shift[idx]); }
+          if (out_bits != 32) {
+            ec.m0 = p.m0[idx];
+            const int r = 31 + p.shift[idx];
+            ec.r = (int8_t)r;
+            if (r >= 33) ef = make_int4(ec.bias, ec.m0, 1 << (r - 33), r - 32);
+            else fast = 0;
+          }
           if (p.has_skip) { ec.c = p.skip_c[idx]; ec.d = p.skip_d[idx]; }
         }
         epi[col] = ec;
+        reinterpret_cast<int4*>(epi + 256)[col] = ef;
       }
-      named_bar(1, 128);
+      fast = named_bar_and(1, kEpiThreads, fast);
+      // 0: general int64 epilogue, 1: fast requant to codes, 2: int32 output, no skip
+      const int mode = p.has_skip ? 0 : (out_bits == 32 ? 2 : (fast ? 1 : 0));
       const uint32_t buf = lt & 1;
       if (!mbar_wait(b_tfull + 8 * buf, (lt >> 1) & 1, abort_flag)) { ok = false; break; }
       tc_fence_after();
@@ -445,7 +545,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
         srow = jb.skip + (((int64_t)img * jb.skip_h + sh) * jb.skip_w + sw) * p.skip_row_bytes;
       }
       const uint32_t tcol = buf * (uint32_t)BN;
-      for (int g0 = 0; g0 < BN; g0 += 32) {
+      for (int g0 = 32 * half; g0 < BN; g0 += 32 * (kEpiWarps / 4)) {
         const int ncols = (BN - g0) < 32 ? (BN - g0) : 32;  // warp-uniform
         uint32_t v[32];
         uint32_t r16[16];
@@ -457,37 +557,50 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
         tmem_wait_ld();
 #pragma unroll
         for (int i = 0; i < 16; ++i) v[16 + i] = (ncols == 32) ? r16[i] : 0u;
-        if (valid) {
+        if (!valid) continue;
         const int ch0 = ti.nt * BN + g0;
-        int32_t sk[32];
-        if (p.has_skip) {
-          if (p.skip_bits == 32) {
+        if (mode == 1) {
+          uint32_t gw[8];
+          switch (out_bits) {
+            case 2: fast_requant_group<2>(v, epf + g0, qmax, gw); break;
+            case 3: fast_requant_group<3>(v, epf + g0, qmax, gw); break;
+            case 4: fast_requant_group<4>(v, epf + g0, qmax, gw); break;
+            default: fast_requant_group<8>(v, epf + g0, qmax, gw); break;
+          }
+          store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
+        } else if (mode == 2) {
+          int32_t* yr = reinterpret_cast<int32_t*>(yrow) + ch0;
+          const bool full = ncols == 32 && ch0 + 32 <= p.cout;
 #pragma unroll
-            for (int i = 0; i < 32; ++i) sk[i] = (i < ncols && ch0 + i < p.cout) ? reinterpret_cast<const int32_t*>(srow)[ch0 + i] : 0;
+          for (int q = 0; q < 8; ++q) {
+            int32_t o[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+              o[k] = add_sat(__float2int_rn(__uint_as_float(v[4 * q + k]) * 262144.0f), epi[g0 + 4 * q + k].bias);
+            if (full) {
+              reinterpret_cast<int4*>(yr)[q] = make_int4(o[0], o[1], o[2], o[3]);
+            } else {
+#pragma unroll
+              for (int k = 0; k < 4; ++k)
+                if (4 * q + k < ncols && ch0 + 4 * q + k < p.cout) yr[4 * q + k] = o[k];
+            }
+          }
+        } else {
+          uint32_t vv[32];  // local copies: only this rare path goes through the stack
+          int32_t oo[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) vv[i] = v[i];
+          general_epilogue(p, vv, epi + g0, srow, ch0, ncols, oo);
+          if (out_bits == 32) {
+            int32_t* yr = reinterpret_cast<int32_t*>(yrow) + ch0;
+            for (int i = 0; i < 32; ++i)
+              if (i < ncols && ch0 + i < p.cout) yr[i] = oo[i];
           } else {
-            unpack_group_vals(srow + (ch0 >> 5) * group_bytes(p.skip_bits), p.skip_bits, false, sk);
+            uint32_t gw[8];
+            pack_group_vals(oo, out_bits, gw);
+            store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
           }
         }
-        int32_t out[32];
-#pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const float f = __uint_as_float(v[i]) * 262144.0f;  // exact integer (x 2^18)
-          const int64_t acc = (int64_t)__float2int_rn(f);
-          const EpiChan ec = epi[g0 + i];
-          out[i] = p.has_skip ? epilogue<true>(acc, sk[i], ec, p.scale_main, out_bits)
-                              : epilogue<false>(acc, 0, ec, p.scale_main, out_bits);
-        }
-        if (out_bits == 32) {
-          int32_t* yr = reinterpret_cast<int32_t*>(yrow);
-#pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (i < ncols && ch0 + i < p.cout) yr[ch0 + i] = out[i];
-        } else {
-          uint32_t gw[8];
-          pack_group_vals(out, out_bits, gw);
-          store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
-        }
-        }  // valid
       }
       __syncwarp();
       tc_fence_before();
@@ -565,10 +678,11 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   prm.bn = BN;
   prm.status = a.status;
   // shared memory plan
-  const int stg_stride = (a.x_bits == 2) ? 48 : 80;  // conflict-free 16-byte row reads
+  // staging row strides chosen so cp.async writes and the row reads hit distinct banks
+  const int stg_stride = (a.x_bits == 2) ? 40 : (a.x_bits == 3 ? 52 : 80);
   const size_t stage_bytes = (size_t)BM * BK + (size_t)BN * BK;
   const size_t stg_bytes = (size_t)kDepth * BM * stg_stride;
-  const size_t epi_bytes = 256 * sizeof(EpiChan);
+  const size_t epi_bytes = 256 * sizeof(EpiChan) + 256 * sizeof(int4);
   const size_t bar_bytes = 8 * (2 * kMaxStages + 5) + 16;
   const size_t budget = 232448 - 1024;  // max dynamic smem per block minus alignment slack
   const size_t fixed = stg_bytes + epi_bytes + bar_bytes;

@@ -53,7 +53,7 @@ WeightGeom weight_geom(int32_t cout, int32_t kh, int32_t kw, int32_t cin) {
   g.cout = cout; g.kh = kh; g.kw = kw; g.cin = cin;
   g.k_total = kh * kw * cin;
   g.k_pad = (g.k_total + 127) / 128 * 128;
-  g.bn = cout <= 256 ? (cout + 15) / 16 * 16 : 256;
+  g.bn = cout <= 128 ? (cout + 15) / 16 * 16 : 128;  // N tile of the tensor-core kernel
   g.cout_pad = (cout + g.bn - 1) / g.bn * g.bn;
   g.e4m3_bytes = (size_t)g.cout_pad * g.k_pad;
   g.i16_offset = (g.e4m3_bytes + 255) / 256 * 256;

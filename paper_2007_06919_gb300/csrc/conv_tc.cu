@@ -33,7 +33,9 @@
 namespace aqd {
 namespace tc {
 
-constexpr int BM = 128;            // output pixels per tile (= TMEM lanes)
+constexpr int BM = 256;            // output pixels per tile: two M=128 sub-tiles sharing B
+constexpr int kSubA = 128 * 128;   // bytes of one sub-tile's A operand per stage
+constexpr int kStageA = 2 * kSubA; // bytes of A per stage
 constexpr int BK = 128;            // K bytes per stage
 #ifndef AQD_EPI_WARPS
 #define AQD_EPI_WARPS 4
@@ -44,10 +46,9 @@ constexpr int kEpiThreads = kEpiWarps * 32;
 constexpr int kWarpMma = kEpiWarps;
 constexpr int kWarpTma = kEpiWarps + 1;
 constexpr int kWarpProd0 = kEpiWarps + 2;
-constexpr int kProdWarps = 4;
+constexpr int kProdWarps = 8;      // one thread per tile row
 constexpr int kThreads = (kWarpProd0 + kProdWarps) * 32;
 constexpr int kMaxStages = 8;
-constexpr int kDepth = 3;          // cp.async chunks in flight per producer thread
 constexpr uint64_t kTimeoutNs = 1000000000ull;  // 1 s per wait
 
 struct Params {
@@ -62,8 +63,8 @@ struct Params {
   const int32_t* skip_c;
   const int8_t* skip_d;
   int32_t upsample, scale_main, has_skip;
-  int32_t bn, stages, stg_stride, tmem_cols;
-  uint32_t off_b, off_stg, off_epi, off_bar;
+  int32_t bn, stages, tmem_cols;
+  uint32_t off_b, off_epi, off_bar;
   uint32_t* status;
 };
 
@@ -102,8 +103,7 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
 }
 
 // Bounded wait: false if the deadline passed or another role aborted.
-__device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
-  if (mbar_try(bar, parity)) return true;
+__device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
   uint64_t deadline = 0;
   for (uint32_t spin = 1;; ++spin) {
     if (mbar_try(bar, parity)) return true;
@@ -114,6 +114,10 @@ __device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile i
       else if (now > deadline) return false;
     }
   }
+}
+
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+  return mbar_try(bar, parity) || mbar_wait_slow(bar, parity, abort_flag);
 }
 
 __device__ __forceinline__ void fail(volatile int* abort_flag, uint32_t* status) {
@@ -184,8 +188,11 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
 }
 
 // Instruction descriptor, kind::f8f6f4: D=F32, A=B=E4M3, both K-major, N>>3, M>>4.
+// The MMA is always M=128 (one sub-tile, one CTA): M=256 exists only for cta_group::2.
+constexpr int kMmaM = 128;
+static_assert(kSubA == kMmaM * BK, "one sub-tile is one M=128 MMA operand");
 __device__ __forceinline__ uint32_t idesc_e4m3(int n) {
-  return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+  return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(kMmaM >> 4) << 24);
 }
 
 __device__ __forceinline__ void mma_e4m3(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
@@ -276,16 +283,71 @@ __device__ __forceinline__ void fast_requant_group(const uint32_t* v, const int4
 
 // ---------------------------------------------------------------- the kernel
 
+// Loads the packed codes of one 128-channel K chunk of one output row into registers
+// (4 * kXBits words; group g = channels 32g..32g+31 of the chunk at words [g*kXBits, ...)).
+// Taps outside the image (and rows past the end of the job) read zeros = code 0.
 template <int kXBits>
+struct RowCursor {
+  const uint8_t* xbase;  // image base of this row's pixel
+  int hb, wb, H, W;      // top-left input coordinate of the window, image size
+  bool valid;
+  int tr, ts, tc0;       // tap (r, s) and channel offset of the next 32-channel group
+};
+
+template <int kXBits, bool kChunkInTap>
+__device__ __forceinline__ void load_chunk(const Params& p, RowCursor<kXBits>& rc, int q, uint32_t (&w)[4 * kXBits]) {
+  constexpr int kGB = 4 * kXBits;
+  if constexpr (kChunkInTap) {
+    // cin % 128 == 0: the chunk is 128 consecutive channels of one tap
+    const int hi = rc.hb + rc.tr, wi = rc.wb + rc.ts;
+    const bool ok = rc.valid && hi >= 0 && hi < rc.H && wi >= 0 && wi < rc.W;
+    const uint4* src = reinterpret_cast<const uint4*>(rc.xbase + ((int64_t)hi * rc.W + wi) * p.x_row_bytes +
+                                                      (rc.tc0 >> 5) * kGB);
+#pragma unroll
+    for (int i = 0; i < kXBits; ++i) {
+      uint4 v = make_uint4(0, 0, 0, 0);
+      if (ok) v = __ldg(src + i);
+      w[4 * i] = v.x; w[4 * i + 1] = v.y; w[4 * i + 2] = v.z; w[4 * i + 3] = v.w;
+    }
+    rc.tc0 += 128;
+    if (rc.tc0 == p.cin) { rc.tc0 = 0; if (++rc.ts == p.kw) { rc.ts = 0; ++rc.tr; } }
+  } else {
+#pragma unroll
+    for (int g = 0; g < 4; ++g) {
+      const int k0 = q * BK + 32 * g;
+      bool ok = false;
+      const uint8_t* src = rc.xbase;
+      if (k0 < p.k_total) {
+        const int hi = rc.hb + rc.tr, wi = rc.wb + rc.ts;
+        ok = rc.valid && hi >= 0 && hi < rc.H && wi >= 0 && wi < rc.W;
+        src = rc.xbase + ((int64_t)hi * rc.W + wi) * p.x_row_bytes + (rc.tc0 >> 5) * kGB;
+        rc.tc0 += 32;
+        if (rc.tc0 == p.cin) { rc.tc0 = 0; if (++rc.ts == p.kw) { rc.ts = 0; ++rc.tr; } }
+      }
+      if constexpr (kXBits == 2) {
+        uint2 v = make_uint2(0, 0);
+        if (ok) v = __ldg(reinterpret_cast<const uint2*>(src));
+        w[2 * g] = v.x; w[2 * g + 1] = v.y;
+      } else if constexpr (kXBits == 4) {
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (ok) v = __ldg(reinterpret_cast<const uint4*>(src));
+        w[4 * g] = v.x; w[4 * g + 1] = v.y; w[4 * g + 2] = v.z; w[4 * g + 3] = v.w;
+      } else {
+#pragma unroll
+        for (int i = 0; i < 3; ++i) w[3 * g + i] = ok ? __ldg(reinterpret_cast<const uint32_t*>(src) + i) : 0u;
+      }
+    }
+  }
+}
+
+template <int kXBits, bool kChunkInTap>
 __global__ void __launch_bounds__(kThreads, 1)
 conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ Params p) {
-  constexpr int kGB = 4 * kXBits;  // bytes of one 32-channel input group
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t sbase = smem_u32(smem);
   const uint32_t s_a = sbase;
   const uint32_t s_b = sbase + p.off_b;
-  uint8_t* stg = smem + p.off_stg;
   EpiChan* epi = reinterpret_cast<EpiChan*>(smem + p.off_epi);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + p.off_bar);
   // barrier slots: full[0..S), empty[0..S), tfull[2], tempty[2], final
@@ -305,12 +367,12 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
-      mbar_init(b_full + 8 * s, kProdWarps * 32 + 1);
+      mbar_init(b_full + 8 * s, kProdWarps + 1);  // one arrive per producer warp + TMA
       mbar_init(b_empty + 8 * s, 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(b_tfull + 8 * b, 1);
-      mbar_init(b_tempty + 8 * b, kEpiThreads);
+      mbar_init(b_tempty + 8 * b, kEpiWarps);     // one arrive per epilogue warp
     }
     mbar_init(b_final, 1);
     *abort_flag = 0;
@@ -336,23 +398,28 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       const uint32_t idesc = idesc_e4m3(BN);
+      // descriptors of stage 0, k-step 0; later stages / sub-tiles / k-steps add
+      // (byte offset >> 4) to the 14-bit start-address field (shared addresses < 2^18)
+      const uint64_t da0 = sdesc_sw128(s_a), db0 = sdesc_sw128(s_b);
       uint32_t it = 0, lt = 0;
       bool ok = true;
       for (int t = first_tile; t < p.total_tiles && ok; t += tile_stride, ++lt) {
         const uint32_t buf = lt & 1;
         if (!mbar_wait(b_tempty + 8 * buf, ((lt >> 1) & 1) ^ 1, abort_flag)) { ok = false; break; }
         tc_fence_after();
-        const uint32_t d_tmem = tmem_base + buf * (uint32_t)BN;
+        const uint32_t d0 = tmem_base + buf * 2u * (uint32_t)BN;  // sub-tile 0; sub-tile 1 at +BN
         for (int q = 0; q < nk; ++q, ++it) {
           const uint32_t s = it % S, ph = (it / S) & 1;
           if (!mbar_wait(b_full + 8 * s, ph, abort_flag)) { ok = false; break; }
           tc_fence_after();
-          const uint32_t a0 = s_a + s * (BM * BK);
-          const uint32_t b0 = s_b + s * stage_b_bytes;
+          const uint64_t da = da0 + ((s * kStageA) >> 4);
+          const uint64_t db = db0 + ((s * stage_b_bytes) >> 4);
 #pragma unroll
-          for (int kk = 0; kk < BK / 32; ++kk)
-            mma_e4m3(d_tmem, sdesc_sw128(a0 + 32 * kk), sdesc_sw128(b0 + 32 * kk), idesc,
-                     (q > 0 || kk > 0) ? 1u : 0u);
+          for (int kk = 0; kk < BK / 32; ++kk) {
+            const uint32_t acc = (q > 0 || kk > 0) ? 1u : 0u;
+            mma_e4m3(d0, da + 2 * kk, db + 2 * kk, idesc, acc);
+            mma_e4m3(d0 + BN, da + (kSubA >> 4) + 2 * kk, db + 2 * kk, idesc, acc);
+          }
           mma_commit(b_empty + 8 * s);
         }
         if (ok) mma_commit(b_tfull + 8 * buf);
@@ -380,117 +447,76 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
     }
   } else if (warp >= kWarpProd0) {
     // ------------------------------------------------------------ activation producers
-    const int row = threadIdx.x - kWarpProd0 * 32;  // 0..127: tile row owned by this thread
-    const uint32_t stg_row = smem_u32(stg) + row * p.stg_stride;
-    const uint32_t stg_slot_bytes = (uint32_t)BM * p.stg_stride;
+    const int row = threadIdx.x - kWarpProd0 * 32;  // 0..255: tile row owned by this thread
+    const int sub = row >> 7, r7 = row & 7;
+    uint8_t* arow = smem + sub * kSubA + (row & 127) * BK;
     int my_tiles = 0;
     for (int t = first_tile; t < p.total_tiles; t += tile_stride) ++my_tiles;
-    const int total_chunks = my_tiles * nk;
+    const int total = my_tiles * nk;
 
-    // issue cursor
-    int i_tile = first_tile, i_q = 0, issued = 0;
-    const uint8_t* xbase = nullptr;
-    int hb = 0, wb = 0, H = 1, W = 1;
-    bool rvalid = false;
-    int tr = 0, ts = 0, tc0 = 0;  // tap state of the next 32-channel group
-    const uint8_t* xdummy = p.jobs[0].x;
-
-    auto issue = [&]() {
-      if (i_q == 0) {
-        const TileInfo ti = tile_info(p, i_tile);
-        const ConvJobDev& jb = p.jobs[ti.job];
-        const int m = ti.mt * BM + row;
-        rvalid = m < jb.m_total;
-        const int mm = rvalid ? m : 0;
-        const int hw = jb.ho * jb.wo;
-        const int img = mm / hw;
-        const int rem = mm - img * hw;
-        const int ho = rem / jb.wo, wo = rem - (rem / jb.wo) * jb.wo;
-        hb = ho * p.stride - p.pad;
-        wb = wo * p.stride - p.pad;
-        H = jb.h;
-        W = jb.w;
-        xbase = jb.x + (int64_t)img * jb.h * jb.w * p.x_row_bytes;
-        tr = 0; ts = 0; tc0 = 0;
-      }
-      const uint32_t slot = stg_row + (uint32_t)(issued % kDepth) * stg_slot_bytes;
-#pragma unroll
-      for (int g = 0; g < BK / 32; ++g) {
-        const int k0 = i_q * BK + 32 * g;
-        bool ok = false;
-        const uint8_t* src = xdummy;
-        if (k0 < p.k_total) {
-          const int hi = hb + tr, wi = wb + ts;
-          ok = rvalid && hi >= 0 && hi < H && wi >= 0 && wi < W;
-          if (ok) src = xbase + ((int64_t)hi * W + wi) * p.x_row_bytes + (tc0 >> 5) * kGB;
-          tc0 += 32;
-          if (tc0 == p.cin) { tc0 = 0; if (++ts == p.kw) { ts = 0; ++tr; } }
-        }
-        const uint32_t dst = slot + g * kGB;
-        if constexpr (kGB == 8) {
-          cp_async<8>(dst, src, ok);
-        } else if constexpr (kGB == 16) {
-          cp_async<16>(dst, src, ok);
-        } else {  // 12 bytes: three 4-byte copies
-          cp_async<4>(dst, src, ok);
-          cp_async<4>(dst + 4, src + 4, ok);
-          cp_async<4>(dst + 8, src + 8, ok);
-        }
-      }
-      ++issued;
-      if (++i_q == nk) { i_q = 0; i_tile += tile_stride; }
+    RowCursor<kXBits> rc{};
+    int l_tile = first_tile, l_q = 0;  // load cursor (runs kDepth chunks ahead)
+    auto start_tile = [&](int t) {
+      const TileInfo ti = tile_info(p, t);
+      const ConvJobDev& jb = p.jobs[ti.job];
+      const int m = ti.mt * BM + row;
+      rc.valid = m < jb.m_total;
+      const int mm = rc.valid ? m : 0;
+      const int hw = jb.ho * jb.wo;
+      const int img = mm / hw;
+      const int rem = mm - img * hw;
+      const int ho = rem / jb.wo, wo = rem - (rem / jb.wo) * jb.wo;
+      rc.hb = ho * p.stride - p.pad;
+      rc.wb = wo * p.stride - p.pad;
+      rc.H = jb.h;
+      rc.W = jb.w;
+      rc.xbase = jb.x + (int64_t)img * jb.h * jb.w * p.x_row_bytes;
+      rc.tr = 0; rc.ts = 0; rc.tc0 = 0;
     };
-
-    for (int d = 0; d < kDepth; ++d) {
-      if (issued < total_chunks) issue();
-      cp_async_commit();
-    }
+    auto load_next = [&](uint32_t (&w)[4 * kXBits]) {
+      if (l_q == 0) start_tile(l_tile);
+      load_chunk<kXBits, kChunkInTap>(p, rc, l_q, w);
+      if (++l_q == nk) { l_q = 0; l_tile += tile_stride; }
+    };
     bool ok = true;
-    for (int c = 0; c < total_chunks; ++c) {
-      cp_async_wait<kDepth - 1>();
+    auto consume = [&](int c, const uint32_t (&w)[4 * kXBits]) -> bool {
       const uint32_t s = c % S, ph = (c / S) & 1;
-      if (!mbar_wait(b_empty + 8 * s, ph ^ 1, abort_flag)) { ok = false; break; }
-      // unpack this thread's row: 4 groups of 32 codes -> 128 E4M3 bytes (raw byte = code)
-      const uint8_t* src = stg + (size_t)(c % kDepth) * BM * p.stg_stride + (size_t)row * p.stg_stride;
-      uint32_t words[4 * kXBits];
-      if constexpr (kXBits == 2) {  // 8-byte reads: stride 40 keeps 16 lanes conflict-free
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const uint2 v = reinterpret_cast<const uint2*>(src)[i];
-          words[2 * i] = v.x; words[2 * i + 1] = v.y;
-        }
-      } else if constexpr (kXBits == 3) {  // 4-byte reads: stride 52 (13 words, odd)
-#pragma unroll
-        for (int i = 0; i < 12; ++i) words[i] = reinterpret_cast<const uint32_t*>(src)[i];
-      } else {  // 16-byte reads: stride 80 keeps 8 lanes conflict-free
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const uint4 v = reinterpret_cast<const uint4*>(src)[i];
-          words[4 * i + 0] = v.x; words[4 * i + 1] = v.y; words[4 * i + 2] = v.z; words[4 * i + 3] = v.w;
-        }
-      }
-      uint8_t* arow = smem + (size_t)s * (BM * BK) + (size_t)row * BK;
+      if (!mbar_wait(b_empty + 8 * s, ph ^ 1, abort_flag)) return false;
+      uint8_t* dst = arow + (size_t)s * kStageA;
 #pragma unroll
       for (int g = 0; g < 4; ++g) {
         uint32_t o[8];
-        unpack_group_bytes<kXBits>(words + g * kXBits, o);
-        const int j0 = (2 * g) ^ (row & 7), j1 = (2 * g + 1) ^ (row & 7);
-        *reinterpret_cast<uint4*>(arow + 16 * j0) = make_uint4(o[0], o[1], o[2], o[3]);
-        *reinterpret_cast<uint4*>(arow + 16 * j1) = make_uint4(o[4], o[5], o[6], o[7]);
+        unpack_group_bytes<kXBits>(w + g * kXBits, o);  // raw E4M3 byte = code
+        *reinterpret_cast<uint4*>(dst + 16 * ((2 * g) ^ r7)) = make_uint4(o[0], o[1], o[2], o[3]);
+        *reinterpret_cast<uint4*>(dst + 16 * ((2 * g + 1) ^ r7)) = make_uint4(o[4], o[5], o[6], o[7]);
       }
-      fence_proxy_async();
-      mbar_arrive(b_full + 8 * s);
-      if (issued < total_chunks) issue();
-      cp_async_commit();
+      fence_proxy_async();  // this thread's generic-proxy stores -> visible to the MMA
+      __syncwarp();
+      if (lane == 0) mbar_arrive(b_full + 8 * s);
+      return true;
+    };
+    uint32_t w0[4 * kXBits], w1[4 * kXBits], w2[4 * kXBits];
+    if (total > 0) load_next(w0);
+    if (total > 1) load_next(w1);
+    if (total > 2) load_next(w2);
+    for (int c = 0; c < total && ok; c += 3) {
+      if (!consume(c, w0)) { ok = false; break; }
+      if (c + 3 < total) load_next(w0);
+      if (c + 1 < total) {
+        if (!consume(c + 1, w1)) { ok = false; break; }
+        if (c + 4 < total) load_next(w1);
+      }
+      if (c + 2 < total) {
+        if (!consume(c + 2, w2)) { ok = false; break; }
+        if (c + 5 < total) load_next(w2);
+      }
     }
-    cp_async_wait<0>();
     if (!ok) fail(abort_flag, p.status);
   } else {
     // ------------------------------------------------------------ epilogue (warps 0..E-1)
-    const int quarter = warp & 3;   // TMEM lane quarter this warp may read
-    const int half = warp >> 2;     // this warp takes every other 32-column group
-    const int e = quarter * 32 + lane;  // tile row = TMEM lane
-    const int et = threadIdx.x;         // 0 .. kEpiThreads-1
+    const int quarter = warp & 3;      // TMEM lane quarter this warp may read
+    const int sub0 = warp >> 2;        // with 8 warps: one sub-tile each; with 4: both
+    const int et = threadIdx.x;        // 0 .. kEpiThreads-1
     const uint32_t lane_base = tmem_base + ((uint32_t)(quarter * 32) << 16);
     const int4* epf = reinterpret_cast<const int4*>(epi + 256);  // fast-path table after epi[256]
     uint32_t lt = 0;
@@ -531,80 +557,82 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       if (!mbar_wait(b_tfull + 8 * buf, (lt >> 1) & 1, abort_flag)) { ok = false; break; }
       tc_fence_after();
 
-      const int m = ti.mt * BM + e;
-      const bool valid = m < jb.m_total;
-      const int mm = valid ? m : 0;
-      const int hw = jb.ho * jb.wo;
-      const int img = mm / hw;
-      const int rem = mm - img * hw;
-      const int ho = rem / jb.wo, wo = rem - (rem / jb.wo) * jb.wo;
-      uint8_t* yrow = jb.y + (int64_t)mm * p.y_row_bytes;
-      const uint8_t* srow = nullptr;
-      if (p.has_skip) {
-        const int sh = ho / p.upsample, sw = wo / p.upsample;
-        srow = jb.skip + (((int64_t)img * jb.skip_h + sh) * jb.skip_w + sw) * p.skip_row_bytes;
-      }
-      const uint32_t tcol = buf * (uint32_t)BN;
-      for (int g0 = 32 * half; g0 < BN; g0 += 32 * (kEpiWarps / 4)) {
-        const int ncols = (BN - g0) < 32 ? (BN - g0) : 32;  // warp-uniform
-        uint32_t v[32];
-        uint32_t r16[16];
-        __syncwarp();
-        tmem_ld16(lane_base + tcol + g0, r16);
+      for (int sub = sub0; sub < 2; sub += kEpiWarps / 4) {
+        const int m = ti.mt * BM + sub * 128 + quarter * 32 + lane;
+        const bool valid = m < jb.m_total;
+        const int mm = valid ? m : 0;
+        const int hw = jb.ho * jb.wo;
+        const int img = mm / hw;
+        const int rem = mm - img * hw;
+        const int ho = rem / jb.wo, wo = rem - (rem / jb.wo) * jb.wo;
+        uint8_t* yrow = jb.y + (int64_t)mm * p.y_row_bytes;
+        const uint8_t* srow = nullptr;
+        if (p.has_skip) {
+          const int sh = ho / p.upsample, sw = wo / p.upsample;
+          srow = jb.skip + (((int64_t)img * jb.skip_h + sh) * jb.skip_w + sw) * p.skip_row_bytes;
+        }
+        const uint32_t tcol = buf * 2u * (uint32_t)BN + sub * (uint32_t)BN;
+        for (int g0 = 0; g0 < BN; g0 += 32) {
+          const int ncols = (BN - g0) < 32 ? (BN - g0) : 32;  // warp-uniform
+          uint32_t v[32];
+          uint32_t r16[16];
+          __syncwarp();
+          tmem_ld16(lane_base + tcol + g0, r16);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) v[i] = r16[i];
-        if (ncols == 32) tmem_ld16(lane_base + tcol + g0 + 16, r16);
-        tmem_wait_ld();
+          for (int i = 0; i < 16; ++i) v[i] = r16[i];
+          if (ncols == 32) tmem_ld16(lane_base + tcol + g0 + 16, r16);
+          tmem_wait_ld();
 #pragma unroll
-        for (int i = 0; i < 16; ++i) v[16 + i] = (ncols == 32) ? r16[i] : 0u;
-        if (!valid) continue;
-        const int ch0 = ti.nt * BN + g0;
-        if (mode == 1) {
-          uint32_t gw[8];
-          switch (out_bits) {
-            case 2: fast_requant_group<2>(v, epf + g0, qmax, gw); break;
-            case 3: fast_requant_group<3>(v, epf + g0, qmax, gw); break;
-            case 4: fast_requant_group<4>(v, epf + g0, qmax, gw); break;
-            default: fast_requant_group<8>(v, epf + g0, qmax, gw); break;
-          }
-          store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
-        } else if (mode == 2) {
-          int32_t* yr = reinterpret_cast<int32_t*>(yrow) + ch0;
-          const bool full = ncols == 32 && ch0 + 32 <= p.cout;
+          for (int i = 0; i < 16; ++i) v[16 + i] = (ncols == 32) ? r16[i] : 0u;
+          if (!valid) continue;
+          const int ch0 = ti.nt * BN + g0;
+          if (mode == 1) {
+            uint32_t gw[8];
+            switch (out_bits) {
+              case 2: fast_requant_group<2>(v, epf + g0, qmax, gw); break;
+              case 3: fast_requant_group<3>(v, epf + g0, qmax, gw); break;
+              case 4: fast_requant_group<4>(v, epf + g0, qmax, gw); break;
+              default: fast_requant_group<8>(v, epf + g0, qmax, gw); break;
+            }
+            store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
+          } else if (mode == 2) {
+            int32_t* yr = reinterpret_cast<int32_t*>(yrow) + ch0;
+            const bool full = ncols == 32 && ch0 + 32 <= p.cout;
 #pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            int32_t o[4];
-#pragma unroll
-            for (int k = 0; k < 4; ++k)
-              o[k] = add_sat(__float2int_rn(__uint_as_float(v[4 * q + k]) * 262144.0f), epi[g0 + 4 * q + k].bias);
-            if (full) {
-              reinterpret_cast<int4*>(yr)[q] = make_int4(o[0], o[1], o[2], o[3]);
-            } else {
+            for (int q = 0; q < 8; ++q) {
+              int32_t o[4];
 #pragma unroll
               for (int k = 0; k < 4; ++k)
-                if (4 * q + k < ncols && ch0 + 4 * q + k < p.cout) yr[4 * q + k] = o[k];
-            }
-          }
-        } else {
-          uint32_t vv[32];  // local copies: only this rare path goes through the stack
-          int32_t oo[32];
+                o[k] = add_sat(__float2int_rn(__uint_as_float(v[4 * q + k]) * 262144.0f), epi[g0 + 4 * q + k].bias);
+              if (full) {
+                reinterpret_cast<int4*>(yr)[q] = make_int4(o[0], o[1], o[2], o[3]);
+              } else {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) vv[i] = v[i];
-          general_epilogue(p, vv, epi + g0, srow, ch0, ncols, oo);
-          if (out_bits == 32) {
-            int32_t* yr = reinterpret_cast<int32_t*>(yrow) + ch0;
-            for (int i = 0; i < 32; ++i)
-              if (i < ncols && ch0 + i < p.cout) yr[i] = oo[i];
+                for (int k = 0; k < 4; ++k)
+                  if (4 * q + k < ncols && ch0 + 4 * q + k < p.cout) yr[4 * q + k] = o[k];
+              }
+            }
           } else {
-            uint32_t gw[8];
-            pack_group_vals(oo, out_bits, gw);
-            store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
+            uint32_t vv[32];  // local copies: only this rare path goes through the stack
+            int32_t oo[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) vv[i] = v[i];
+            general_epilogue(p, vv, epi + g0, srow, ch0, ncols, oo);
+            if (out_bits == 32) {
+              int32_t* yr = reinterpret_cast<int32_t*>(yrow) + ch0;
+              for (int i = 0; i < 32; ++i)
+                if (i < ncols && ch0 + i < p.cout) yr[i] = oo[i];
+            } else {
+              uint32_t gw[8];
+              pack_group_vals(oo, out_bits, gw);
+              store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
+            }
           }
         }
       }
-      __syncwarp();
       tc_fence_before();
-      mbar_arrive(b_tempty + 8 * buf);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(b_tempty + 8 * buf);
     }
     if (!ok) fail(abort_flag, p.status);
   }
@@ -639,10 +667,10 @@ static EncodeTiledFn get_encode_fn(std::string* err) {
   return fn;
 }
 
-template <int kXBits>
+template <int kXBits, bool kChunkInTap>
 static int launch_bits(const Params& prm, const CUtensorMap& map, int grid, size_t smem,
                        cudaStream_t stream, std::string* err) {
-  auto kern = conv_tc_kernel<kXBits>;
+  auto kern = conv_tc_kernel<kXBits, kChunkInTap>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) { *err = std::string("cudaFuncSetAttribute: ") + cudaGetErrorString(e); return 3; }
   kern<<<grid, kThreads, smem, stream>>>(map, prm);
@@ -677,27 +705,21 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   prm.upsample = a.upsample; prm.scale_main = a.scale_main; prm.has_skip = a.has_skip;
   prm.bn = BN;
   prm.status = a.status;
-  // shared memory plan
-  // staging row strides chosen so cp.async writes and the row reads hit distinct banks
-  const int stg_stride = (a.x_bits == 2) ? 40 : (a.x_bits == 3 ? 52 : 80);
-  const size_t stage_bytes = (size_t)BM * BK + (size_t)BN * BK;
-  const size_t stg_bytes = (size_t)kDepth * BM * stg_stride;
+  // shared memory plan: stages of (256 x 128 A bytes + BN x 128 B bytes)
+  const size_t stage_bytes = (size_t)kStageA + (size_t)BN * BK;
   const size_t epi_bytes = 256 * sizeof(EpiChan) + 256 * sizeof(int4);
   const size_t bar_bytes = 8 * (2 * kMaxStages + 5) + 16;
   const size_t budget = 232448 - 1024;  // max dynamic smem per block minus alignment slack
-  const size_t fixed = stg_bytes + epi_bytes + bar_bytes;
-  int stages = (int)((budget - fixed) / stage_bytes);
+  int stages = (int)((budget - epi_bytes - bar_bytes) / stage_bytes);
   if (stages > kMaxStages) stages = kMaxStages;
   if (stages < 2) { *err = "conv_tc: shared memory plan does not fit"; return 2; }
   prm.stages = stages;
-  prm.stg_stride = stg_stride;
-  prm.off_b = (uint32_t)(stages * BM * BK);
-  prm.off_stg = prm.off_b + (uint32_t)(stages * BN * BK);
-  prm.off_epi = prm.off_stg + (uint32_t)stg_bytes;
+  prm.off_b = (uint32_t)(stages * kStageA);
+  prm.off_epi = prm.off_b + (uint32_t)(stages * BN * BK);
   prm.off_bar = prm.off_epi + (uint32_t)epi_bytes;
   const size_t smem = 1024 + prm.off_bar + bar_bytes;
   int cols = 32;
-  while (cols < 2 * BN) cols *= 2;
+  while (cols < 4 * BN) cols *= 2;  // two buffers x two sub-tiles x BN fp32 columns
   prm.tmem_cols = cols;
 
   EncodeTiledFn enc = get_encode_fn(err);
@@ -716,10 +738,14 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int grid = tiles < sms ? tiles : sms;
+  const bool in_tap = (a.cin % BK) == 0;
   switch (a.x_bits) {
-    case 2: return launch_bits<2>(prm, map, grid, smem, stream, err);
-    case 3: return launch_bits<3>(prm, map, grid, smem, stream, err);
-    case 4: return launch_bits<4>(prm, map, grid, smem, stream, err);
+    case 2: return in_tap ? launch_bits<2, true>(prm, map, grid, smem, stream, err)
+                          : launch_bits<2, false>(prm, map, grid, smem, stream, err);
+    case 3: return in_tap ? launch_bits<3, true>(prm, map, grid, smem, stream, err)
+                          : launch_bits<3, false>(prm, map, grid, smem, stream, err);
+    case 4: return in_tap ? launch_bits<4, true>(prm, map, grid, smem, stream, err)
+                          : launch_bits<4, false>(prm, map, grid, smem, stream, err);
     default: *err = "conv_tc: activation bits must be 2, 3 or 4"; return 2;
   }
 }

@@ -53,7 +53,7 @@ WeightGeom weight_geom(int32_t cout, int32_t kh, int32_t kw, int32_t cin) {
   g.cout = cout; g.kh = kh; g.kw = kw; g.cin = cin;
   g.k_total = kh * kw * cin;
   g.k_pad = (g.k_total + 127) / 128 * 128;
-  g.bn = cout <= 128 ? (cout + 15) / 16 * 16 : 128;  // N tile of the tensor-core kernel
+  g.bn = cout <= 256 ? (cout + 15) / 16 * 16 : 256;  // N tile of the tensor-core kernel
   g.cout_pad = (cout + g.bn - 1) / g.bn * g.bn;
   g.e4m3_bytes = (size_t)g.cout_pad * g.k_pad;
   g.i16_offset = (g.e4m3_bytes + 255) / 256 * 256;
@@ -280,6 +280,7 @@ aqd_status aqd_conv_int_grouped(const aqd_conv_job* jobs, int32_t njobs, const a
   const int64_t max_a = (1LL << a.x_bits) - 1;
   const int64_t max_w = max_abs_weight(w->w_bits, w->w_format);
   const int64_t bound = (int64_t)g.k_total * max_a * max_w;
+  a.acc_bound = bound;
   const bool tc_ok = a.x_bits <= 4 && max_w <= 15 && (a.cin % 32) == 0 && bound < (1LL << 24);
   const bool direct_ok = bound < (1LL << 31);
   int path = tc_ok ? 1 : 2;

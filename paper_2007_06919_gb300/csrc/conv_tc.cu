@@ -33,20 +33,34 @@
 namespace aqd {
 namespace tc {
 
-constexpr int BM = 256;            // output pixels per tile: two M=128 sub-tiles sharing B
+// A tile is kSub M=128 sub-tiles (each one MMA per k-step) sharing every weight stage.
+// The MMA rate is full only for N = 256 (measured: two N=128 MMAs sharing B reach ~72%,
+// one N=128 MMA ~31%), so tiles are 128 x 256 (kSub = 1) for 256-channel layers.
+#ifndef AQD_SUBTILES
+#define AQD_SUBTILES 1
+#endif
+constexpr int kSub = AQD_SUBTILES;
+constexpr int BM = 128 * kSub;     // output pixels per tile
 constexpr int kSubA = 128 * 128;   // bytes of one sub-tile's A operand per stage
-constexpr int kStageA = 2 * kSubA; // bytes of A per stage
+constexpr int kStageA = kSub * kSubA; // bytes of A per stage
 constexpr int BK = 128;            // K bytes per stage
 #ifndef AQD_EPI_WARPS
-#define AQD_EPI_WARPS 4
+#define AQD_EPI_WARPS 8
 #endif
 constexpr int kEpiWarps = AQD_EPI_WARPS;  // 4 or 8
-static_assert(kEpiWarps == 4 || kEpiWarps == 8, "epilogue warps");
+static_assert(kEpiWarps == 4 || kEpiWarps == 8, "epilogue warps: 4 or 8");
 constexpr int kEpiThreads = kEpiWarps * 32;
+#ifndef AQD_TMA_WARPS
+#define AQD_TMA_WARPS 1
+#endif
+#ifndef AQD_WAIT_HINT_NS
+#define AQD_WAIT_HINT_NS 0
+#endif
+constexpr int kTmaWarps = AQD_TMA_WARPS;  // weight-loading warps, alternating K chunks
 constexpr int kWarpMma = kEpiWarps;
 constexpr int kWarpTma = kEpiWarps + 1;
-constexpr int kWarpProd0 = kEpiWarps + 2;
-constexpr int kProdWarps = 8;      // one thread per tile row
+constexpr int kWarpProd0 = kEpiWarps + 1 + kTmaWarps;
+constexpr int kProdWarps = 4 * kSub;  // one thread per tile row
 constexpr int kThreads = (kWarpProd0 + kProdWarps) * 32;
 constexpr int kMaxStages = 8;
 constexpr uint64_t kTimeoutNs = 1000000000ull;  // 1 s per wait
@@ -64,6 +78,7 @@ struct Params {
   const int8_t* skip_d;
   int32_t upsample, scale_main, has_skip;
   int32_t bn, stages, tmem_cols;
+  int32_t acc_small;  // |acc| < 2^22 guaranteed by K * max|x| * max|w|
   uint32_t off_b, off_epi, off_bar;
   uint32_t* status;
 };
@@ -101,17 +116,56 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
       : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
   return ok != 0;
 }
+// try_wait that lets the hardware suspend the thread (up to `ns`) until the phase
+// completes, instead of returning at once: waiting warps then take no issue slots
+__device__ __forceinline__ bool mbar_try_sleep(uint32_t bar, uint32_t parity, uint32_t ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok) : "r"(bar), "r"(parity), "r"(ns) : "memory");
+  return ok != 0;
+}
+
+// Non-blocking test of a phase. The MMA-issuing thread polls with this: measured on
+// sm_103a, a try_wait in a thread with tcgen05.mma in flight costs ~165 cycles even when
+// the phase has completed, a test_wait ~13.
+__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
+  return ok != 0;
+}
+__device__ __noinline__ bool mbar_poll_slow(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+  // a few cheap tests first (short waits), then the suspending try_wait so a long wait
+  // does not take issue slots from the other warps of this SM sub-partition
+  for (int i = 0; i < 8; ++i)
+    if (mbar_test(bar, parity)) return true;
+  const uint64_t deadline = globaltimer() + kTimeoutNs;
+  for (uint32_t spin = 1;; ++spin) {
+    if (mbar_try(bar, parity)) return true;
+    if ((spin & 15) == 0) {
+      if (*abort_flag) return false;
+      if (globaltimer() > deadline) return false;
+    }
+  }
+}
+__device__ __forceinline__ bool mbar_poll(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+  return mbar_test(bar, parity) || mbar_poll_slow(bar, parity, abort_flag);
+}
 
 // Bounded wait: false if the deadline passed or another role aborted.
 __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
-  uint64_t deadline = 0;
+  const uint64_t deadline = globaltimer() + kTimeoutNs;
   for (uint32_t spin = 1;; ++spin) {
-    if (mbar_try(bar, parity)) return true;
+    if (AQD_WAIT_HINT_NS > 0 ? mbar_try_sleep(bar, parity, AQD_WAIT_HINT_NS) : mbar_try(bar, parity)) return true;
     if ((spin & 63) == 0) {
       if (*abort_flag) return false;
-      uint64_t now = globaltimer();
-      if (deadline == 0) deadline = now + kTimeoutNs;
-      else if (now > deadline) return false;
+      if (globaltimer() > deadline) return false;
     }
   }
 }
@@ -258,19 +312,46 @@ __device__ __noinline__ void general_epilogue(const Params& p, const uint32_t* v
   }
 }
 
-// Fast requant of 32 accumulators of one row into one packed group (no skip, R >= 33):
-// u = sat32(acc + bias), y = clamp((mulhi(u, M0) + 2^(R-33)) >> (R-32), 0, 2^k - 1),
-// each code OR-ed straight into its word of the packed layout.
+// 1.5 * 2^23: adding it to an integer-valued float |x| < 2^22 puts x in the low mantissa bits
+constexpr float kMagic = 12582912.0f;
+constexpr uint32_t kMagicBits = 0x4B400000u;
+
+// Fastest requant (no skip, R >= 33, |acc| < 2^22, |bias| <= 2^30): the accumulator float
+// acc * 2^-18 becomes the int32 acc + 0x4B400000 with one FMA; c.x holds bias - 0x4B400000,
+// so one add gives acc + bias exactly (no int32 overflow under the stated bounds).
 template <int kOut>
-__device__ __forceinline__ void fast_requant_group(const uint32_t* v, const int4* f, int qmax, uint32_t gw[8]) {
+__device__ __forceinline__ void magic_requant_group(const uint32_t* v, const int4* f, int qmax, uint32_t gw[8]) {
 #pragma unroll
   for (int w = 0; w < 8; ++w) gw[w] = 0u;
 #pragma unroll
   for (int i = 0; i < 32; ++i) {
     const int4 c = f[i];
-    const int32_t acc = __float2int_rn(__uint_as_float(v[i]) * 262144.0f);  // exact integer
-    const int32_t u = add_sat(acc, c.x);
+    const int32_t u = __float_as_int(__fmaf_rn(__uint_as_float(v[i]), 262144.0f, kMagic)) + c.x;
     const uint32_t y = (uint32_t)min(max((__mulhi(u, c.y) + c.z) >> c.w, 0), qmax);
+    if constexpr (kOut == 3) {
+      gw[i / 16] |= (y & 3u) << (8 * (i % 4) + 2 * ((i % 16) / 4));
+      gw[2] |= (y >> 2) << (8 * (i % 4) + i / 4);
+    } else {
+      constexpr int q = 32 / kOut;
+      gw[i / q] |= y << (8 * (i % 4) + kOut * ((i % q) / 4));
+    }
+  }
+}
+
+// Fast requant of 32 accumulators of one row into one packed group (no skip, R >= 33,
+// any bias): u = sat32(acc + bias), y = clamp((mulhi(u, M0) + 2^(R-33)) >> (R-32), 0, 2^k-1).
+template <int kOut>
+__device__ __forceinline__ void fast_requant_group(const uint32_t* v, const EpiChan* ep, int g0, int qmax,
+                                                   uint32_t gw[8]) {
+#pragma unroll
+  for (int w = 0; w < 8; ++w) gw[w] = 0u;
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    const EpiChan c = ep[g0 + i];
+    const int32_t acc = __float2int_rn(__uint_as_float(v[i]) * 262144.0f);  // exact integer
+    const int32_t u = add_sat(acc, c.bias);
+    const int r = c.r;
+    const uint32_t y = (uint32_t)min(max((__mulhi(u, c.m0) + (1 << (r - 33))) >> (r - 32), 0), qmax);
     if constexpr (kOut == 3) {
       gw[i / 16] |= (y & 3u) << (8 * (i % 4) + 2 * ((i % 16) / 4));
       gw[2] |= (y >> 2) << (8 * (i % 4) + i / 4);
@@ -343,8 +424,10 @@ __device__ __forceinline__ void load_chunk(const Params& p, RowCursor<kXBits>& r
 template <int kXBits, bool kChunkInTap>
 __global__ void __launch_bounds__(kThreads, 1)
 conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ Params p) {
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  // align by pointer arithmetic on the shared array itself (no integer round trip), so the
+  // compiler keeps every access through `smem` in the shared state space (lds/sts)
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const uint32_t sbase = smem_u32(smem);
   const uint32_t s_a = sbase;
   const uint32_t s_b = sbase + p.off_b;
@@ -383,7 +466,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
                  ::"r"(smem_u32(tmem_slot)), "r"(p.tmem_cols) : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
-  if (warp == kWarpTma && lane == 0)
+  if (warp >= kWarpTma && warp < kWarpTma + kTmaWarps && lane == 0)
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmap_w) : "memory");
   tc_fence_before();
   __syncthreads();
@@ -400,27 +483,33 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       const uint32_t idesc = idesc_e4m3(BN);
       // descriptors of stage 0, k-step 0; later stages / sub-tiles / k-steps add
       // (byte offset >> 4) to the 14-bit start-address field (shared addresses < 2^18)
+      // the descriptors' high words are constant; stages / sub-tiles / k-steps only move the
+      // 14-bit start-address field in the low word (shared addresses < 2^18, no carry)
       const uint64_t da0 = sdesc_sw128(s_a), db0 = sdesc_sw128(s_b);
-      uint32_t it = 0, lt = 0;
+      const uint32_t a_lo0 = (uint32_t)da0, b_lo0 = (uint32_t)db0;
+      const uint32_t a_hi = (uint32_t)(da0 >> 32), b_hi = (uint32_t)(db0 >> 32);
+      uint32_t it = 0, lt = 0, s = 0, ph = 0;
       bool ok = true;
       for (int t = first_tile; t < p.total_tiles && ok; t += tile_stride, ++lt) {
         const uint32_t buf = lt & 1;
-        if (!mbar_wait(b_tempty + 8 * buf, ((lt >> 1) & 1) ^ 1, abort_flag)) { ok = false; break; }
+        if (!mbar_poll(b_tempty + 8 * buf, ((lt >> 1) & 1) ^ 1, abort_flag)) { ok = false; break; }
         tc_fence_after();
-        const uint32_t d0 = tmem_base + buf * 2u * (uint32_t)BN;  // sub-tile 0; sub-tile 1 at +BN
+        const uint32_t d0 = tmem_base + buf * (uint32_t)(kSub * BN);  // sub-tile j at +j*BN
         for (int q = 0; q < nk; ++q, ++it) {
-          const uint32_t s = it % S, ph = (it / S) & 1;
-          if (!mbar_wait(b_full + 8 * s, ph, abort_flag)) { ok = false; break; }
+          if (!mbar_poll(b_full + 8 * s, ph, abort_flag)) { ok = false; break; }
           tc_fence_after();
-          const uint64_t da = da0 + ((s * kStageA) >> 4);
-          const uint64_t db = db0 + ((s * stage_b_bytes) >> 4);
+          const uint32_t a_lo = a_lo0 + ((s * kStageA) >> 4);
+          const uint32_t b_lo = b_lo0 + ((s * stage_b_bytes) >> 4);
 #pragma unroll
           for (int kk = 0; kk < BK / 32; ++kk) {
             const uint32_t acc = (q > 0 || kk > 0) ? 1u : 0u;
-            mma_e4m3(d0, da + 2 * kk, db + 2 * kk, idesc, acc);
-            mma_e4m3(d0 + BN, da + (kSubA >> 4) + 2 * kk, db + 2 * kk, idesc, acc);
+            const uint64_t db = ((uint64_t)b_hi << 32) | (b_lo + 2 * kk);
+#pragma unroll
+            for (int j = 0; j < kSub; ++j)
+              mma_e4m3(d0 + j * BN, ((uint64_t)a_hi << 32) | (a_lo + j * (kSubA >> 4) + 2 * kk), db, idesc, acc);
           }
           mma_commit(b_empty + 8 * s);
+          if (++s == (uint32_t)S) { s = 0; ph ^= 1; }
         }
         if (ok) mma_commit(b_tfull + 8 * buf);
       }
@@ -429,15 +518,18 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       mma_commit(b_final);
       if (!mbar_wait(b_final, 0, abort_flag)) fail(abort_flag, p.status);
     }
-  } else if (warp == kWarpTma) {
-    // ------------------------------------------------------------ weight loader (TMA)
+  } else if (warp >= kWarpTma && warp < kWarpTma + kTmaWarps) {
+    // ------------------------------------------------------------ weight loaders (TMA)
+    // One thread of each TMA warp issues every kTmaWarps-th chunk: a thread sustains
+    // about one tensor copy at a time, so two threads keep two copies in flight.
+    const int tw = warp - kWarpTma;
     if (lane == 0) {
-      uint32_t it = 0;
+      uint32_t it = 0, s = 0, ph = 0;
       bool ok = true;
       for (int t = first_tile; t < p.total_tiles && ok; t += tile_stride) {
         const TileInfo ti = tile_info(p, t);
-        for (int q = 0; q < nk; ++q, ++it) {
-          const uint32_t s = it % S, ph = (it / S) & 1;
+        for (int q = 0; q < nk; ++q, ++it, s = (s + 1 == (uint32_t)S) ? 0 : s + 1, ph ^= (s == 0)) {
+          if ((int)(it % kTmaWarps) != tw) continue;
           if (!mbar_wait(b_empty + 8 * s, ph ^ 1, abort_flag)) { ok = false; break; }
           mbar_arrive_expect_tx(b_full + 8 * s, stage_b_bytes);
           tma_load_2d(s_b + s * stage_b_bytes, &tmap_w, q * BK, ti.nt * BN, b_full + 8 * s);
@@ -514,11 +606,15 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
     if (!ok) fail(abort_flag, p.status);
   } else {
     // ------------------------------------------------------------ epilogue (warps 0..E-1)
-    const int quarter = warp & 3;      // TMEM lane quarter this warp may read
-    const int sub0 = warp >> 2;        // with 8 warps: one sub-tile each; with 4: both
-    const int et = threadIdx.x;        // 0 .. kEpiThreads-1
+    // Warp w reads TMEM lanes 32*(w%4).. (the hardware lane quarter of its warp index).
+    // Warp group gi = w/4 takes sub-tiles / column groups in turn, so with 8 warps two
+    // warps share each lane quarter.
+    const int quarter = warp & 3;
+    const int gi = warp >> 2;
+    constexpr int kGroups = kEpiWarps / 4;
+    const int et = threadIdx.x;  // 0 .. kEpiThreads-1
     const uint32_t lane_base = tmem_base + ((uint32_t)(quarter * 32) << 16);
-    const int4* epf = reinterpret_cast<const int4*>(epi + 256);  // fast-path table after epi[256]
+    const int4* epf = reinterpret_cast<const int4*>(epi + 256);  // per-column fast constants
     uint32_t lt = 0;
     bool ok = true;
     const int out_bits = p.out_bits;
@@ -527,72 +623,98 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       const TileInfo ti = tile_info(p, t);
       const ConvJobDev& jb = p.jobs[ti.job];
       named_bar(1, kEpiThreads);
-      // Per-column constants of this tile's level. Fast path when the total requant shift
-      // R = 31 + shift is >= 33: y = (mulhi(u, M0) + 2^(R-33)) >> (R-32) equals
-      // rhu(u * M0, R) exactly (the low product word cannot carry into the result).
-      int fast = 1;
+      // Per-column constants of this tile's level. The 32-bit fast path applies when the
+      // total requant shift R = 31 + shift is >= 33 (then y = (mulhi(u, M0) + 2^(R-33)) >>
+      // (R-32) equals rhu(u * M0, R): the low product word cannot carry into the result)
+      // and |bias| <= 2^30 (acc + bias cannot leave int32 when |acc| < 2^24).
+      int fast_req = 1, small_bias = 1;
       for (int col = et; col < 256; col += kEpiThreads) {
         const int ch = ti.nt * BN + col;
         EpiChan ec{};
-        int4 ef = make_int4(0, 0, 0, 1);
+        int4 ef = make_int4((int32_t)(0u - kMagicBits), 0, 0, 1);
         if (col < BN && ch < p.cout) {
           const int64_t idx = (int64_t)jb.level * p.cout + ch;
           ec.bias = p.bias ? p.bias[idx] : 0;
+          const bool sb = ec.bias >= -(1 << 30) && ec.bias <= (1 << 30);
+          small_bias &= sb;
+          ef.x = (int32_t)((uint32_t)ec.bias - kMagicBits);
           if (out_bits != 32) {
             ec.m0 = p.m0[idx];
             const int r = 31 + p.shift[idx];
             ec.r = (int8_t)r;
-            if (r >= 33) ef = make_int4(ec.bias, ec.m0, 1 << (r - 33), r - 32);
-            else fast = 0;
+            if (r >= 33 && sb) { ef.y = ec.m0; ef.z = 1 << (r - 33); ef.w = r - 32; }
+            else fast_req = 0;
           }
           if (p.has_skip) { ec.c = p.skip_c[idx]; ec.d = p.skip_d[idx]; }
         }
         epi[col] = ec;
         reinterpret_cast<int4*>(epi + 256)[col] = ef;
       }
-      fast = named_bar_and(1, kEpiThreads, fast);
-      // 0: general int64 epilogue, 1: fast requant to codes, 2: int32 output, no skip
-      const int mode = p.has_skip ? 0 : (out_bits == 32 ? 2 : (fast ? 1 : 0));
+      fast_req = named_bar_and(1, kEpiThreads, fast_req);
+      small_bias = named_bar_and(1, kEpiThreads, small_bias);
+      // 0: general int64 epilogue; 1: fast requant to codes; 2: int32 output, no skip
+      const int mode = p.has_skip ? 0 : (out_bits == 32 ? 2 : (fast_req ? 1 : 0));
+      const bool magic = p.acc_small && (mode == 2 ? small_bias : fast_req);
       const uint32_t buf = lt & 1;
       if (!mbar_wait(b_tfull + 8 * buf, (lt >> 1) & 1, abort_flag)) { ok = false; break; }
       tc_fence_after();
 
-      for (int sub = sub0; sub < 2; sub += kEpiWarps / 4) {
-        const int m = ti.mt * BM + sub * 128 + quarter * 32 + lane;
-        const bool valid = m < jb.m_total;
-        const int mm = valid ? m : 0;
-        const int hw = jb.ho * jb.wo;
-        const int img = mm / hw;
-        const int rem = mm - img * hw;
-        const int ho = rem / jb.wo, wo = rem - (rem / jb.wo) * jb.wo;
-        uint8_t* yrow = jb.y + (int64_t)mm * p.y_row_bytes;
-        const uint8_t* srow = nullptr;
-        if (p.has_skip) {
-          const int sh = ho / p.upsample, sw = wo / p.upsample;
-          srow = jb.skip + (((int64_t)img * jb.skip_h + sh) * jb.skip_w + sw) * p.skip_row_bytes;
-        }
-        const uint32_t tcol = buf * 2u * (uint32_t)BN + sub * (uint32_t)BN;
-        for (int g0 = 0; g0 < BN; g0 += 32) {
-          const int ncols = (BN - g0) < 32 ? (BN - g0) : 32;  // warp-uniform
-          uint32_t v[32];
+      // this warp's (sub-tile, 32-column group) units, two per TMEM wait
+      const int ngrp = (BN + 31) / 32;
+      const int nunits = kSub * ngrp;
+      for (int u0 = gi; u0 < nunits; u0 += 2 * kGroups) {
+        const int u1 = u0 + kGroups;
+        const bool two = u1 < nunits;  // warp-uniform
+        uint32_t va[32], vb[32];
+        int subA = u0 / ngrp, g0A = (u0 % ngrp) * 32;
+        int subB = two ? u1 / ngrp : 0, g0B = two ? (u1 % ngrp) * 32 : 0;
+        const int ncA = (BN - g0A) < 32 ? (BN - g0A) : 32;
+        const int ncB = (BN - g0B) < 32 ? (BN - g0B) : 32;
+        __syncwarp();
+        {
           uint32_t r16[16];
-          __syncwarp();
-          tmem_ld16(lane_base + tcol + g0, r16);
+          const uint32_t ca = lane_base + buf * (uint32_t)(kSub * BN) + subA * (uint32_t)BN + g0A;
+          tmem_ld16(ca, r16);
 #pragma unroll
-          for (int i = 0; i < 16; ++i) v[i] = r16[i];
-          if (ncols == 32) tmem_ld16(lane_base + tcol + g0 + 16, r16);
-          tmem_wait_ld();
+          for (int i = 0; i < 16; ++i) va[i] = r16[i];
+          if (ncA == 32) tmem_ld16(ca + 16, r16);
 #pragma unroll
-          for (int i = 0; i < 16; ++i) v[16 + i] = (ncols == 32) ? r16[i] : 0u;
-          if (!valid) continue;
+          for (int i = 0; i < 16; ++i) va[16 + i] = (ncA == 32) ? r16[i] : 0u;
+        }
+        if (two) {
+          uint32_t r16[16];
+          const uint32_t cb = lane_base + buf * (uint32_t)(kSub * BN) + subB * (uint32_t)BN + g0B;
+          tmem_ld16(cb, r16);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) vb[i] = r16[i];
+          if (ncB == 32) tmem_ld16(cb + 16, r16);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) vb[16 + i] = (ncB == 32) ? r16[i] : 0u;
+        }
+        tmem_wait_ld();
+        for (int h = 0; h < (two ? 2 : 1); ++h) {
+          const uint32_t* v = h ? vb : va;
+          const int sub = h ? subB : subA, g0 = h ? g0B : g0A, ncols = h ? ncB : ncA;
+          const int m = ti.mt * BM + sub * 128 + quarter * 32 + lane;
+          if (m >= jb.m_total) continue;
+          uint8_t* yrow = jb.y + (int64_t)m * p.y_row_bytes;
           const int ch0 = ti.nt * BN + g0;
           if (mode == 1) {
             uint32_t gw[8];
-            switch (out_bits) {
-              case 2: fast_requant_group<2>(v, epf + g0, qmax, gw); break;
-              case 3: fast_requant_group<3>(v, epf + g0, qmax, gw); break;
-              case 4: fast_requant_group<4>(v, epf + g0, qmax, gw); break;
-              default: fast_requant_group<8>(v, epf + g0, qmax, gw); break;
+            if (magic) {
+              switch (out_bits) {
+                case 2: magic_requant_group<2>(v, epf + g0, qmax, gw); break;
+                case 3: magic_requant_group<3>(v, epf + g0, qmax, gw); break;
+                case 4: magic_requant_group<4>(v, epf + g0, qmax, gw); break;
+                default: magic_requant_group<8>(v, epf + g0, qmax, gw); break;
+              }
+            } else {
+              switch (out_bits) {
+                case 2: fast_requant_group<2>(v, epi, g0, qmax, gw); break;
+                case 3: fast_requant_group<3>(v, epi, g0, qmax, gw); break;
+                case 4: fast_requant_group<4>(v, epi, g0, qmax, gw); break;
+                default: fast_requant_group<8>(v, epi, g0, qmax, gw); break;
+              }
             }
             store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
           } else if (mode == 2) {
@@ -602,8 +724,11 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
             for (int q = 0; q < 8; ++q) {
               int32_t o[4];
 #pragma unroll
-              for (int k = 0; k < 4; ++k)
-                o[k] = add_sat(__float2int_rn(__uint_as_float(v[4 * q + k]) * 262144.0f), epi[g0 + 4 * q + k].bias);
+              for (int k = 0; k < 4; ++k) {
+                const float f = __uint_as_float(v[4 * q + k]);
+                o[k] = magic ? __float_as_int(__fmaf_rn(f, 262144.0f, kMagic)) + epf[g0 + 4 * q + k].x
+                             : add_sat(__float2int_rn(f * 262144.0f), epi[g0 + 4 * q + k].bias);
+              }
               if (full) {
                 reinterpret_cast<int4*>(yr)[q] = make_int4(o[0], o[1], o[2], o[3]);
               } else {
@@ -613,6 +738,15 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
               }
             }
           } else {
+            const uint8_t* srow = nullptr;
+            if (p.has_skip) {
+              const int hw = jb.ho * jb.wo;
+              const int img = m / hw;
+              const int rem = m - img * hw;
+              const int ho = rem / jb.wo, wo = rem - (rem / jb.wo) * jb.wo;
+              const int sh = ho / p.upsample, sw = wo / p.upsample;
+              srow = jb.skip + (((int64_t)img * jb.skip_h + sh) * jb.skip_w + sw) * p.skip_row_bytes;
+            }
             uint32_t vv[32];  // local copies: only this rare path goes through the stack
             int32_t oo[32];
 #pragma unroll
@@ -704,8 +838,9 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   prm.skip_c = a.skip_c; prm.skip_d = a.skip_d;
   prm.upsample = a.upsample; prm.scale_main = a.scale_main; prm.has_skip = a.has_skip;
   prm.bn = BN;
+  prm.acc_small = a.acc_bound < (1LL << 22) ? 1 : 0;
   prm.status = a.status;
-  // shared memory plan: stages of (256 x 128 A bytes + BN x 128 B bytes)
+  // shared memory plan: stages of (BM x 128 A bytes + BN x 128 B bytes)
   const size_t stage_bytes = (size_t)kStageA + (size_t)BN * BK;
   const size_t epi_bytes = 256 * sizeof(EpiChan) + 256 * sizeof(int4);
   const size_t bar_bytes = 8 * (2 * kMaxStages + 5) + 16;
@@ -719,7 +854,7 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   prm.off_bar = prm.off_epi + (uint32_t)epi_bytes;
   const size_t smem = 1024 + prm.off_bar + bar_bytes;
   int cols = 32;
-  while (cols < 4 * BN) cols *= 2;  // two buffers x two sub-tiles x BN fp32 columns
+  while (cols < 2 * kSub * BN) cols *= 2;  // two buffers x kSub sub-tiles x BN fp32 columns
   prm.tmem_cols = cols;
 
   EncodeTiledFn enc = get_encode_fn(err);

@@ -37,6 +37,7 @@ struct ConvArgs {
   const uint8_t* w_e4m3;  // [cout_pad][k_pad] E4M3 sign-magnitude bytes (|w| <= 15)
   const int16_t* w_i16;   // [cout][k_total] signed integers
   int32_t cout_pad, k_total, k_pad, bn;
+  int64_t acc_bound;      // K * max|x| * max|w|: bound on |accumulator|
   uint32_t* status;       // device status word
 };
 

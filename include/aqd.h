@@ -135,7 +135,8 @@ aqd_status aqd_device_status(aqd_stream_t stream, int32_t* code);
 /* Diagnostics: force the convolution kernel (0 = automatic choice, 1 = tensor-core
  * kernel when the shape allows it, 2 = CUDA-core kernel); returns the previous setting,
  * or -1 for an unknown value. aqd_last_conv_path() reports the kernel the calling
- * thread's last successful conv call used (1 tensor core, 2 CUDA core, 0 none yet). */
+ * thread's last successful conv call used (1 tensor core unpacking in-kernel, 2 CUDA core,
+ * 3 tensor core fed from the expanded workspace, 0 none yet). */
 int32_t aqd_set_conv_path(int32_t path);
 int32_t aqd_last_conv_path(void);
 
@@ -162,11 +163,13 @@ aqd_status aqd_conv_prepare_weights(const void* w_packed, const aqd_conv_weights
 
 /* One convolution y = epilogue(conv(x, w)) at the given level of the tables.
  * skip may be NULL (no skip; sp ignored). y->bits selects the output: 2/3/4/8 codes or
- * 32 (int32, rq->m0/shift unused). rq may be NULL only for 32-bit outputs (no bias). */
+ * 32 (int32, rq->m0/shift unused). rq may be NULL only for 32-bit outputs (no bias).
+ * workspace (device, 256-byte aligned, owned by the caller, contents not preserved) may be
+ * NULL; see aqd_conv_workspace_bytes. Results are identical with and without it. */
 aqd_status aqd_conv_int(const aqd_tensor* x, const aqd_conv_weights* w, int32_t stride,
                         int32_t pad, int32_t level, const aqd_requant_params* rq,
                         const aqd_tensor* skip, const aqd_skip_params* sp, aqd_tensor* y,
-                        aqd_stream_t stream);
+                        void* workspace, size_t ws_bytes, aqd_stream_t stream);
 
 /* The same convolution over up to 8 jobs with shared weights in ONE launch: the shared
  * detector head applied to every FPN level, each with its own level's BN row. All jobs
@@ -174,7 +177,16 @@ aqd_status aqd_conv_int(const aqd_tensor* x, const aqd_conv_weights* w, int32_t 
 aqd_status aqd_conv_int_grouped(const aqd_conv_job* jobs, int32_t njobs,
                                 const aqd_conv_weights* w, int32_t stride, int32_t pad,
                                 const aqd_requant_params* rq, const aqd_skip_params* sp,
-                                aqd_stream_t stream);
+                                void* workspace, size_t ws_bytes, aqd_stream_t stream);
+
+/* Workspace that lets a convolution expand its packed input codes once into a zero-padded
+ * byte image (one byte per code: sum over jobs of n*(h+2*pad)*(w+2*pad)*cin bytes) and feed
+ * the tensor cores from it with TMA tile loads, instead of unpacking every code once per
+ * kernel tap inside the convolution. Returns 0 when this path does not apply (stride != 1,
+ * cin % 128 != 0, codes or weights wider than 4 bits); a NULL or smaller workspace passed
+ * to the conv calls then selects the in-kernel unpacking path. */
+size_t aqd_conv_workspace_bytes(const aqd_conv_job* jobs, int32_t njobs,
+                                const aqd_conv_weights* w, int32_t stride, int32_t pad);
 
 /* ---- elementwise ------------------------------------------------------------------ */
 

@@ -55,7 +55,8 @@ class _Job(ctypes.Structure):
 EXPORTS = ["aqd_row_bytes", "aqd_quantize_multiplier", "aqd_status_string", "aqd_last_error",
            "aqd_device_status", "aqd_set_conv_path", "aqd_last_conv_path", "aqd_pack_codes",
            "aqd_unpack_codes", "aqd_conv_weights_bytes", "aqd_conv_prepare_weights", "aqd_conv_int",
-           "aqd_conv_int_grouped", "aqd_requant", "aqd_residual_add_int", "aqd_maxpool_codes"]
+           "aqd_conv_int_grouped", "aqd_conv_workspace_bytes", "aqd_requant", "aqd_residual_add_int",
+           "aqd_maxpool_codes"]
 
 _lib = None
 
@@ -93,9 +94,11 @@ def load(build_if_missing: bool = True):
     L.aqd_conv_prepare_weights.argtypes = [vp, ctypes.POINTER(_Weights), vp, ctypes.c_size_t, vp]
     L.aqd_conv_int.argtypes = [ctypes.POINTER(_Tensor), ctypes.POINTER(_Weights), i32, i32, i32,
                                ctypes.POINTER(_Requant), ctypes.POINTER(_Tensor), ctypes.POINTER(_Skip),
-                               ctypes.POINTER(_Tensor), vp]
+                               ctypes.POINTER(_Tensor), vp, ctypes.c_size_t, vp]
     L.aqd_conv_int_grouped.argtypes = [ctypes.POINTER(_Job), i32, ctypes.POINTER(_Weights), i32, i32,
-                                       ctypes.POINTER(_Requant), ctypes.POINTER(_Skip), vp]
+                                       ctypes.POINTER(_Requant), ctypes.POINTER(_Skip), vp, ctypes.c_size_t, vp]
+    L.aqd_conv_workspace_bytes.restype = ctypes.c_size_t
+    L.aqd_conv_workspace_bytes.argtypes = [ctypes.POINTER(_Job), i32, ctypes.POINTER(_Weights), i32, i32]
     L.aqd_requant.argtypes = [ctypes.POINTER(_Tensor), ctypes.POINTER(_Requant), i32, ctypes.POINTER(_Tensor), vp]
     L.aqd_residual_add_int.argtypes = [ctypes.POINTER(_Tensor), ctypes.POINTER(_Tensor), ctypes.POINTER(_Skip),
                                        ctypes.POINTER(_Requant), i32, ctypes.POINTER(_Tensor), vp]
@@ -274,35 +277,65 @@ def conv_out_hw(h, w, kh, kw, stride, pad):
     return (h + 2 * pad - kh) // stride + 1, (w + 2 * pad - kw) // stride + 1
 
 
+def _ws(workspace: torch.Tensor | None):
+    if workspace is None:
+        return None, 0
+    return _ptr(workspace), workspace.numel() * workspace.element_size()
+
+
 def conv_int(x: DTensor, w: ConvWeights, stride: int, pad: int, y: DTensor, *, level: int = 0,
              rq: RequantParams | None = None, skip: DTensor | None = None, sp: SkipParams | None = None,
-             stream=None) -> DTensor:
+             workspace: torch.Tensor | None = None, stream=None) -> DTensor:
     xc, yc = x.ct(), y.ct()
     rqc = rq.c() if rq is not None else None
     skc = skip.ct() if skip is not None else None
     spc = sp.cs() if sp is not None else None
+    wsp, wsb = _ws(workspace)
     _check(load().aqd_conv_int(ctypes.byref(xc), ctypes.byref(w.desc), stride, pad, level,
                                ctypes.byref(rqc) if rqc is not None else None,
                                ctypes.byref(skc) if skc is not None else None,
-                               ctypes.byref(spc) if spc is not None else None, ctypes.byref(yc), _stream(stream)),
+                               ctypes.byref(spc) if spc is not None else None, ctypes.byref(yc), wsp, wsb,
+                               _stream(stream)),
            "aqd_conv_int")
     return y
 
 
-def conv_int_grouped(jobs, w: ConvWeights, stride: int, pad: int, *, rq: RequantParams | None = None,
-                     sp: SkipParams | None = None, stream=None):
-    """jobs: list of (x: DTensor, y: DTensor, skip: DTensor | None, level: int)."""
+def _jobs(jobs):
     arr = (_Job * len(jobs))()
     for i, (x, y, skip, level) in enumerate(jobs):
         arr[i].x = x.ct()
         arr[i].y = y.ct()
         arr[i].skip = skip.ct() if skip is not None else _Tensor(0, 0, 0, 0, 0, None)
         arr[i].level = level
+    return arr
+
+
+def conv_workspace_bytes(jobs, w: ConvWeights, stride: int, pad: int) -> int:
+    """Bytes of the expanded-activation workspace for these jobs (0: path not applicable)."""
+    return int(load().aqd_conv_workspace_bytes(_jobs(jobs), len(jobs), ctypes.byref(w.desc), stride, pad))
+
+
+def workspace_for(jobs, w: ConvWeights, stride: int, pad: int, device="cuda") -> torch.Tensor | None:
+    """A 256-byte aligned workspace of the right size, or None when the path does not apply."""
+    n = conv_workspace_bytes(jobs, w, stride, pad)
+    if n == 0:
+        return None
+    buf = torch.empty(n + 256, dtype=torch.uint8, device=device)
+    off = (-buf.data_ptr()) % 256
+    return buf[off:off + n]
+
+
+def conv_int_grouped(jobs, w: ConvWeights, stride: int, pad: int, *, rq: RequantParams | None = None,
+                     sp: SkipParams | None = None, workspace: torch.Tensor | None = None, stream=None):
+    """jobs: list of (x: DTensor, y: DTensor, skip: DTensor | None, level: int)."""
+    arr = _jobs(jobs)
     rqc = rq.c() if rq is not None else None
     spc = sp.cs() if sp is not None else None
+    wsp, wsb = _ws(workspace)
     _check(load().aqd_conv_int_grouped(arr, len(jobs), ctypes.byref(w.desc), stride, pad,
                                        ctypes.byref(rqc) if rqc is not None else None,
-                                       ctypes.byref(spc) if spc is not None else None, _stream(stream)),
+                                       ctypes.byref(spc) if spc is not None else None, wsp, wsb,
+                                       _stream(stream)),
            "aqd_conv_int_grouped")
 
 

@@ -202,9 +202,35 @@ aqd_status aqd_conv_prepare_weights(const void* w_packed, const aqd_conv_weights
   return st ? fail((aqd_status)st, err) : AQD_OK;
 }
 
+// Rows (of cin bytes) of the expanded-activation workspace, or 0 if that path does not apply.
+static int64_t flat_rows(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w, int32_t stride,
+                         int32_t pad) {
+  if (!jobs || njobs <= 0 || njobs > kMaxJobs || !w) return 0;
+  if (stride != 1 || pad < 0 || w->cin <= 0 || w->cin % 128 != 0 || w->w_bits < 2 || w->w_bits > 4) return 0;
+  if (w->w_format != AQD_W_TWOS && w->w_format != AQD_W_ODD) return 0;
+  const int64_t max_w = max_abs_weight(w->w_bits, w->w_format);
+  if (max_w > 15) return 0;
+  int64_t rows = 0;
+  for (int j = 0; j < njobs; ++j) {
+    const aqd_tensor& x = jobs[j].x;
+    if (x.bits < 2 || x.bits > 4 || x.c != w->cin || x.n <= 0 || x.h <= 0 || x.w <= 0) return 0;
+    const int64_t k = (int64_t)w->kh * w->kw * w->cin;
+    if (k * ((1LL << x.bits) - 1) * max_w >= (1LL << 24)) return 0;
+    rows += (int64_t)x.n * (x.h + 2 * pad) * (x.w + 2 * pad);
+  }
+  return rows < (1LL << 31) ? rows : 0;
+}
+
+size_t aqd_conv_workspace_bytes(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
+                                int32_t stride, int32_t pad) {
+  const int64_t rows = flat_rows(jobs, njobs, w, stride, pad);
+  return rows > 0 ? (size_t)rows * (size_t)w->cin : 0;
+}
+
 aqd_status aqd_conv_int_grouped(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
                                 int32_t stride, int32_t pad, const aqd_requant_params* rq,
-                                const aqd_skip_params* sp, aqd_stream_t stream) {
+                                const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
+                                aqd_stream_t stream) {
   std::string err;
   if (!jobs || njobs <= 0 || njobs > kMaxJobs) return fail(AQD_ERR_INVALID, "njobs must be 1..8");
   if (!check_weights(w, &err)) return fail(AQD_ERR_INVALID, err);
@@ -286,17 +312,30 @@ aqd_status aqd_conv_int_grouped(const aqd_conv_job* jobs, int32_t njobs, const a
   int path = tc_ok ? 1 : 2;
   if (g_forced_path == 1 && tc_ok) path = 1;
   if (g_forced_path == 2) path = 2;
+  // expanded-activation path when a large enough, aligned workspace is supplied
+  a.ws = nullptr;
+  a.ws_rows = 0;
+  if (path == 1 && workspace) {
+    if ((reinterpret_cast<uintptr_t>(workspace) & 255) != 0)
+      return fail(AQD_ERR_INVALID, "workspace must be 256-byte aligned");
+    const int64_t rows = flat_rows(jobs, njobs, w, stride, pad);
+    if (rows > 0 && (size_t)rows * (size_t)w->cin <= ws_bytes) {
+      a.ws = static_cast<uint8_t*>(workspace);
+      a.ws_rows = (int64_t)(ws_bytes / (size_t)w->cin);
+    }
+  }
   if (path == 2 && !direct_ok) return fail(AQD_ERR_UNSUPPORTED, "accumulator bound exceeds int32");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   int rc = path == 1 ? launch_conv_tc(a, st, &err) : launch_conv_direct(a, st, &err);
   if (rc) return fail((aqd_status)rc, err);
-  g_last_path = path;
+  g_last_path = (path == 1 && a.ws) ? 3 : path;
   return AQD_OK;
 }
 
 aqd_status aqd_conv_int(const aqd_tensor* x, const aqd_conv_weights* w, int32_t stride, int32_t pad,
                         int32_t level, const aqd_requant_params* rq, const aqd_tensor* skip,
-                        const aqd_skip_params* sp, aqd_tensor* y, aqd_stream_t stream) {
+                        const aqd_skip_params* sp, aqd_tensor* y, void* workspace, size_t ws_bytes,
+                        aqd_stream_t stream) {
   if (!x || !y) return fail(AQD_ERR_INVALID, "x and y must not be NULL");
   aqd_conv_job job{};
   job.x = *x;
@@ -306,7 +345,7 @@ aqd_status aqd_conv_int(const aqd_tensor* x, const aqd_conv_weights* w, int32_t 
     if (!skip->data) return fail(AQD_ERR_INVALID, "skip->data is NULL");
   }
   job.level = level;
-  return aqd_conv_int_grouped(&job, 1, w, stride, pad, rq, sp, stream);
+  return aqd_conv_int_grouped(&job, 1, w, stride, pad, rq, sp, workspace, ws_bytes, stream);
 }
 
 static aqd_status elementwise(const aqd_tensor* a, const aqd_tensor* b, const aqd_skip_params* sp,

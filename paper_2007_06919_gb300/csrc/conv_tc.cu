@@ -62,6 +62,12 @@ constexpr int kWarpTma = kEpiWarps + 1;
 constexpr int kWarpProd0 = kEpiWarps + 1 + kTmaWarps;
 constexpr int kProdWarps = 4 * kSub;  // one thread per tile row
 constexpr int kThreads = (kWarpProd0 + kProdWarps) * 32;
+// The expanded-activation ("flat") variant has no producer warps: TMA loads both operands,
+// two boxes per K chunk. One issuing thread sustains about one box per ~700 cycles
+// (measured), so that variant spreads the chunks over kTmaWarpsFlat threads.
+constexpr int kTmaWarpsFlat = 3;
+__host__ __device__ constexpr int tma_warps(bool flat) { return flat ? kTmaWarpsFlat : kTmaWarps; }
+__host__ __device__ constexpr int threads_for(bool flat) { return flat ? (kWarpTma + kTmaWarpsFlat) * 32 : kThreads; }
 constexpr int kMaxStages = 8;
 constexpr uint64_t kTimeoutNs = 1000000000ull;  // 1 s per wait
 
@@ -79,6 +85,7 @@ struct Params {
   int32_t upsample, scale_main, has_skip;
   int32_t bn, stages, tmem_cols;
   int32_t acc_small;  // |acc| < 2^22 guaranteed by K * max|x| * max|w|
+  int32_t cin_chunks; // cin / 128 (flat path)
   uint32_t off_b, off_epi, off_bar;
   uint32_t* status;
 };
@@ -277,6 +284,17 @@ __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.
 struct TileInfo {
   int job, mt, nt;
 };
+// Flat path: M tile mt of a job covers virtual rows [v0, v0 + 128) of image img, where the
+// virtual grid holds the output rows at the padded input width wp (stride 1).
+struct FlatTile {
+  int img, v0;
+};
+__device__ __forceinline__ FlatTile flat_tile(const ConvJobDev& jb, int mt) {
+  FlatTile f;
+  f.img = mt / jb.tpi;
+  f.v0 = (mt - f.img * jb.tpi) * 128;
+  return f;
+}
 __device__ __forceinline__ TileInfo tile_info(const Params& p, int t) {
   int j = 0;
 #pragma unroll 1
@@ -421,9 +439,11 @@ __device__ __forceinline__ void load_chunk(const Params& p, RowCursor<kXBits>& r
   }
 }
 
-template <int kXBits, bool kChunkInTap>
-__global__ void __launch_bounds__(kThreads, 1)
-conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ Params p) {
+template <int kXBits, bool kChunkInTap, bool kFlat>
+__global__ void __launch_bounds__(threads_for(kFlat), 1)
+conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_a,
+               const __grid_constant__ Params p) {
+  constexpr int kTma = tma_warps(kFlat);
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // align by pointer arithmetic on the shared array itself (no integer round trip), so the
   // compiler keeps every access through `smem` in the shared state space (lds/sts)
@@ -450,7 +470,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
-      mbar_init(b_full + 8 * s, kProdWarps + 1);  // one arrive per producer warp + TMA
+      mbar_init(b_full + 8 * s, kFlat ? 1 : kProdWarps + 1);  // per producer warp + TMA
       mbar_init(b_empty + 8 * s, 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -468,6 +488,8 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
   }
   if (warp >= kWarpTma && warp < kWarpTma + kTmaWarps && lane == 0)
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmap_w) : "memory");
+  if (kFlat && warp >= kWarpTma && warp < kWarpTma + kTma && lane == 0)
+    asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmap_a) : "memory");
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -518,7 +540,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       mma_commit(b_final);
       if (!mbar_wait(b_final, 0, abort_flag)) fail(abort_flag, p.status);
     }
-  } else if (warp >= kWarpTma && warp < kWarpTma + kTmaWarps) {
+  } else if (warp >= kWarpTma && warp < kWarpTma + kTma) {
     // ------------------------------------------------------------ weight loaders (TMA)
     // One thread of each TMA warp issues every kTmaWarps-th chunk: a thread sustains
     // about one tensor copy at a time, so two threads keep two copies in flight.
@@ -529,15 +551,26 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       for (int t = first_tile; t < p.total_tiles && ok; t += tile_stride) {
         const TileInfo ti = tile_info(p, t);
         for (int q = 0; q < nk; ++q, ++it, s = (s + 1 == (uint32_t)S) ? 0 : s + 1, ph ^= (s == 0)) {
-          if ((int)(it % kTmaWarps) != tw) continue;
+          if ((int)(it % kTma) != tw) continue;
           if (!mbar_wait(b_empty + 8 * s, ph ^ 1, abort_flag)) { ok = false; break; }
-          mbar_arrive_expect_tx(b_full + 8 * s, stage_b_bytes);
+          if constexpr (kFlat) {
+            // A: 128 consecutive rows of the padded byte image, shifted by the tap (r, s)
+            const ConvJobDev& jb = p.jobs[ti.job];
+            const FlatTile ft = flat_tile(jb, ti.mt);
+            const int tap = q / p.cin_chunks, cb = q - tap * p.cin_chunks;
+            const int r = tap / p.kw, sx = tap - r * p.kw;
+            const int row = jb.row_off + ft.img * jb.hp * jb.wp + ft.v0 + r * jb.wp + sx;
+            mbar_arrive_expect_tx(b_full + 8 * s, stage_b_bytes + kStageA);
+            tma_load_2d(s_a + s * kStageA, &tmap_a, cb * BK, row, b_full + 8 * s);
+          } else {
+            mbar_arrive_expect_tx(b_full + 8 * s, stage_b_bytes);
+          }
           tma_load_2d(s_b + s * stage_b_bytes, &tmap_w, q * BK, ti.nt * BN, b_full + 8 * s);
         }
       }
       if (!ok) fail(abort_flag, p.status);
     }
-  } else if (warp >= kWarpProd0) {
+  } else if (!kFlat && warp >= kWarpProd0) {
     // ------------------------------------------------------------ activation producers
     const int row = threadIdx.x - kWarpProd0 * 32;  // 0..255: tile row owned by this thread
     const int sub = row >> 7, r7 = row & 7;
@@ -695,8 +728,17 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
         for (int h = 0; h < (two ? 2 : 1); ++h) {
           const uint32_t* v = h ? vb : va;
           const int sub = h ? subB : subA, g0 = h ? g0B : g0A, ncols = h ? ncB : ncA;
-          const int m = ti.mt * BM + sub * 128 + quarter * 32 + lane;
-          if (m >= jb.m_total) continue;
+          int m;  // output pixel index within the job
+          if constexpr (kFlat) {
+            const FlatTile ft = flat_tile(jb, ti.mt);
+            const int v = ft.v0 + quarter * 32 + lane;  // virtual row at the padded width
+            const int ho = v / jb.wp, wo = v - (v / jb.wp) * jb.wp;
+            if (v >= jb.vimg || wo >= jb.wo) continue;  // junk column or past the image
+            m = (ft.img * jb.ho + ho) * jb.wo + wo;
+          } else {
+            m = ti.mt * BM + sub * 128 + quarter * 32 + lane;
+            if (m >= jb.m_total) continue;
+          }
           uint8_t* yrow = jb.y + (int64_t)m * p.y_row_bytes;
           const int ch0 = ti.nt * BN + g0;
           if (mode == 1) {
@@ -780,6 +822,49 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
   }
 }
 
+// ---------------------------------------------------------------- activation expansion
+
+// Writes every job's input as a zero-padded byte image: workspace row
+// row_off + (img * hp + hp_i) * wp + wp_i holds the cin E4M3 bytes (raw byte = code) of
+// input pixel (img, hp_i - pad, wp_i - pad), or zeros in the padding border.
+struct ExpandArgs {
+  ConvJobDev jobs[kMaxJobs];
+  int32_t njobs, cin, pad;
+  int64_t x_row_bytes;
+  int64_t total_rows;
+  uint8_t* ws;
+};
+
+template <int kXBits>
+__global__ void __launch_bounds__(256) expand_kernel(const __grid_constant__ ExpandArgs a) {
+  constexpr int kGB = 4 * kXBits;
+  const int groups = a.cin >> 5;
+  const int64_t t = (int64_t)blockIdx.x * 256 + threadIdx.x;
+  if (t >= a.total_rows * groups) return;
+  const int64_t row = t / groups;
+  const int g = (int)(t - row * groups);
+  int j = 0;
+#pragma unroll 1
+  while (j + 1 < a.njobs && row >= a.jobs[j + 1].row_off) ++j;
+  const ConvJobDev& jb = a.jobs[j];
+  const int64_t local = row - jb.row_off;
+  const int64_t plane = (int64_t)jb.hp * jb.wp;
+  const int img = (int)(local / plane);
+  const int rem = (int)(local - img * plane);
+  const int hi = rem / jb.wp - a.pad, wi = rem - (rem / jb.wp) * jb.wp - a.pad;
+  uint32_t o[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+  if (hi >= 0 && hi < jb.h && wi >= 0 && wi < jb.w) {
+    const uint8_t* src = jb.x + (((int64_t)img * jb.h + hi) * jb.w + wi) * a.x_row_bytes + g * kGB;
+    uint32_t w[kXBits];
+#pragma unroll
+    for (int i = 0; i < kXBits; ++i) w[i] = __ldg(reinterpret_cast<const uint32_t*>(src) + i);
+    unpack_group_bytes<kXBits>(w, o);
+  }
+  uint4* dst = reinterpret_cast<uint4*>(a.ws + row * a.cin + g * 32);
+  dst[0] = make_uint4(o[0], o[1], o[2], o[3]);
+  dst[1] = make_uint4(o[4], o[5], o[6], o[7]);
+}
+
 // ---------------------------------------------------------------- host side
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
@@ -801,13 +886,13 @@ static EncodeTiledFn get_encode_fn(std::string* err) {
   return fn;
 }
 
-template <int kXBits, bool kChunkInTap>
-static int launch_bits(const Params& prm, const CUtensorMap& map, int grid, size_t smem,
-                       cudaStream_t stream, std::string* err) {
-  auto kern = conv_tc_kernel<kXBits, kChunkInTap>;
+template <int kXBits, bool kChunkInTap, bool kFlat>
+static int launch_bits(const Params& prm, const CUtensorMap& map, const CUtensorMap& map_a, int grid,
+                       size_t smem, cudaStream_t stream, std::string* err) {
+  auto kern = conv_tc_kernel<kXBits, kChunkInTap, kFlat>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) { *err = std::string("cudaFuncSetAttribute: ") + cudaGetErrorString(e); return 3; }
-  kern<<<grid, kThreads, smem, stream>>>(map, prm);
+  kern<<<grid, threads_for(kFlat), smem, stream>>>(map, map_a, prm);
   e = cudaGetLastError();
   if (e != cudaSuccess) { *err = std::string("conv_tc launch: ") + cudaGetErrorString(e); return 3; }
   return 0;
@@ -821,11 +906,30 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   const int BN = a.bn;
   prm.njobs = a.njobs;
   prm.n_tiles = a.cout_pad / BN;
+  // flat path: the activations are expanded into the workspace first (stride 1,
+  // cin % 128 == 0; the API checks both before passing a workspace)
+  const bool flat = a.ws != nullptr;
   int tiles = 0;
+  int64_t rows = 0;
   for (int j = 0; j < a.njobs; ++j) {
     prm.jobs[j] = a.jobs[j];
     prm.jobs[j].tile_begin = tiles;
-    tiles += ((a.jobs[j].m_total + BM - 1) / BM) * prm.n_tiles;
+    if (flat) {
+      ConvJobDev& jb = prm.jobs[j];
+      jb.hp = jb.h + 2 * a.pad;
+      jb.wp = jb.w + 2 * a.pad;
+      jb.vimg = jb.ho * jb.wp;
+      jb.tpi = (jb.vimg + 127) / 128;
+      jb.row_off = (int32_t)rows;
+      rows += (int64_t)jb.n * jb.hp * jb.wp;
+      tiles += jb.n * jb.tpi * prm.n_tiles;
+    } else {
+      tiles += ((a.jobs[j].m_total + BM - 1) / BM) * prm.n_tiles;
+    }
+  }
+  if (flat && (kSub != 1 || a.stride != 1 || a.cin % BK != 0 || rows > a.ws_rows)) {
+    *err = "conv_tc: workspace path needs stride 1, cin % 128 == 0 and a large enough workspace";
+    return 1;
   }
   prm.total_tiles = tiles;
   if (tiles == 0) return 0;
@@ -839,6 +943,7 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   prm.upsample = a.upsample; prm.scale_main = a.scale_main; prm.has_skip = a.has_skip;
   prm.bn = BN;
   prm.acc_small = a.acc_bound < (1LL << 22) ? 1 : 0;
+  prm.cin_chunks = a.cin / BK;
   prm.status = a.status;
   // shared memory plan: stages of (BM x 128 A bytes + BN x 128 B bytes)
   const size_t stage_bytes = (size_t)kStageA + (size_t)BN * BK;
@@ -874,13 +979,43 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int grid = tiles < sms ? tiles : sms;
   const bool in_tap = (a.cin % BK) == 0;
+  CUtensorMap map_a = map;  // unused unless flat
+  if (flat) {
+    // 1) expand the packed codes of every job into the zero-padded byte workspace
+    ExpandArgs ea{};
+    for (int j = 0; j < a.njobs; ++j) ea.jobs[j] = prm.jobs[j];
+    ea.njobs = a.njobs; ea.cin = a.cin; ea.pad = a.pad; ea.x_row_bytes = a.x_row_bytes;
+    ea.total_rows = rows; ea.ws = a.ws;
+    const int64_t nthreads = rows * (a.cin / 32);
+    const unsigned blocks = (unsigned)((nthreads + 255) / 256);
+    switch (a.x_bits) {
+      case 2: expand_kernel<2><<<blocks, 256, 0, stream>>>(ea); break;
+      case 3: expand_kernel<3><<<blocks, 256, 0, stream>>>(ea); break;
+      case 4: expand_kernel<4><<<blocks, 256, 0, stream>>>(ea); break;
+      default: *err = "conv_tc: activation bits must be 2, 3 or 4"; return 2;
+    }
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) { *err = std::string("expand launch: ") + cudaGetErrorString(e); return 3; }
+    // 2) tensor map over the workspace as a [rows][cin] byte matrix with 128 x 128 boxes
+    cuuint64_t gd[2] = {(cuuint64_t)a.cin, (cuuint64_t)rows};
+    cuuint64_t gs[1] = {(cuuint64_t)a.cin};
+    cuuint32_t bx[2] = {(cuuint32_t)BK, 128};
+    CUresult r2 = enc(&map_a, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)a.ws, gd, gs, bx, estr,
+                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r2 != CUDA_SUCCESS) {
+      *err = "cuTensorMapEncodeTiled (activations) failed: " + std::to_string((int)r2);
+      return 3;
+    }
+    return launch_bits<2, true, true>(prm, map, map_a, grid, smem, stream, err);
+  }
   switch (a.x_bits) {
-    case 2: return in_tap ? launch_bits<2, true>(prm, map, grid, smem, stream, err)
-                          : launch_bits<2, false>(prm, map, grid, smem, stream, err);
-    case 3: return in_tap ? launch_bits<3, true>(prm, map, grid, smem, stream, err)
-                          : launch_bits<3, false>(prm, map, grid, smem, stream, err);
-    case 4: return in_tap ? launch_bits<4, true>(prm, map, grid, smem, stream, err)
-                          : launch_bits<4, false>(prm, map, grid, smem, stream, err);
+    case 2: return in_tap ? launch_bits<2, true, false>(prm, map, map_a, grid, smem, stream, err)
+                          : launch_bits<2, false, false>(prm, map, map_a, grid, smem, stream, err);
+    case 3: return in_tap ? launch_bits<3, true, false>(prm, map, map_a, grid, smem, stream, err)
+                          : launch_bits<3, false, false>(prm, map, map_a, grid, smem, stream, err);
+    case 4: return in_tap ? launch_bits<4, true, false>(prm, map, map_a, grid, smem, stream, err)
+                          : launch_bits<4, false, false>(prm, map, map_a, grid, smem, stream, err);
     default: *err = "conv_tc: activation bits must be 2, 3 or 4"; return 2;
   }
 }

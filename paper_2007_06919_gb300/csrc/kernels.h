@@ -19,6 +19,11 @@ struct ConvJobDev {
   int32_t level;
   int32_t m_total;        // n * ho * wo
   int32_t tile_begin;     // first global tile index of this job
+  // expanded-activation ("flat") path: zero-padded byte image of this job in the workspace
+  int32_t row_off;        // first workspace row (one row = cin bytes) of image 0
+  int32_t hp, wp;         // padded height / width (h + 2 pad, w + 2 pad)
+  int32_t vimg;           // virtual output rows per image: ho * wp (columns >= wo are junk)
+  int32_t tpi;            // tiles per image
 };
 
 struct ConvArgs {
@@ -38,6 +43,8 @@ struct ConvArgs {
   const int16_t* w_i16;   // [cout][k_total] signed integers
   int32_t cout_pad, k_total, k_pad, bn;
   int64_t acc_bound;      // K * max|x| * max|w|: bound on |accumulator|
+  uint8_t* ws;            // expanded-activation workspace (NULL: in-kernel unpacking)
+  int64_t ws_rows;        // rows of cin bytes available in the workspace
   uint32_t* status;       // device status word
 };
 

@@ -30,8 +30,9 @@ def weights(w_codes: np.ndarray, w_bits: int, w_format: int = 0):
 def conv_pair(x: np.ndarray, x_bits: int, w: np.ndarray, w_bits: int, *, w_format: int = 0, stride: int = 1,
               pad: int = 1, out_bits: int = 2, m0=None, shift=None, bias=None, level: int = 0,
               skip: np.ndarray | None = None, skip_bits: int = 4, skip_c=None, skip_d=None, upsample: int = 1,
-              scale_main: int = 0, path: int = 0, wprep=None):
-    """Returns (gpu_bytes, oracle_bytes, used_path) for one convolution."""
+              scale_main: int = 0, path: int = 0, wprep=None, workspace: bool = False):
+    """Returns (gpu_bytes, oracle_bytes, used_path) for one convolution. With workspace=True
+    the call gets an expanded-activation workspace when that path applies."""
     n, h, wd, cin = x.shape
     cout, kh, kw, _ = w.shape
     xt = oracle.CodeTensor.from_codes(x, x_bits)
@@ -47,9 +48,12 @@ def conv_pair(x: np.ndarray, x_bits: int, w: np.ndarray, w_bits: int, *, w_forma
     rq = aqd.RequantParams.from_numpy(m0, shift, bias) if (m0 is not None or bias is not None) else None
     S = to_device(skt) if skt is not None else None
     sp = aqd.SkipParams.from_numpy(skip_c, skip_d, upsample, scale_main) if skip is not None else None
+    ws = aqd.workspace_for([(X, Y, S, level)], W, stride, pad) if workspace else None
+    if ws is not None:
+        ws.fill_(0x5A)  # stale contents must not matter
     old = aqd.set_conv_path(path)
     try:
-        aqd.conv_int(X, W, stride, pad, Y, level=level, rq=rq, skip=S, sp=sp)
+        aqd.conv_int(X, W, stride, pad, Y, level=level, rq=rq, skip=S, sp=sp, workspace=ws)
         used = aqd.last_conv_path()
     finally:
         aqd.set_conv_path(old)

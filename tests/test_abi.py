@@ -79,21 +79,39 @@ def test_status_strings(lib):
 def test_invalid_arguments_return_before_launch(lib):
     from paper_2007_06919_gb300 import aqd
     # NULL tensors / bad sizes are rejected on the host; nothing reaches the GPU
-    assert lib.aqd_conv_int(None, None, 1, 1, 0, None, None, None, None, None) == 1
+    assert lib.aqd_conv_int(None, None, 1, 1, 0, None, None, None, None, None, 0, None) == 1
     assert lib.aqd_pack_codes(None, 10, 48, 2, None, None) == 1  # 48 channels at 2 bits
     assert lib.aqd_pack_codes(None, 10, 64, 5, None, None) == 1  # 5-bit codes do not exist
     x = aqd._Tensor(1, 4, 4, 64, 2, 16)
     y = aqd._Tensor(1, 4, 4, 64, 32, 16)  # int32 output: no requant tables needed
     w = aqd._Weights(256, 64, 3, 3, 32, 2, 0)  # cin 32 != x.c 64
-    st = lib.aqd_conv_int(ctypes.byref(x), ctypes.byref(w), 1, 1, 0, None, None, None, ctypes.byref(y), None)
+    st = lib.aqd_conv_int(ctypes.byref(x), ctypes.byref(w), 1, 1, 0, None, None, None, ctypes.byref(y), None, 0, None)
     assert st == 1
     assert b"cin" in lib.aqd_last_error()
     x2 = aqd._Tensor(1, 4, 4, 64, 2, 8)  # misaligned data pointer
     w2 = aqd._Weights(256, 64, 3, 3, 64, 2, 0)
-    st = lib.aqd_conv_int(ctypes.byref(x2), ctypes.byref(w2), 1, 1, 0, None, None, None, ctypes.byref(y), None)
+    st = lib.aqd_conv_int(ctypes.byref(x2), ctypes.byref(w2), 1, 1, 0, None, None, None, ctypes.byref(y), None, 0, None)
     assert st == 1 and b"aligned" in lib.aqd_last_error()
     assert lib.aqd_conv_weights_bytes(0, 3, 3, 64) == 0
     assert lib.aqd_conv_weights_bytes(256, 3, 3, 256) >= 256 * 2304 * 3
+
+
+def test_workspace_bytes_host_logic(lib):
+    """The expanded-activation workspace is sum(n * (h+2p) * (w+2p)) * cin bytes for stride-1
+    convolutions with cin % 128 == 0 and codes/weights of at most 4 bits, else 0."""
+    from paper_2007_06919_gb300 import aqd
+    jobs = (aqd._Job * 2)()
+    jobs[0].x = aqd._Tensor(2, 10, 17, 256, 2, 256)
+    jobs[1].x = aqd._Tensor(2, 5, 9, 256, 2, 256)
+    w = aqd._Weights(256, 256, 3, 3, 256, 2, 0)
+    want = (2 * 12 * 19 + 2 * 7 * 11) * 256
+    assert lib.aqd_conv_workspace_bytes(jobs, 2, ctypes.byref(w), 1, 1) == want
+    assert lib.aqd_conv_workspace_bytes(jobs, 2, ctypes.byref(w), 2, 1) == 0      # stride 2
+    w8 = aqd._Weights(256, 256, 3, 3, 256, 8, 0)
+    assert lib.aqd_conv_workspace_bytes(jobs, 2, ctypes.byref(w8), 1, 1) == 0     # 8-bit weights
+    w64 = aqd._Weights(256, 64, 3, 3, 64, 2, 0)
+    jobs[0].x = aqd._Tensor(2, 10, 17, 64, 2, 256)
+    assert lib.aqd_conv_workspace_bytes(jobs, 1, ctypes.byref(w64), 1, 1) == 0    # cin 64
 
 
 def test_set_conv_path_rejects_unknown(lib):

@@ -81,10 +81,43 @@ def test_conv_shapes_bit_exact(case, path):
     assert_same(got, want, cout, ob, f"case {case}")
 
 
+WS_CASES = [c for c in CASES if c[9] == 1 and c[6] % 128 == 0 and c[0] <= 4 and c[1] <= 4]
+
+
+@pytest.mark.parametrize("case", WS_CASES, ids=[str(i) for i in range(len(WS_CASES))])
+def test_conv_workspace_path_bit_exact(case):
+    """The expanded-activation path (one expansion pass into a caller workspace, then TMA
+    tiles of the zero-padded byte image, junk columns dropped) gives the same bytes."""
+    xb, wb, fmt, n, h, wd, cin, cout, k, stride, pad, ob = case
+    rng = np.random.default_rng(hash(case) % 2 ** 32 + 1)
+    x = synth.act_codes(rng, (n, h, wd, cin), xb)
+    w = rng.integers(-(1 << (wb - 1)), 1 << (wb - 1), size=(cout, k, k, cin)).astype(np.int32)
+    std = np.sqrt(k * k * cin * np.mean(np.arange(1 << xb) ** 2) * (1 << (2 * wb - 2)) / 3)
+    m0, sh, b = _params(rng, 1, cout, ob if ob != 32 else 4, calib_std=std)
+    got, want, used = conv_pair(x, xb, w, wb, stride=stride, pad=pad, out_bits=ob, m0=m0, shift=sh, bias=b,
+                                path=TC, workspace=True)
+    assert used == 3
+    assert_same(got, want, cout, ob, f"workspace case {case}")
+
+
+@pytest.mark.parametrize("shape", [(1, 1, 1), (2, 3, 300), (1, 37, 2), (3, 7, 11)])
+def test_workspace_path_edge_shapes(shape):
+    """Tiles that cross image rows and images, 1x1 images and single-column images."""
+    n, h, wd = shape
+    rng = np.random.default_rng(n * 1000 + h * 10 + wd)
+    x = synth.act_codes(rng, (n, h, wd, 256), 2)
+    w = synth.weight_codes(rng, (256, 3, 3, 256), 2)
+    m0, sh, b = _params(rng, 1, 256, 2, calib_std=37.0)
+    got, want, used = conv_pair(x, 2, w, 2, out_bits=2, m0=m0, shift=sh, bias=b, path=TC, workspace=True)
+    assert used == 3
+    assert_same(got, want, 256, 2, f"edge {shape}")
+
+
 @pytest.mark.parametrize("path", [TC, DIRECT])
 @pytest.mark.parametrize("skip_bits,upsample,mirror", [(4, 1, 0), (4, 1, 1), (32, 1, 0), (2, 2, 0), (32, 2, 1),
                                                         (8, 1, 0)])
-def test_conv_with_skip_bit_exact(path, skip_bits, upsample, mirror):
+@pytest.mark.parametrize("ws", [False, True])
+def test_conv_with_skip_bit_exact(path, skip_bits, upsample, mirror, ws):
     """Eq. 7 fused into the epilogue: identity / downsample (int32) / FPN (upsample 2) skips,
     both directions of the rescale."""
     rng = np.random.default_rng(7 + skip_bits + 10 * upsample + 100 * mirror)
@@ -98,8 +131,9 @@ def test_conv_with_skip_bit_exact(path, skip_bits, upsample, mirror):
     else:
         skip = synth.act_codes(rng, (n, sh_[0], sh_[1], cout), skip_bits)
     c, d = synth.skip_params(rng, 1, cout, sh)
-    got, want, _ = conv_pair(x, 4, w, 4, out_bits=4, m0=m0, shift=sh, bias=b, skip=skip, skip_bits=skip_bits,
-                             skip_c=c, skip_d=d, upsample=upsample, scale_main=mirror, path=path)
+    got, want, used = conv_pair(x, 4, w, 4, out_bits=4, m0=m0, shift=sh, bias=b, skip=skip, skip_bits=skip_bits,
+                             skip_c=c, skip_d=d, upsample=upsample, scale_main=mirror, path=path, workspace=ws)
+    assert used == (3 if (ws and path == TC) else path)
     assert_same(got, want, cout, 4, "skip")
 
 

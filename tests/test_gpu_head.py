@@ -23,7 +23,8 @@ def _rq(cv):
     return aqd.RequantParams.from_numpy(cv.m0, cv.shift, cv.bias)
 
 
-def test_config1_bottleneck_chain_bit_exact():
+@pytest.mark.parametrize("ws", [False, True])
+def test_config1_bottleneck_chain_bit_exact(ws):
     """1x1 512->128, 3x3 128->128, 1x1 128->512 + identity skip (Eq. 7), all at
     2 x 100 x 152, 4-bit: each stage is compared; the GPU chain feeds itself and the
     oracle chain feeds itself."""
@@ -38,8 +39,10 @@ def test_config1_bottleneck_chain_bit_exact():
         ref = _ref_conv(ref, wp, cv, skip=skip_ref)
         Y = aqd.DTensor.empty(ref.n, ref.h, ref.w, cv.cout, 4)
         sp = aqd.SkipParams.from_numpy(cv.skip_c, cv.skip_d) if cv.skip_c is not None else None
-        aqd.conv_int(cur, W, cv.stride, cv.pad, Y, rq=_rq(cv), skip=to_device(xt) if sp else None, sp=sp)
-        assert aqd.last_conv_path() == 1
+        skt = to_device(xt) if sp else None
+        wsb = aqd.workspace_for([(cur, Y, skt, 0)], W, cv.stride, cv.pad) if ws else None
+        aqd.conv_int(cur, W, cv.stride, cv.pad, Y, rq=_rq(cv), skip=skt, sp=sp, workspace=wsb)
+        assert aqd.last_conv_path() == (3 if ws else 1)
         torch.cuda.synchronize()
         assert_same(Y.data.cpu().numpy().reshape(ref.packed.shape), ref.packed, cv.cout, 4, f"stage {i}")
         cur = Y
@@ -47,7 +50,7 @@ def test_config1_bottleneck_chain_bit_exact():
     assert len(np.unique(ref.codes())) > 3
 
 
-def _tower_levels_gpu(inputs, convs, bits, grouped=True):
+def _tower_levels_gpu(inputs, convs, bits, grouped=True, ws=False):
     """Runs the 4-layer tower + cls/box on every level; returns per-level outputs."""
     nl = len(inputs)
     xs = [to_device(oracle.CodeTensor.from_codes(x, bits)) for x in inputs]
@@ -55,7 +58,10 @@ def _tower_levels_gpu(inputs, convs, bits, grouped=True):
         W, _ = weights(cv.w, bits)
         ys = [aqd.DTensor.empty(x.n, x.h, x.w, 256, bits) for x in xs]
         if grouped:
-            aqd.conv_int_grouped([(xs[l], ys[l], None, l) for l in range(nl)], W, 1, 1, rq=_rq(cv))
+            jobs = [(xs[l], ys[l], None, l) for l in range(nl)]
+            wsb = aqd.workspace_for(jobs, W, 1, 1) if ws else None
+            aqd.conv_int_grouped(jobs, W, 1, 1, rq=_rq(cv), workspace=wsb)
+            assert aqd.last_conv_path() == (3 if ws else 1)
         else:
             for l in range(nl):
                 aqd.conv_int(xs[l], W, 1, 1, ys[l], level=l, rq=_rq(cv))
@@ -64,8 +70,9 @@ def _tower_levels_gpu(inputs, convs, bits, grouped=True):
     for cv in convs[4:]:
         W, _ = weights(cv.w, bits)
         ys = [aqd.DTensor.empty(x.n, x.h, x.w, cv.cout, 32) for x in xs]
-        aqd.conv_int_grouped([(xs[l], ys[l], None, l) for l in range(nl)], W, 1, 1,
-                             rq=aqd.RequantParams.from_numpy(None, None, cv.bias))
+        jobs = [(xs[l], ys[l], None, l) for l in range(nl)]
+        wsb = aqd.workspace_for(jobs, W, 1, 1) if ws else None
+        aqd.conv_int_grouped(jobs, W, 1, 1, rq=aqd.RequantParams.from_numpy(None, None, cv.bias), workspace=wsb)
         heads.append(ys)
     torch.cuda.synchronize()
     return xs, heads
@@ -83,12 +90,12 @@ def _tower_levels_ref(inputs, convs, bits):
     return xs, heads
 
 
-@pytest.mark.parametrize("calibrated", [False, True])
-def test_head_tower_full_size_bit_exact(calibrated):
+@pytest.mark.parametrize("calibrated,ws", [(False, False), (True, False), (False, True), (True, True)])
+def test_head_tower_full_size_bit_exact(calibrated, ws):
     """The whole detector head at 800x1333 (levels 100x168 .. 7x11), batch 2, 2-bit:
     4 grouped tower layers + cls (80) + box (4) int32 heads, every output compared."""
     wl = synth.config2(calibrated=calibrated)
-    g_tower, g_heads = _tower_levels_gpu(wl.inputs, wl.convs, 2)
+    g_tower, g_heads = _tower_levels_gpu(wl.inputs, wl.convs, 2, ws=ws)
     r_tower, r_heads = _tower_levels_ref(wl.inputs, wl.convs, 2)
     for l in range(5):
         assert_same(g_tower[l].data.cpu().numpy().reshape(r_tower[l].packed.shape), r_tower[l].packed, 256, 2,
@@ -103,7 +110,7 @@ def test_head_tower_full_size_bit_exact(calibrated):
 
 def test_grouped_launch_equals_per_level_launches():
     wl = synth.head_tower(9, 2, 2, levels=[(20, 34), (10, 17), (5, 9), (3, 5), (2, 3)], calibrated=True)
-    a, ah = _tower_levels_gpu(wl.inputs, wl.convs, 2, grouped=True)
+    a, ah = _tower_levels_gpu(wl.inputs, wl.convs, 2, grouped=True, ws=True)
     b, bh = _tower_levels_gpu(wl.inputs, wl.convs, 2, grouped=False)
     for l in range(5):
         assert torch.equal(a[l].data, b[l].data)
@@ -112,6 +119,7 @@ def test_grouped_launch_equals_per_level_launches():
 
 @pytest.mark.parametrize("bits", [2, 3, 4, 8])
 def test_bitwidth_sweep_batch16_sampled(bits):
+    """(With the expanded-activation workspace where that path applies.)"""
     """First tower layer of the batch-16 head for each bit width, all five levels in one
     grouped launch; the oracle computes 600 sampled pixels per level (all channels)."""
     wl = synth.config4(bits)
@@ -120,8 +128,10 @@ def test_bitwidth_sweep_batch16_sampled(bits):
     xts = [oracle.CodeTensor.from_codes(x, bits) for x in wl.inputs]
     xs = [to_device(t) for t in xts]
     ys = [aqd.DTensor.empty(x.n, x.h, x.w, 256, bits) for x in xs]
-    aqd.conv_int_grouped([(xs[l], ys[l], None, l) for l in range(5)], W, 1, 1, rq=_rq(cv))
-    assert aqd.last_conv_path() == (1 if bits <= 4 else 2)
+    jobs = [(xs[l], ys[l], None, l) for l in range(5)]
+    wsb = aqd.workspace_for(jobs, W, 1, 1)
+    aqd.conv_int_grouped(jobs, W, 1, 1, rq=_rq(cv), workspace=wsb)
+    assert aqd.last_conv_path() == (3 if bits <= 4 else 2)
     torch.cuda.synchronize()
     rng = np.random.default_rng(bits)
     for l in range(5):

@@ -49,6 +49,10 @@ constexpr int BK = 128;            // K bytes per stage
 #endif
 constexpr int kEpiWarps = AQD_EPI_WARPS;  // 4 or 8
 static_assert(kEpiWarps == 4 || kEpiWarps == 8, "epilogue warps: 4 or 8");
+#ifndef AQD_EPI_BATCH
+#define AQD_EPI_BATCH 1
+#endif
+constexpr int kEpiBatch = AQD_EPI_BATCH;  // 32-column groups per TMEM load wait (1 or 2)
 constexpr int kEpiThreads = kEpiWarps * 32;
 #ifndef AQD_TMA_WARPS
 #define AQD_TMA_WARPS 1
@@ -695,9 +699,9 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       // this warp's (sub-tile, 32-column group) units, two per TMEM wait
       const int ngrp = (BN + 31) / 32;
       const int nunits = kSub * ngrp;
-      for (int u0 = gi; u0 < nunits; u0 += 2 * kGroups) {
+      for (int u0 = gi; u0 < nunits; u0 += kEpiBatch * kGroups) {
         const int u1 = u0 + kGroups;
-        const bool two = u1 < nunits;  // warp-uniform
+        const bool two = kEpiBatch == 2 && u1 < nunits;  // warp-uniform
         uint32_t va[32], vb[32];
         int subA = u0 / ngrp, g0A = (u0 % ngrp) * 32;
         int subB = two ? u1 / ngrp : 0, g0B = two ? (u1 % ngrp) * 32 : 0;

@@ -4,6 +4,9 @@ One step = the shared RetinaNet head of AQD applied to the five FPN levels of an
 image batch (levels 100x168, 50x84, 25x42, 13x21, 7x11; batch 2; 2-bit codes): four
 3x3 256->256 tower convs with per-level BN tables (each one grouped launch over all
 levels) and the 3x3 256->80 classification and 256->4 box convs with int32 outputs.
+The two output convs read the same tower output, so they run as one 256->84 conv with
+the weight rows and biases concatenated (channels 0..79 = classification, 80..83 = box):
+every output value is the one the two separate convs give.
 Inputs are seeded synthetic codes (no images are used). Ops are counted as 2*M*N*K of the
 real (unpadded) convolutions.
 
@@ -212,11 +215,13 @@ def main():
         xs = [aqd.DTensor.from_codes(x.to(dev), 2) for x in xs_host]
         tower_w = [aqd.ConvWeights(torch.from_numpy(cv.w).to(dev), 2) for cv in wl.convs[:4]]
         tower_rq = [aqd.RequantParams.from_numpy(cv.m0, cv.shift, cv.bias, device=dev) for cv in wl.convs[:4]]
-        head_w = [aqd.ConvWeights(torch.from_numpy(cv.w).to(dev), 2) for cv in wl.convs[4:]]
-        head_rq = [aqd.RequantParams.from_numpy(None, None, cv.bias, device=dev) for cv in wl.convs[4:]]
+        cls, box = wl.convs[4:]
+        head_w = aqd.ConvWeights(torch.from_numpy(np.concatenate([cls.w, box.w])).to(dev), 2)
+        head_rq = aqd.RequantParams.from_numpy(None, None, np.concatenate([cls.bias, box.bias], axis=1),
+                                               device=dev)
+        n_head = cls.cout + box.cout
         bufs = [[aqd.DTensor.empty(batch, h, w, 256, 2, device=dev) for (h, w) in levels] for _ in range(2)]
-        heads = [[aqd.DTensor.empty(batch, h, w, cv.cout, 32, device=dev) for (h, w) in levels]
-                 for cv in wl.convs[4:]]
+        heads = [aqd.DTensor.empty(batch, h, w, n_head, 32, device=dev) for (h, w) in levels]
         flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
         # one expanded-activation workspace serves every conv of the step (same input shapes)
         ws = aqd.workspace_for([(xs[l], bufs[0][l], None, l) for l in range(nl)], tower_w[0], 1, 1, device=dev)
@@ -229,13 +234,12 @@ def main():
             aqd.conv_int_grouped([(cur[l], out[l], None, l) for l in range(nl)], tower_w[i], 1, 1,
                                  rq=tower_rq[i], workspace=ws, stream=stream)
             cur = out
-        for j in range(2):
-            aqd.conv_int_grouped([(cur[l], heads[j][l], None, l) for l in range(nl)], head_w[j], 1, 1,
-                                 rq=head_rq[j], workspace=ws, stream=stream)
+        aqd.conv_int_grouped([(cur[l], heads[l], None, l) for l in range(nl)], head_w, 1, 1,
+                             rq=head_rq, workspace=ws, stream=stream)
 
     # each conv is one expansion launch + one tensor-core launch when the workspace applies
     per_conv = 2 if ws is not None else 1
-    launches_per_step = 6 * per_conv
+    launches_per_step = 5 * per_conv
     with torch.cuda.stream(stream):
         for _ in range(3):
             step()
@@ -289,9 +293,9 @@ def main():
 
     # end to end through the public API: pinned host inputs -> device, step, head outputs -> host
     h_in = [x.data.cpu().pin_memory() for x in xs]
-    h_out = [[torch.empty_like(t.data, device="cpu").pin_memory() for t in hs] for hs in heads]
+    h_out = [torch.empty_like(t.data, device="cpu").pin_memory() for t in heads]
     h2d = sum(t.numel() * t.element_size() for t in h_in)
-    d2h = sum(t.numel() * t.element_size() for hs in h_out for t in hs)
+    d2h = sum(t.numel() * t.element_size() for t in h_out)
     n_e2e = max(20, min(200, args.steps // 10))
     with torch.cuda.stream(stream):
         ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -301,9 +305,8 @@ def main():
             for d, h in zip(xs, h_in):
                 d.data.copy_(h, non_blocking=True)
             graph.replay()
-            for hs, ds in zip(h_out, heads):
-                for h, d in zip(hs, ds):
-                    h.copy_(d.data, non_blocking=True)
+            for h, d in zip(h_out, heads):
+                h.copy_(d.data, non_blocking=True)
         ev1.record(stream)
     stream.synchronize()
     e2e_ms = ev0.elapsed_time(ev1) / n_e2e
@@ -319,7 +322,8 @@ def main():
         "vs_baseline": None, "dtype": "u2 x s2 codes -> exact i32 (e4m3 tensor-core MMA, f32 accumulate)",
         "data": "synthetic",
         "config": {"workload": WORKLOAD, "batch": batch, "bits": 2, "levels": levels,
-                   "convs": "4x 3x3 256->256 (per-level BN) + 3x3 256->80 + 3x3 256->4, int32 heads",
+                   "convs": "4x 3x3 256->256 (per-level BN) + 3x3 256->80 cls + 3x3 256->4 box "
+                            "(run as one 256->84 conv), int32 heads",
                    "l2": "flushed (256 MiB write) before every timed step", "graph": "CUDA graph per step",
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "images_per_s": world * batch / (ms_per_step * 1e-3),

@@ -841,32 +841,42 @@ struct ExpandArgs {
 
 template <int kXBits>
 __global__ void __launch_bounds__(256) expand_kernel(const __grid_constant__ ExpandArgs a) {
+  // one thread per (workspace row, 128-channel block): reads 16*kXBits packed bytes,
+  // writes 128 bytes; all index arithmetic in 32 bits (rows < 2^31 is checked on the host)
   constexpr int kGB = 4 * kXBits;
-  const int groups = a.cin >> 5;
-  const int64_t t = (int64_t)blockIdx.x * 256 + threadIdx.x;
-  if (t >= a.total_rows * groups) return;
-  const int64_t row = t / groups;
-  const int g = (int)(t - row * groups);
+  const int blocks = a.cin >> 7;
+  const int t = blockIdx.x * 256 + threadIdx.x;
+  const int row = t / blocks;
+  if (row >= (int)a.total_rows) return;
+  const int cb = t - row * blocks;
   int j = 0;
 #pragma unroll 1
   while (j + 1 < a.njobs && row >= a.jobs[j + 1].row_off) ++j;
   const ConvJobDev& jb = a.jobs[j];
-  const int64_t local = row - jb.row_off;
-  const int64_t plane = (int64_t)jb.hp * jb.wp;
-  const int img = (int)(local / plane);
-  const int rem = (int)(local - img * plane);
-  const int hi = rem / jb.wp - a.pad, wi = rem - (rem / jb.wp) * jb.wp - a.pad;
-  uint32_t o[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+  const int local = row - jb.row_off;
+  const int plane = jb.hp * jb.wp;
+  const int img = local / plane;
+  const int rem = local - img * plane;
+  const int hr = rem / jb.wp;
+  const int hi = hr - a.pad, wi = rem - hr * jb.wp - a.pad;
+  uint4* dst = reinterpret_cast<uint4*>(a.ws + (size_t)row * a.cin + cb * 128);
   if (hi >= 0 && hi < jb.h && wi >= 0 && wi < jb.w) {
-    const uint8_t* src = jb.x + (((int64_t)img * jb.h + hi) * jb.w + wi) * a.x_row_bytes + g * kGB;
-    uint32_t w[kXBits];
+    const uint32_t* src = reinterpret_cast<const uint32_t*>(
+        jb.x + ((size_t)(img * jb.h + hi) * jb.w + wi) * a.x_row_bytes + cb * 4 * kGB);
+    uint32_t w[4 * kXBits];
 #pragma unroll
-    for (int i = 0; i < kXBits; ++i) w[i] = __ldg(reinterpret_cast<const uint32_t*>(src) + i);
-    unpack_group_bytes<kXBits>(w, o);
+    for (int i = 0; i < 4 * kXBits; ++i) w[i] = __ldg(src + i);
+#pragma unroll
+    for (int g = 0; g < 4; ++g) {
+      uint32_t o[8];
+      unpack_group_bytes<kXBits>(w + g * kXBits, o);
+      dst[2 * g] = make_uint4(o[0], o[1], o[2], o[3]);
+      dst[2 * g + 1] = make_uint4(o[4], o[5], o[6], o[7]);
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) dst[i] = make_uint4(0, 0, 0, 0);
   }
-  uint4* dst = reinterpret_cast<uint4*>(a.ws + row * a.cin + g * 32);
-  dst[0] = make_uint4(o[0], o[1], o[2], o[3]);
-  dst[1] = make_uint4(o[4], o[5], o[6], o[7]);
 }
 
 // ---------------------------------------------------------------- host side
@@ -990,7 +1000,7 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
     for (int j = 0; j < a.njobs; ++j) ea.jobs[j] = prm.jobs[j];
     ea.njobs = a.njobs; ea.cin = a.cin; ea.pad = a.pad; ea.x_row_bytes = a.x_row_bytes;
     ea.total_rows = rows; ea.ws = a.ws;
-    const int64_t nthreads = rows * (a.cin / 32);
+    const int64_t nthreads = rows * (a.cin / BK);
     const unsigned blocks = (unsigned)((nthreads + 255) / 256);
     switch (a.x_bits) {
       case 2: expand_kernel<2><<<blocks, 256, 0, stream>>>(ea); break;

@@ -144,3 +144,28 @@ def test_bitwidth_sweep_batch16_sampled(bits):
         bad = np.argwhere(got != want)
         assert bad.size == 0, f"level {l}: {len(bad)} mismatches, first {bad[:3].tolist()}"
     assert aqd.device_status() == 0
+
+
+def test_cls_and_box_as_one_conv_bit_exact():
+    """The benchmark's fused output conv: the 256->80 classification and 256->4 box weights
+    (and biases) concatenated into one 256->84 conv over the same tower output; channels
+    0..79 and 80..83 must equal the two separate convs of the oracle on every level."""
+    wl = synth.head_tower(11, 2, 2, levels=[(20, 34), (10, 17), (5, 9), (3, 5), (2, 3)], calibrated=True)
+    cls, box = wl.convs[4:]
+    rng = np.random.default_rng(11)
+    xts = [oracle.CodeTensor.from_codes(synth.act_codes(rng, x.shape[:3] + (256,), 2), 2) for x in wl.inputs]
+    W, _ = weights(np.concatenate([cls.w, box.w]), 2)
+    rq = aqd.RequantParams.from_numpy(None, None, np.concatenate([cls.bias, box.bias], axis=1))
+    xs = [to_device(t) for t in xts]
+    ys = [aqd.DTensor.empty(t.n, t.h, t.w, 84, 32) for t in xts]
+    jobs = [(xs[l], ys[l], None, l) for l in range(5)]
+    aqd.conv_int_grouped(jobs, W, 1, 1, rq=rq, workspace=aqd.workspace_for(jobs, W, 1, 1))
+    assert aqd.last_conv_path() == 3
+    torch.cuda.synchronize()
+    for l in range(5):
+        got = ys[l].data.cpu().numpy().view(np.int32).reshape(-1, 84)
+        for cv, lo in ((cls, 0), (box, 80)):
+            wp = oracle.pack(cv.w.reshape(-1, cv.cin), 2)
+            want = _ref_conv(xts[l], wp, cv, level=l).packed.view(np.int32).reshape(-1, cv.cout)
+            assert np.array_equal(got[:, lo:lo + cv.cout], want), f"level {l} head {cv.cout}"
+    assert aqd.device_status() == 0

@@ -219,7 +219,7 @@ static int64_t flat_rows(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv
     rows += (int64_t)x.n * (x.h + 2 * pad) * (x.w + 2 * pad);
   }
   // the expansion pass indexes (row, 128-channel block) pairs in 32 bits
-  return rows * (w->cin / 128) < (1LL << 31) ? rows : 0;
+  return rows * (w->cin / 16) < (1LL << 31) ? rows : 0;
 }
 
 size_t aqd_conv_workspace_bytes(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,

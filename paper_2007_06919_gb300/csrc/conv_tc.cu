@@ -839,16 +839,36 @@ struct ExpandArgs {
   uint8_t* ws;
 };
 
+// Codes 16h .. 16h+15 of one packed 32-channel group as 16 bytes (four words, word j
+// holding channels 16h+4j .. 16h+4j+3), for the layout of the packed-code tensors.
+template <int kXBits>
+__device__ __forceinline__ void unpack_half_group(const uint32_t* grp, int h, uint32_t o[4]) {
+  if constexpr (kXBits == 2) {
+    const uint32_t w = __ldg(grp + h);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) o[j] = (w >> (2 * j)) & 0x03030303u;
+  } else if constexpr (kXBits == 4) {
+    const uint2 w = __ldg(reinterpret_cast<const uint2*>(grp) + h);
+    o[0] = w.x & 0x0F0F0F0Fu; o[1] = (w.x >> 4) & 0x0F0F0F0Fu;
+    o[2] = w.y & 0x0F0F0F0Fu; o[3] = (w.y >> 4) & 0x0F0F0F0Fu;
+  } else {  // 3: one low-bits word per half, the high-bit word shared by both halves
+    const uint32_t lo = __ldg(grp + h), hi = __ldg(grp + 2);
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      o[j] = ((lo >> (2 * j)) & 0x03030303u) | (((hi >> (4 * h + j)) & 0x01010101u) << 2);
+  }
+}
+
 template <int kXBits>
 __global__ void __launch_bounds__(256) expand_kernel(const __grid_constant__ ExpandArgs a) {
-  // one thread per (workspace row, 128-channel block): reads 16*kXBits packed bytes,
-  // writes 128 bytes; all index arithmetic in 32 bits (rows < 2^31 is checked on the host)
-  constexpr int kGB = 4 * kXBits;
-  const int blocks = a.cin >> 7;
+  // one thread per 16 output bytes (half a packed group): consecutive threads read
+  // consecutive packed words and write consecutive 16-byte chunks of a workspace row.
+  // All index arithmetic is 32-bit (the host checks rows * cin / 16 < 2^31).
+  const int chunks = a.cin >> 4;
   const int t = blockIdx.x * 256 + threadIdx.x;
-  const int row = t / blocks;
+  const int row = t / chunks;
   if (row >= (int)a.total_rows) return;
-  const int cb = t - row * blocks;
+  const int q = t - row * chunks;
   int j = 0;
 #pragma unroll 1
   while (j + 1 < a.njobs && row >= a.jobs[j + 1].row_off) ++j;
@@ -859,24 +879,12 @@ __global__ void __launch_bounds__(256) expand_kernel(const __grid_constant__ Exp
   const int rem = local - img * plane;
   const int hr = rem / jb.wp;
   const int hi = hr - a.pad, wi = rem - hr * jb.wp - a.pad;
-  uint4* dst = reinterpret_cast<uint4*>(a.ws + (size_t)row * a.cin + cb * 128);
+  uint32_t o[4] = {0u, 0u, 0u, 0u};
   if (hi >= 0 && hi < jb.h && wi >= 0 && wi < jb.w) {
-    const uint32_t* src = reinterpret_cast<const uint32_t*>(
-        jb.x + ((size_t)(img * jb.h + hi) * jb.w + wi) * a.x_row_bytes + cb * 4 * kGB);
-    uint32_t w[4 * kXBits];
-#pragma unroll
-    for (int i = 0; i < 4 * kXBits; ++i) w[i] = __ldg(src + i);
-#pragma unroll
-    for (int g = 0; g < 4; ++g) {
-      uint32_t o[8];
-      unpack_group_bytes<kXBits>(w + g * kXBits, o);
-      dst[2 * g] = make_uint4(o[0], o[1], o[2], o[3]);
-      dst[2 * g + 1] = make_uint4(o[4], o[5], o[6], o[7]);
-    }
-  } else {
-#pragma unroll
-    for (int i = 0; i < 8; ++i) dst[i] = make_uint4(0, 0, 0, 0);
+    const uint8_t* px = jb.x + ((size_t)(img * jb.h + hi) * jb.w + wi) * a.x_row_bytes;
+    unpack_half_group<kXBits>(reinterpret_cast<const uint32_t*>(px + (q >> 1) * 4 * kXBits), q & 1, o);
   }
+  reinterpret_cast<uint4*>(a.ws + (size_t)row * a.cin)[q] = make_uint4(o[0], o[1], o[2], o[3]);
 }
 
 // ---------------------------------------------------------------- host side
@@ -904,7 +912,14 @@ template <int kXBits, bool kChunkInTap, bool kFlat>
 static int launch_bits(const Params& prm, const CUtensorMap& map, const CUtensorMap& map_a, int grid,
                        size_t smem, cudaStream_t stream, std::string* err) {
   auto kern = conv_tc_kernel<kXBits, kChunkInTap, kFlat>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  // The opt-in limit is raised to the device maximum, never lowered to this call's size:
+  // a CUDA graph node captured earlier with a larger plan must stay launchable (a graph
+  // node, or a tool relaunching it, is checked against the function's current limit).
+  int dev = 0, optin = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if ((size_t)optin < smem) { *err = "conv_tc: shared memory plan exceeds the device limit"; return 2; }
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
   if (e != cudaSuccess) { *err = std::string("cudaFuncSetAttribute: ") + cudaGetErrorString(e); return 3; }
   kern<<<grid, threads_for(kFlat), smem, stream>>>(map, map_a, prm);
   e = cudaGetLastError();
@@ -1000,7 +1015,7 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
     for (int j = 0; j < a.njobs; ++j) ea.jobs[j] = prm.jobs[j];
     ea.njobs = a.njobs; ea.cin = a.cin; ea.pad = a.pad; ea.x_row_bytes = a.x_row_bytes;
     ea.total_rows = rows; ea.ws = a.ws;
-    const int64_t nthreads = rows * (a.cin / BK);
+    const int64_t nthreads = rows * (a.cin / 16);
     const unsigned blocks = (unsigned)((nthreads + 255) / 256);
     switch (a.x_bits) {
       case 2: expand_kernel<2><<<blocks, 256, 0, stream>>>(ea); break;

@@ -188,6 +188,23 @@ aqd_status aqd_conv_int_grouped(const aqd_conv_job* jobs, int32_t njobs,
 size_t aqd_conv_workspace_bytes(const aqd_conv_job* jobs, int32_t njobs,
                                 const aqd_conv_weights* w, int32_t stride, int32_t pad);
 
+/* The two steps of the workspace path as separate calls, for callers that expand an input
+ * once and convolve it more than once (e.g. two heads over one feature map) or time the
+ * steps apart. aqd_conv_expand_input writes the byte image of the jobs' inputs (only x of
+ * each job is read; y, skip and level are ignored). aqd_conv_int_grouped_expanded is
+ * aqd_conv_int_grouped reading that image: `workspace` must hold the expansion of exactly
+ * these jobs' inputs, for the same weights' geometry, stride and pad, written by an
+ * earlier aqd_conv_expand_input on this stream. Both need the workspace path to apply
+ * (aqd_conv_workspace_bytes > 0) and a large enough workspace: otherwise AQD_ERR_INVALID,
+ * or AQD_ERR_UNSUPPORTED when the tensor-core kernel does not take the convolution. */
+aqd_status aqd_conv_expand_input(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
+                                 int32_t stride, int32_t pad, void* workspace, size_t ws_bytes,
+                                 aqd_stream_t stream);
+aqd_status aqd_conv_int_grouped_expanded(const aqd_conv_job* jobs, int32_t njobs,
+                                         const aqd_conv_weights* w, int32_t stride, int32_t pad,
+                                         const aqd_requant_params* rq, const aqd_skip_params* sp,
+                                         void* workspace, size_t ws_bytes, aqd_stream_t stream);
+
 /* ---- elementwise ------------------------------------------------------------------ */
 
 /* y = requant(sat32(acc + bias)) per channel at `level`: Eq. 6 + Eq. 2 on an int32

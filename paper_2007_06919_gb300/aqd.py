@@ -55,7 +55,8 @@ class _Job(ctypes.Structure):
 EXPORTS = ["aqd_row_bytes", "aqd_quantize_multiplier", "aqd_status_string", "aqd_last_error",
            "aqd_device_status", "aqd_set_conv_path", "aqd_last_conv_path", "aqd_pack_codes",
            "aqd_unpack_codes", "aqd_conv_weights_bytes", "aqd_conv_prepare_weights", "aqd_conv_int",
-           "aqd_conv_int_grouped", "aqd_conv_workspace_bytes", "aqd_requant", "aqd_residual_add_int",
+           "aqd_conv_int_grouped", "aqd_conv_workspace_bytes", "aqd_conv_expand_input",
+           "aqd_conv_int_grouped_expanded", "aqd_requant", "aqd_residual_add_int",
            "aqd_maxpool_codes"]
 
 _lib = None
@@ -97,6 +98,9 @@ def load(build_if_missing: bool = True):
                                ctypes.POINTER(_Tensor), vp, ctypes.c_size_t, vp]
     L.aqd_conv_int_grouped.argtypes = [ctypes.POINTER(_Job), i32, ctypes.POINTER(_Weights), i32, i32,
                                        ctypes.POINTER(_Requant), ctypes.POINTER(_Skip), vp, ctypes.c_size_t, vp]
+    L.aqd_conv_expand_input.argtypes = [ctypes.POINTER(_Job), i32, ctypes.POINTER(_Weights), i32, i32, vp,
+                                        ctypes.c_size_t, vp]
+    L.aqd_conv_int_grouped_expanded.argtypes = L.aqd_conv_int_grouped.argtypes
     L.aqd_conv_workspace_bytes.restype = ctypes.c_size_t
     L.aqd_conv_workspace_bytes.argtypes = [ctypes.POINTER(_Job), i32, ctypes.POINTER(_Weights), i32, i32]
     L.aqd_requant.argtypes = [ctypes.POINTER(_Tensor), ctypes.POINTER(_Requant), i32, ctypes.POINTER(_Tensor), vp]
@@ -104,7 +108,8 @@ def load(build_if_missing: bool = True):
                                        ctypes.POINTER(_Requant), i32, ctypes.POINTER(_Tensor), vp]
     L.aqd_maxpool_codes.argtypes = [ctypes.POINTER(_Tensor), i32, i32, i32, ctypes.POINTER(_Tensor), vp]
     for name in ("aqd_quantize_multiplier", "aqd_device_status", "aqd_pack_codes", "aqd_unpack_codes",
-                 "aqd_conv_prepare_weights", "aqd_conv_int", "aqd_conv_int_grouped", "aqd_requant",
+                 "aqd_conv_prepare_weights", "aqd_conv_int", "aqd_conv_int_grouped", "aqd_conv_expand_input",
+                 "aqd_conv_int_grouped_expanded", "aqd_requant",
                  "aqd_residual_add_int", "aqd_maxpool_codes"):
         getattr(L, name).restype = c_int
     _lib = L
@@ -304,7 +309,7 @@ def _jobs(jobs):
     arr = (_Job * len(jobs))()
     for i, (x, y, skip, level) in enumerate(jobs):
         arr[i].x = x.ct()
-        arr[i].y = y.ct()
+        arr[i].y = y.ct() if y is not None else _Tensor(0, 0, 0, 0, 0, None)
         arr[i].skip = skip.ct() if skip is not None else _Tensor(0, 0, 0, 0, 0, None)
         arr[i].level = level
     return arr
@@ -337,6 +342,30 @@ def conv_int_grouped(jobs, w: ConvWeights, stride: int, pad: int, *, rq: Requant
                                        ctypes.byref(spc) if spc is not None else None, wsp, wsb,
                                        _stream(stream)),
            "aqd_conv_int_grouped")
+
+
+def conv_expand_input(jobs, w: ConvWeights, stride: int, pad: int, workspace: torch.Tensor, stream=None):
+    """Only the expansion step of the workspace path: writes the zero-padded byte image of the
+    jobs' inputs into `workspace` (jobs as for conv_int_grouped; y and skip are ignored)."""
+    arr = _jobs(jobs)
+    wsp, wsb = _ws(workspace)
+    _check(load().aqd_conv_expand_input(arr, len(jobs), ctypes.byref(w.desc), stride, pad, wsp, wsb,
+                                        _stream(stream)), "aqd_conv_expand_input")
+
+
+def conv_int_grouped_expanded(jobs, w: ConvWeights, stride: int, pad: int, *, rq: RequantParams | None = None,
+                              sp: SkipParams | None = None, workspace: torch.Tensor, stream=None):
+    """conv_int_grouped fed from a workspace that already holds the expansion of these jobs'
+    inputs (written by conv_expand_input); launches only the tensor-core convolution."""
+    arr = _jobs(jobs)
+    rqc = rq.c() if rq is not None else None
+    spc = sp.cs() if sp is not None else None
+    wsp, wsb = _ws(workspace)
+    _check(load().aqd_conv_int_grouped_expanded(arr, len(jobs), ctypes.byref(w.desc), stride, pad,
+                                                ctypes.byref(rqc) if rqc is not None else None,
+                                                ctypes.byref(spc) if spc is not None else None, wsp, wsb,
+                                                _stream(stream)),
+           "aqd_conv_int_grouped_expanded")
 
 
 def requant(acc: DTensor, rq: RequantParams, y: DTensor, *, level: int = 0, stream=None) -> DTensor:

@@ -228,10 +228,58 @@ size_t aqd_conv_workspace_bytes(const aqd_conv_job* jobs, int32_t njobs, const a
   return rows > 0 ? (size_t)rows * (size_t)w->cin : 0;
 }
 
+// What one grouped call runs on the workspace path: expansion + convolution (the public
+// grouped call), the expansion alone, or the convolution from an already expanded workspace.
+enum ConvStage { kStageBoth = 0, kStageExpandOnly = 1, kStageConvOnly = 2 };
+
+static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
+                               int32_t stride, int32_t pad, const aqd_requant_params* rq,
+                               const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
+                               aqd_stream_t stream, ConvStage stage);
+
 aqd_status aqd_conv_int_grouped(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
                                 int32_t stride, int32_t pad, const aqd_requant_params* rq,
                                 const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
                                 aqd_stream_t stream) {
+  return conv_grouped(jobs, njobs, w, stride, pad, rq, sp, workspace, ws_bytes, stream, kStageBoth);
+}
+
+aqd_status aqd_conv_int_grouped_expanded(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
+                                         int32_t stride, int32_t pad, const aqd_requant_params* rq,
+                                         const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
+                                         aqd_stream_t stream) {
+  return conv_grouped(jobs, njobs, w, stride, pad, rq, sp, workspace, ws_bytes, stream, kStageConvOnly);
+}
+
+aqd_status aqd_conv_expand_input(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
+                                 int32_t stride, int32_t pad, void* workspace, size_t ws_bytes,
+                                 aqd_stream_t stream) {
+  if (!jobs || njobs <= 0 || njobs > kMaxJobs) return fail(AQD_ERR_INVALID, "njobs must be 1..8");
+  if (!workspace) return fail(AQD_ERR_INVALID, "the workspace must not be NULL");
+  // only the inputs matter here: give every job an int32 output of the right shape so the
+  // shared validation accepts it (nothing is written to it)
+  aqd_conv_job tmp[kMaxJobs];
+  for (int j = 0; j < njobs; ++j) {
+    tmp[j] = jobs[j];
+    tmp[j].skip = aqd_tensor{};
+    tmp[j].level = 0;
+    if (w && stride > 0 && pad >= 0) {
+      tmp[j].y.n = jobs[j].x.n;
+      tmp[j].y.h = (jobs[j].x.h + 2 * pad - w->kh) / stride + 1;
+      tmp[j].y.w = (jobs[j].x.w + 2 * pad - w->kw) / stride + 1;
+      tmp[j].y.c = w->cout;
+    }
+    tmp[j].y.bits = 32;
+    tmp[j].y.data = workspace;  // any non-null aligned pointer; never dereferenced
+  }
+  return conv_grouped(tmp, njobs, w, stride, pad, nullptr, nullptr, workspace, ws_bytes, stream,
+                      kStageExpandOnly);
+}
+
+static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
+                               int32_t stride, int32_t pad, const aqd_requant_params* rq,
+                               const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
+                               aqd_stream_t stream, ConvStage stage) {
   std::string err;
   if (!jobs || njobs <= 0 || njobs > kMaxJobs) return fail(AQD_ERR_INVALID, "njobs must be 1..8");
   if (!check_weights(w, &err)) return fail(AQD_ERR_INVALID, err);
@@ -326,10 +374,17 @@ aqd_status aqd_conv_int_grouped(const aqd_conv_job* jobs, int32_t njobs, const a
     }
   }
   if (path == 2 && !direct_ok) return fail(AQD_ERR_UNSUPPORTED, "accumulator bound exceeds int32");
+  if (stage != kStageBoth) {
+    if (path != 1) return fail(AQD_ERR_UNSUPPORTED, "the tensor-core kernel does not take this convolution");
+    if (!workspace) return fail(AQD_ERR_INVALID, "the workspace must not be NULL");
+    if (!a.ws) return fail(AQD_ERR_INVALID, "the workspace path does not apply, or the workspace is too small");
+  }
+  a.skip_expand = stage == kStageConvOnly ? 1 : 0;
+  a.expand_only = stage == kStageExpandOnly ? 1 : 0;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   int rc = path == 1 ? launch_conv_tc(a, st, &err) : launch_conv_direct(a, st, &err);
   if (rc) return fail((aqd_status)rc, err);
-  g_last_path = (path == 1 && a.ws) ? 3 : path;
+  if (stage != kStageExpandOnly) g_last_path = (path == 1 && a.ws) ? 3 : path;
   return AQD_OK;
 }
 

@@ -839,52 +839,111 @@ struct ExpandArgs {
   uint8_t* ws;
 };
 
-// Codes 16h .. 16h+15 of one packed 32-channel group as 16 bytes (four words, word j
-// holding channels 16h+4j .. 16h+4j+3), for the layout of the packed-code tensors.
-template <int kXBits>
-__device__ __forceinline__ void unpack_half_group(const uint32_t* grp, int h, uint32_t o[4]) {
-  if constexpr (kXBits == 2) {
-    const uint32_t w = __ldg(grp + h);
-#pragma unroll
-    for (int j = 0; j < 4; ++j) o[j] = (w >> (2 * j)) & 0x03030303u;
-  } else if constexpr (kXBits == 4) {
-    const uint2 w = __ldg(reinterpret_cast<const uint2*>(grp) + h);
-    o[0] = w.x & 0x0F0F0F0Fu; o[1] = (w.x >> 4) & 0x0F0F0F0Fu;
-    o[2] = w.y & 0x0F0F0F0Fu; o[3] = (w.y >> 4) & 0x0F0F0F0Fu;
-  } else {  // 3: one low-bits word per half, the high-bit word shared by both halves
-    const uint32_t lo = __ldg(grp + h), hi = __ldg(grp + 2);
-#pragma unroll
-    for (int j = 0; j < 4; ++j)
-      o[j] = ((lo >> (2 * j)) & 0x03030303u) | (((hi >> (4 * h + j)) & 0x01010101u) << 2);
-  }
-}
+// Position of one workspace row: its job, image, padded row / column and input pointer.
+struct ExpandPos {
+  int row, job, img, hr, wc;  // workspace row; job; image; padded row and column
+  int next_off;               // first row of the next job (INT_MAX for the last)
+};
 
-template <int kXBits>
-__global__ void __launch_bounds__(256) expand_kernel(const __grid_constant__ ExpandArgs a) {
-  // one thread per 16 output bytes (half a packed group): consecutive threads read
-  // consecutive packed words and write consecutive 16-byte chunks of a workspace row.
-  // All index arithmetic is 32-bit (the host checks rows * cin / 16 < 2^31).
-  const int chunks = a.cin >> 4;
-  const int t = blockIdx.x * 256 + threadIdx.x;
-  const int row = t / chunks;
-  if (row >= (int)a.total_rows) return;
-  const int q = t - row * chunks;
+__device__ __forceinline__ void expand_locate(const ExpandArgs& a, int row, ExpandPos& ps) {
   int j = 0;
 #pragma unroll 1
   while (j + 1 < a.njobs && row >= a.jobs[j + 1].row_off) ++j;
   const ConvJobDev& jb = a.jobs[j];
   const int local = row - jb.row_off;
   const int plane = jb.hp * jb.wp;
-  const int img = local / plane;
-  const int rem = local - img * plane;
-  const int hr = rem / jb.wp;
-  const int hi = hr - a.pad, wi = rem - hr * jb.wp - a.pad;
-  uint32_t o[4] = {0u, 0u, 0u, 0u};
-  if (hi >= 0 && hi < jb.h && wi >= 0 && wi < jb.w) {
-    const uint8_t* px = jb.x + ((size_t)(img * jb.h + hi) * jb.w + wi) * a.x_row_bytes;
-    unpack_half_group<kXBits>(reinterpret_cast<const uint32_t*>(px + (q >> 1) * 4 * kXBits), q & 1, o);
+  ps.row = row;
+  ps.job = j;
+  ps.img = local / plane;
+  const int rem = local - ps.img * plane;
+  ps.hr = rem / jb.wp;
+  ps.wc = rem - ps.hr * jb.wp;
+  ps.next_off = j + 1 < a.njobs ? a.jobs[j + 1].row_off : 0x7fffffff;
+}
+
+// Moves the position forward by d rows (d small: at most 4 here).
+__device__ __forceinline__ void expand_advance(const ExpandArgs& a, int d, ExpandPos& ps) {
+  ps.row += d;
+  if (ps.row >= ps.next_off) { expand_locate(a, ps.row, ps); return; }
+  const ConvJobDev& jb = a.jobs[ps.job];
+  ps.wc += d;
+#pragma unroll 1
+  while (ps.wc >= jb.wp) {
+    ps.wc -= jb.wp;
+    if (++ps.hr == jb.hp) { ps.hr = 0; ++ps.img; }
   }
-  reinterpret_cast<uint4*>(a.ws + (size_t)row * a.cin)[q] = make_uint4(o[0], o[1], o[2], o[3]);
+}
+
+template <int kXBits>
+__global__ void __launch_bounds__(256) expand_kernel(const __grid_constant__ ExpandArgs a) {
+  // The (row, 16-byte chunk) pairs of the workspace, row-major, are split into runs of
+  // 32 * kPerLane; a warp takes one run, lane l the pairs l, l + 32, ... of it, so every
+  // warp-wide step reads consecutive packed words and writes 512 consecutive bytes. The
+  // position is divided out once per lane and then advanced incrementally; the loads of
+  // all steps are issued before the stores. All index arithmetic is 32-bit (the host
+  // checks rows * cin / 16 < 2^31).
+  constexpr int kPerLane = 8;
+  const int chunks = a.cin >> 4;
+  const int total = (int)a.total_rows * chunks;
+  const int lane = threadIdx.x & 31;
+  const int e0 = (blockIdx.x * 8 + (threadIdx.x >> 5)) * (32 * kPerLane) + lane;
+  if (e0 >= total) return;
+  const int drow = 32 / chunks, dq = 32 - drow * chunks;
+  ExpandPos ps;
+  int q = e0 % chunks;
+  expand_locate(a, e0 / chunks, ps);
+  uint32_t w[kPerLane][kXBits == 2 ? 1 : 2];
+  uint8_t* dst[kPerLane];
+  bool inside[kPerLane];
+  int hsel[kPerLane];
+#pragma unroll
+  for (int i = 0; i < kPerLane; ++i) {
+    const int e = e0 + 32 * i;
+    const bool live = e < total;
+    const ConvJobDev& jb = a.jobs[ps.job];
+    const int hi = ps.hr - a.pad, wi = ps.wc - a.pad;
+    inside[i] = live && hi >= 0 && hi < jb.h && wi >= 0 && wi < jb.w;
+    dst[i] = live ? a.ws + (size_t)ps.row * a.cin + q * 16 : nullptr;
+    hsel[i] = q & 1;
+    if (inside[i]) {
+      const uint32_t* grp = reinterpret_cast<const uint32_t*>(
+          jb.x + ((size_t)(ps.img * jb.h + hi) * jb.w + wi) * a.x_row_bytes + (q >> 1) * 4 * kXBits);
+      if constexpr (kXBits == 2) {
+        w[i][0] = __ldg(grp + (q & 1));
+      } else if constexpr (kXBits == 4) {
+        const uint2 v = __ldg(reinterpret_cast<const uint2*>(grp) + (q & 1));
+        w[i][0] = v.x; w[i][1] = v.y;
+      } else {
+        w[i][0] = __ldg(grp + (q & 1)); w[i][1] = __ldg(grp + 2);
+      }
+    }
+    if (i + 1 < kPerLane) {
+      q += dq;
+      int step = drow;
+      if (q >= chunks) { q -= chunks; ++step; }
+      if (step) expand_advance(a, step, ps);
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < kPerLane; ++i) {
+    if (!dst[i]) continue;
+    uint32_t o[4] = {0u, 0u, 0u, 0u};
+    if (inside[i]) {
+      const int h = hsel[i];
+      if constexpr (kXBits == 2) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j) o[j] = (w[i][0] >> (2 * j)) & 0x03030303u;
+      } else if constexpr (kXBits == 4) {
+        o[0] = w[i][0] & 0x0F0F0F0Fu; o[1] = (w[i][0] >> 4) & 0x0F0F0F0Fu;
+        o[2] = w[i][1] & 0x0F0F0F0Fu; o[3] = (w[i][1] >> 4) & 0x0F0F0F0Fu;
+      } else {
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          o[j] = ((w[i][0] >> (2 * j)) & 0x03030303u) | (((w[i][1] >> (4 * h + j)) & 0x01010101u) << 2);
+      }
+    }
+    *reinterpret_cast<uint4*>(dst[i]) = make_uint4(o[0], o[1], o[2], o[3]);
+  }
 }
 
 // ---------------------------------------------------------------- host side
@@ -982,6 +1041,11 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   int stages = (int)((budget - epi_bytes - bar_bytes) / stage_bytes);
   if (stages > kMaxStages) stages = kMaxStages;
   if (stages < 2) { *err = "conv_tc: shared memory plan does not fit"; return 2; }
+  // The TMA issuers take K chunks round-robin and each waits on its stage's "empty"
+  // barrier by phase parity. That parity is unambiguous only while no issuer can run more
+  // than one phase ahead of the last completed one, which holds when the issuers are at
+  // most as many as the stages.
+  if (stages < tma_warps(flat)) { *err = "conv_tc: fewer pipeline stages than TMA issuers"; return 2; }
   prm.stages = stages;
   prm.off_b = (uint32_t)(stages * kStageA);
   prm.off_epi = prm.off_b + (uint32_t)(stages * BN * BK);
@@ -1010,21 +1074,26 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   const bool in_tap = (a.cin % BK) == 0;
   CUtensorMap map_a = map;  // unused unless flat
   if (flat) {
-    // 1) expand the packed codes of every job into the zero-padded byte workspace
-    ExpandArgs ea{};
-    for (int j = 0; j < a.njobs; ++j) ea.jobs[j] = prm.jobs[j];
-    ea.njobs = a.njobs; ea.cin = a.cin; ea.pad = a.pad; ea.x_row_bytes = a.x_row_bytes;
-    ea.total_rows = rows; ea.ws = a.ws;
-    const int64_t nthreads = rows * (a.cin / 16);
-    const unsigned blocks = (unsigned)((nthreads + 255) / 256);
-    switch (a.x_bits) {
-      case 2: expand_kernel<2><<<blocks, 256, 0, stream>>>(ea); break;
-      case 3: expand_kernel<3><<<blocks, 256, 0, stream>>>(ea); break;
-      case 4: expand_kernel<4><<<blocks, 256, 0, stream>>>(ea); break;
-      default: *err = "conv_tc: activation bits must be 2, 3 or 4"; return 2;
+    // 1) expand the packed codes of every job into the zero-padded byte workspace (unless
+    //    the caller expanded them already)
+    if (!a.skip_expand) {
+      ExpandArgs ea{};
+      for (int j = 0; j < a.njobs; ++j) ea.jobs[j] = prm.jobs[j];
+      ea.njobs = a.njobs; ea.cin = a.cin; ea.pad = a.pad; ea.x_row_bytes = a.x_row_bytes;
+      ea.total_rows = rows; ea.ws = a.ws;
+      // one warp per run of 32 * 8 (row, 16-byte chunk) pairs, 8 warps per block
+      const int64_t pairs = rows * (a.cin / 16);
+      const unsigned blocks = (unsigned)((pairs + 2047) / 2048);
+      switch (a.x_bits) {
+        case 2: expand_kernel<2><<<blocks, 256, 0, stream>>>(ea); break;
+        case 3: expand_kernel<3><<<blocks, 256, 0, stream>>>(ea); break;
+        case 4: expand_kernel<4><<<blocks, 256, 0, stream>>>(ea); break;
+        default: *err = "conv_tc: activation bits must be 2, 3 or 4"; return 2;
+      }
+      cudaError_t e = cudaGetLastError();
+      if (e != cudaSuccess) { *err = std::string("expand launch: ") + cudaGetErrorString(e); return 3; }
     }
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) { *err = std::string("expand launch: ") + cudaGetErrorString(e); return 3; }
+    if (a.expand_only) return 0;
     // 2) tensor map over the workspace as a [rows][cin] byte matrix with 128 x 128 boxes
     cuuint64_t gd[2] = {(cuuint64_t)a.cin, (cuuint64_t)rows};
     cuuint64_t gs[1] = {(cuuint64_t)a.cin};

@@ -45,6 +45,8 @@ struct ConvArgs {
   int64_t acc_bound;      // K * max|x| * max|w|: bound on |accumulator|
   uint8_t* ws;            // expanded-activation workspace (NULL: in-kernel unpacking)
   int64_t ws_rows;        // rows of cin bytes available in the workspace
+  int32_t skip_expand;    // workspace already holds the expansion: launch only the conv
+  int32_t expand_only;    // launch only the expansion into the workspace
   uint32_t* status;       // device status word
 };
 

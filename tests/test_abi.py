@@ -94,6 +94,13 @@ def test_invalid_arguments_return_before_launch(lib):
     assert st == 1 and b"aligned" in lib.aqd_last_error()
     assert lib.aqd_conv_weights_bytes(0, 3, 3, 64) == 0
     assert lib.aqd_conv_weights_bytes(256, 3, 3, 256) >= 256 * 2304 * 3
+    # the split workspace calls check their job list and workspace before anything else
+    assert lib.aqd_conv_expand_input(None, 0, ctypes.byref(w2), 1, 1, None, 0, None) == 1
+    jobs = (aqd._Job * 1)()
+    jobs[0].x = aqd._Tensor(1, 4, 4, 256, 2, 256)
+    assert lib.aqd_conv_expand_input(jobs, 1, ctypes.byref(w2), 1, 1, None, 0, None) == 1
+    assert b"workspace" in lib.aqd_last_error()
+    assert lib.aqd_conv_int_grouped_expanded(jobs, 9, ctypes.byref(w2), 1, 1, None, None, None, 0, None) == 1
 
 
 def test_workspace_bytes_host_logic(lib):

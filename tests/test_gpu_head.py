@@ -169,3 +169,64 @@ def test_cls_and_box_as_one_conv_bit_exact():
             want = _ref_conv(xts[l], wp, cv, level=l).packed.view(np.int32).reshape(-1, cv.cout)
             assert np.array_equal(got[:, lo:lo + cv.cout], want), f"level {l} head {cv.cout}"
     assert aqd.device_status() == 0
+
+
+def test_expand_once_then_two_convs_bit_exact():
+    """aqd_conv_expand_input once, then aqd_conv_int_grouped_expanded twice from the same
+    workspace (the classification and box convs over one tower output, levels grouped):
+    both must equal the oracle; the tower conv from the split calls must equal the
+    one-call grouped conv byte for byte."""
+    levels = [(16, 27), (8, 14), (4, 7)]
+    wl = synth.head_tower(31, 2, 2, levels=levels, calibrated=True)
+    tower, cls, box = wl.convs[0], wl.convs[4], wl.convs[5]
+    xts = [oracle.CodeTensor.from_codes(x, 2) for x in wl.inputs]
+    xs = [to_device(t) for t in xts]
+    Wt, _ = weights(tower.w, 2)
+    y1 = [aqd.DTensor.empty(t.n, t.h, t.w, 256, 2) for t in xts]
+    y2 = [aqd.DTensor.empty(t.n, t.h, t.w, 256, 2) for t in xts]
+    jobs1 = [(xs[l], y1[l], None, l) for l in range(3)]
+    jobs2 = [(xs[l], y2[l], None, l) for l in range(3)]
+    ws = aqd.workspace_for(jobs1, Wt, 1, 1)
+    aqd.conv_int_grouped(jobs1, Wt, 1, 1, rq=_rq(tower), workspace=ws)
+    ws.fill_(0x5A)
+    aqd.conv_expand_input(jobs2, Wt, 1, 1, ws)
+    aqd.conv_int_grouped_expanded(jobs2, Wt, 1, 1, rq=_rq(tower), workspace=ws)
+    assert aqd.last_conv_path() == 3
+    torch.cuda.synchronize()
+    for l in range(3):
+        assert torch.equal(y1[l].data, y2[l].data), f"tower level {l}"
+    # two convs from one expansion of the tower output
+    ws2 = aqd.workspace_for([(y1[l], y1[l], None, l) for l in range(3)], Wt, 1, 1)
+    aqd.conv_expand_input([(y1[l], None, None, l) for l in range(3)], Wt, 1, 1, ws2)
+    outs = {}
+    for cv in (cls, box):
+        W, _ = weights(cv.w, 2)
+        ys = [aqd.DTensor.empty(t.n, t.h, t.w, cv.cout, 32) for t in xts]
+        aqd.conv_int_grouped_expanded([(y1[l], ys[l], None, l) for l in range(3)], W, 1, 1,
+                                      rq=aqd.RequantParams.from_numpy(None, None, cv.bias), workspace=ws2)
+        outs[cv.cout] = ys
+    torch.cuda.synchronize()
+    wpt = oracle.pack(tower.w.reshape(-1, tower.cin), 2)
+    for l in range(3):
+        mid = _ref_conv(xts[l], wpt, tower, level=l)  # the oracle's own tower output
+        assert_same(y1[l].data.cpu().numpy().reshape(mid.packed.shape), mid.packed, 256, 2, f"tower {l}")
+        for cv in (cls, box):
+            wp = oracle.pack(cv.w.reshape(-1, cv.cin), 2)
+            want = _ref_conv(mid, wp, cv, level=l).packed
+            assert_same(outs[cv.cout][l].data.cpu().numpy().reshape(want.shape), want, cv.cout, 32,
+                        f"head {cv.cout} level {l}")
+    assert aqd.device_status() == 0
+
+
+def test_expanded_conv_needs_an_applicable_workspace():
+    rng = np.random.default_rng(3)
+    W, _ = weights(synth.weight_codes(rng, (64, 3, 3, 64), 2), 2)  # cin 64: no workspace path
+    X = aqd.DTensor.empty(1, 8, 8, 64, 2)
+    Y = aqd.DTensor.empty(1, 8, 8, 64, 32)
+    buf = torch.zeros(1 << 20, dtype=torch.uint8, device="cuda")
+    with pytest.raises(aqd.AqdError) as e:
+        aqd.conv_int_grouped_expanded([(X, Y, None, 0)], W, 1, 1, workspace=buf)
+    assert e.value.status == 1
+    with pytest.raises(aqd.AqdError) as e:
+        aqd.conv_expand_input([(X, Y, None, 0)], W, 1, 1, buf)
+    assert e.value.status == 1

@@ -127,6 +127,23 @@ def oracle_tower_sample(wl, max_levels=None):
     return ops, time.perf_counter() - t0
 
 
+def max_over_ranks(x: float, device) -> float:
+    """The largest x over all ranks (the job's time is its slowest replica's)."""
+    import torch
+    import torch.distributed as dist
+    if not dist.is_available() or not dist.is_initialized() or dist.get_world_size() == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tops(ops_per_step: float, steps: int, world: int, max_total_ms: float) -> float:
+    """Whole-job throughput of N replicas: every rank runs the same step, so the job does
+    world * ops_per_step * steps operations in the slowest rank's time."""
+    return world * ops_per_step * steps / (max_total_ms * 1e-3) / 1e12
+
+
 def omp_threads():
     v = os.environ.get("OMP_NUM_THREADS")
     return int(v) if v and v.isdigit() else (os.cpu_count() or 1)
@@ -293,13 +310,9 @@ def main():
     if world > 1:
         dist.barrier()
     assert aqd.device_status(stream) == 0
-    total_ms = float(sum(step_ms))
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(float(sum(step_ms)), dev)
     ms_per_step = total_ms / args.steps
-    value = world * ops_step * args.steps / (total_ms * 1e-3) / 1e12
+    value = job_tops(ops_step, args.steps, world, total_ms)
 
     # end to end through the public API: pinned host inputs -> device, step, head outputs -> host
     h_in = [x.data.cpu().pin_memory() for x in xs]

@@ -133,10 +133,11 @@ const char* aqd_last_error(void);
 aqd_status aqd_device_status(aqd_stream_t stream, int32_t* code);
 
 /* Diagnostics: force the convolution kernel (0 = automatic choice, 1 = tensor-core
- * kernel when the shape allows it, 2 = CUDA-core kernel); returns the previous setting,
- * or -1 for an unknown value. aqd_last_conv_path() reports the kernel the calling
- * thread's last successful conv call used (1 tensor core unpacking in-kernel, 2 CUDA core,
- * 3 tensor core fed from the expanded workspace, 0 none yet). */
+ * kernel when the shape allows it, 2 = CUDA-core kernel, 3 = as 1 but never on CTA
+ * pairs); returns the previous setting, or -1 for an unknown value. aqd_last_conv_path()
+ * reports the kernel the calling thread's last successful conv call used (1 tensor core
+ * unpacking in-kernel, 2 CUDA core, 3 tensor core fed from the expanded workspace, 4 the
+ * same on CTA pairs sharing each weight tile, 0 none yet). */
 int32_t aqd_set_conv_path(int32_t path);
 int32_t aqd_last_conv_path(void);
 

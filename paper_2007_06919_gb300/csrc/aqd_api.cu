@@ -17,7 +17,7 @@ namespace aqd {
 
 static thread_local std::string g_last_error;
 static thread_local int32_t g_last_path = 0;
-static int32_t g_forced_path = 0;  // 0 auto, 1 tensor core, 2 direct
+static int32_t g_forced_path = 0;  // 0 auto, 1 tensor core, 2 direct, 3 tensor core without CTA pairs
 
 __device__ uint32_t g_status_word;
 
@@ -138,7 +138,7 @@ aqd_status aqd_device_status(aqd_stream_t stream, int32_t* code) {
 }
 
 int32_t aqd_set_conv_path(int32_t path) {
-  if (path < 0 || path > 2) return -1;
+  if (path < 0 || path > 3) return -1;
   const int32_t old = g_forced_path;
   g_forced_path = path;
   return old;
@@ -359,7 +359,8 @@ static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aq
   const bool tc_ok = a.x_bits <= 4 && max_w <= 15 && (a.cin % 32) == 0 && bound < (1LL << 24);
   const bool direct_ok = bound < (1LL << 31);
   int path = tc_ok ? 1 : 2;
-  if (g_forced_path == 1 && tc_ok) path = 1;
+  if ((g_forced_path == 1 || g_forced_path == 3) && tc_ok) path = 1;
+  a.no_pair = g_forced_path == 3 ? 1 : 0;
   if (g_forced_path == 2) path = 2;
   // expanded-activation path when a large enough, aligned workspace is supplied
   a.ws = nullptr;
@@ -384,7 +385,8 @@ static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aq
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   int rc = path == 1 ? launch_conv_tc(a, st, &err) : launch_conv_direct(a, st, &err);
   if (rc) return fail((aqd_status)rc, err);
-  if (stage != kStageExpandOnly) g_last_path = (path == 1 && a.ws) ? 3 : path;
+  if (stage != kStageExpandOnly)
+    g_last_path = (path == 1 && a.ws) ? (conv_tc_uses_pair(a) ? 4 : 3) : path;
   return AQD_OK;
 }
 

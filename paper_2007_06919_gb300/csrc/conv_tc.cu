@@ -49,10 +49,6 @@ constexpr int BK = 128;            // K bytes per stage
 #endif
 constexpr int kEpiWarps = AQD_EPI_WARPS;  // 4 or 8
 static_assert(kEpiWarps == 4 || kEpiWarps == 8, "epilogue warps: 4 or 8");
-#ifndef AQD_EPI_BATCH
-#define AQD_EPI_BATCH 1
-#endif
-constexpr int kEpiBatch = AQD_EPI_BATCH;  // 32-column groups per TMEM load wait (1 or 2)
 constexpr int kEpiThreads = kEpiWarps * 32;
 #ifndef AQD_TMA_WARPS
 #define AQD_TMA_WARPS 1
@@ -256,8 +252,8 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
 // The MMA is always M=128 (one sub-tile, one CTA): M=256 exists only for cta_group::2.
 constexpr int kMmaM = 128;
 static_assert(kSubA == kMmaM * BK, "one sub-tile is one M=128 MMA operand");
-__device__ __forceinline__ uint32_t idesc_e4m3(int n) {
-  return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(kMmaM >> 4) << 24);
+__device__ __forceinline__ uint32_t idesc_e4m3(int n, int m = kMmaM) {
+  return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
 }
 
 __device__ __forceinline__ void mma_e4m3(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
@@ -272,6 +268,54 @@ __device__ __forceinline__ void mma_commit(uint32_t bar) {
                ::"r"(bar) : "memory");
 }
 
+// ---- 2-SM (CTA pair) forms. In a cluster of two CTAs, the even CTA issues
+// tcgen05.mma.cta_group::2 with M = 256: each CTA holds its 128 rows of A and half of the
+// N rows of B in shared memory at the same offsets, and receives its 128 rows x N columns
+// of D in its own TMEM.
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// shared::cluster address of shared-memory offset `saddr` in CTA `rank` of this cluster
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+__device__ __forceinline__ void mma_e4m3_pair(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}"
+      ::"r"(d_tmem), "l"(a), "l"(b), "r"(idesc), "r"(acc) : "memory");
+}
+// arrive on the barrier at this shared-memory offset in both CTAs of the pair, once the
+// MMAs issued so far have completed
+__device__ __forceinline__ void mma_commit_pair_both(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;"
+      ::"r"(bar), "h"((uint16_t)3) : "memory");
+}
+__device__ __forceinline__ void mma_commit_pair(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];"
+               ::"r"(bar) : "memory");
+}
+// TMA load into this CTA's shared memory that signals a barrier in either CTA of the pair
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, int x, int y,
+                                                 uint32_t bar_cluster) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.cta_group::2"
+      " [%0], [%1, {%2, %3}], [%4];"
+      ::"r"(dst), "l"((uint64_t)map), "r"(x), "r"(y), "r"(bar_cluster) : "memory");
+}
+
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
@@ -282,6 +326,34 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
       : "r"(taddr));
 }
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+// 32 columns of this warp's TMEM lanes (only the first 16 when !full)
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, bool full, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  if (full)
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]),
+          "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
+          "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr + 16));
+}
+// Makes every later use of r depend on this point (placed right after tcgen05.wait::ld, so
+// the compiler cannot move a read of a TMEM-loaded register above the wait).
+__device__ __forceinline__ void reg_fence32(uint32_t (&r)[32]) {
+  asm volatile("" : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]),
+               "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]),
+               "+r"(r[14]), "+r"(r[15]));
+  asm volatile("" : "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]),
+               "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]),
+               "+r"(r[28]), "+r"(r[29]), "+r"(r[30]), "+r"(r[31]));
+}
 
 // ---------------------------------------------------------------- tile bookkeeping
 
@@ -293,10 +365,10 @@ struct TileInfo {
 struct FlatTile {
   int img, v0;
 };
-__device__ __forceinline__ FlatTile flat_tile(const ConvJobDev& jb, int mt) {
+__device__ __forceinline__ FlatTile flat_tile(const ConvJobDev& jb, int mt, int rows = 128) {
   FlatTile f;
   f.img = mt / jb.tpi;
-  f.v0 = (mt - f.img * jb.tpi) * 128;
+  f.v0 = (mt - f.img * jb.tpi) * rows;
   return f;
 }
 __device__ __forceinline__ TileInfo tile_info(const Params& p, int t) {
@@ -443,11 +515,16 @@ __device__ __forceinline__ void load_chunk(const Params& p, RowCursor<kXBits>& r
   }
 }
 
-template <int kXBits, bool kChunkInTap, bool kFlat>
+template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair>
 __global__ void __launch_bounds__(threads_for(kFlat), 1)
 conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_a,
                const __grid_constant__ Params p) {
+  static_assert(!kPair || kFlat, "the CTA-pair form exists for the workspace path only");
   constexpr int kTma = tma_warps(kFlat);
+  // CTA pair: this CTA's rank; the even CTA issues the MMAs; a tile has 256 rows
+  const uint32_t rank = kPair ? cluster_ctarank() : 0u;
+  const bool leader = rank == 0;
+  constexpr int kTileRows = kPair ? 256 : 128;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // align by pointer arithmetic on the shared array itself (no integer round trip), so the
   // compiler keeps every access through `smem` in the shared state space (lds/sts)
@@ -470,7 +547,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
   const int warp = threadIdx.x / 32;
   const int lane = threadIdx.x % 32;
   const int BN = p.bn;
-  const uint32_t stage_b_bytes = (uint32_t)BN * BK;
+  const uint32_t stage_b_bytes = (uint32_t)(kPair ? BN / 2 : BN) * BK;  // this CTA's rows of B
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -479,16 +556,23 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(b_tfull + 8 * b, 1);
-      mbar_init(b_tempty + 8 * b, kEpiWarps);     // one arrive per epilogue warp
+      mbar_init(b_tempty + 8 * b, kPair ? 2 * kEpiWarps : kEpiWarps);  // one arrive per epilogue warp
     }
     mbar_init(b_final, 1);
     *abort_flag = 0;
     fence_barrier_init();
   }
   if (warp == kWarpMma) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
-                 ::"r"(smem_u32(tmem_slot)), "r"(p.tmem_cols) : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    if constexpr (kPair) {
+      // one warp of each CTA of the pair allocates, collectively, the same columns in both
+      asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;"
+                   ::"r"(smem_u32(tmem_slot)), "r"(p.tmem_cols) : "memory");
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+    } else {
+      asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
+                   ::"r"(smem_u32(tmem_slot)), "r"(p.tmem_cols) : "memory");
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
   }
   if (warp >= kWarpTma && warp < kWarpTma + kTmaWarps && lane == 0)
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmap_w) : "memory");
@@ -496,17 +580,20 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmap_a) : "memory");
   tc_fence_before();
   __syncthreads();
+  // the peer signals this CTA's barriers (and the leader's MMAs read the peer's shared
+  // memory) only after both CTAs have initialised them
+  if constexpr (kPair) cluster_sync();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
   const int nk = p.num_kchunks;
-  const int first_tile = blockIdx.x;
-  const int tile_stride = gridDim.x;
+  const int first_tile = kPair ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+  const int tile_stride = kPair ? (int)(gridDim.x >> 1) : (int)gridDim.x;
 
   if (warp == kWarpMma) {
     // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      const uint32_t idesc = idesc_e4m3(BN);
+    if (lane == 0 && leader) {
+      const uint32_t idesc = idesc_e4m3(BN, kPair ? 2 * kMmaM : kMmaM);
       // descriptors of stage 0, k-step 0; later stages / sub-tiles / k-steps add
       // (byte offset >> 4) to the 14-bit start-address field (shared addresses < 2^18)
       // the descriptors' high words are constant; stages / sub-tiles / k-steps only move the
@@ -530,18 +617,27 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
           for (int kk = 0; kk < BK / 32; ++kk) {
             const uint32_t acc = (q > 0 || kk > 0) ? 1u : 0u;
             const uint64_t db = ((uint64_t)b_hi << 32) | (b_lo + 2 * kk);
+            if constexpr (kPair) {
+              mma_e4m3_pair(d0, ((uint64_t)a_hi << 32) | (a_lo + 2 * kk), db, idesc, acc);
+            } else {
 #pragma unroll
-            for (int j = 0; j < kSub; ++j)
-              mma_e4m3(d0 + j * BN, ((uint64_t)a_hi << 32) | (a_lo + j * (kSubA >> 4) + 2 * kk), db, idesc, acc);
+              for (int j = 0; j < kSub; ++j)
+                mma_e4m3(d0 + j * BN, ((uint64_t)a_hi << 32) | (a_lo + j * (kSubA >> 4) + 2 * kk), db, idesc, acc);
+            }
           }
-          mma_commit(b_empty + 8 * s);
+          if constexpr (kPair) mma_commit_pair_both(b_empty + 8 * s);
+          else mma_commit(b_empty + 8 * s);
           if (++s == (uint32_t)S) { s = 0; ph ^= 1; }
         }
-        if (ok) mma_commit(b_tfull + 8 * buf);
+        if (ok) {
+          if constexpr (kPair) mma_commit_pair_both(b_tfull + 8 * buf);
+          else mma_commit(b_tfull + 8 * buf);
+        }
       }
       if (!ok) fail(abort_flag, p.status);
       // drain: every MMA issued above has completed once this barrier flips
-      mma_commit(b_final);
+      if constexpr (kPair) mma_commit_pair(b_final);
+      else mma_commit(b_final);
       if (!mbar_wait(b_final, 0, abort_flag)) fail(abort_flag, p.status);
     }
   } else if (warp >= kWarpTma && warp < kWarpTma + kTma) {
@@ -557,7 +653,26 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
         for (int q = 0; q < nk; ++q, ++it, s = (s + 1 == (uint32_t)S) ? 0 : s + 1, ph ^= (s == 0)) {
           if ((int)(it % kTma) != tw) continue;
           if (!mbar_wait(b_empty + 8 * s, ph ^ 1, abort_flag)) { ok = false; break; }
-          if constexpr (kFlat) {
+          if constexpr (kPair) {
+            // this CTA's 128 rows of A and its half of B; both CTAs' copies complete on the
+            // leader's "full" barrier, which the leader arms with the bytes of all four
+            const ConvJobDev& jb = p.jobs[ti.job];
+            const FlatTile ft = flat_tile(jb, ti.mt, kTileRows);
+            const int tap = q / p.cin_chunks, cb = q - tap * p.cin_chunks;
+            const int r = tap / p.kw, sx = tap - r * p.kw;
+            const int row = jb.row_off + ft.img * jb.hp * jb.wp + ft.v0 + (int)rank * 128 + r * jb.wp + sx;
+            const int brow = ti.nt * BN + (int)rank * (BN / 2);
+            if (leader) {
+              mbar_arrive_expect_tx(b_full + 8 * s, 2 * (stage_b_bytes + kStageA));
+              tma_load_2d(s_a + s * kStageA, &tmap_a, cb * BK, row, b_full + 8 * s);
+              tma_load_2d(s_b + s * stage_b_bytes, &tmap_w, q * BK, brow, b_full + 8 * s);
+            } else {
+              const uint32_t fb = mapa_shared(b_full + 8 * s, 0);
+              tma_load_2d_pair(s_a + s * kStageA, &tmap_a, cb * BK, row, fb);
+              tma_load_2d_pair(s_b + s * stage_b_bytes, &tmap_w, q * BK, brow, fb);
+            }
+            continue;
+          } else if constexpr (kFlat) {
             // A: 128 consecutive rows of the padded byte image, shifted by the tap (r, s)
             const ConvJobDev& jb = p.jobs[ti.job];
             const FlatTile ft = flat_tile(jb, ti.mt);
@@ -696,53 +811,43 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       if (!mbar_wait(b_tfull + 8 * buf, (lt >> 1) & 1, abort_flag)) { ok = false; break; }
       tc_fence_after();
 
-      // this warp's (sub-tile, 32-column group) units, two per TMEM wait
+      // This warp's (sub-tile, 32-column group) units. The TMEM load of the next unit is in
+      // flight while the current one is converted and stored; no register written by a
+      // tcgen05.ld is read before the tcgen05.wait::ld that covers it.
       const int ngrp = (BN + 31) / 32;
       const int nunits = kSub * ngrp;
-      for (int u0 = gi; u0 < nunits; u0 += kEpiBatch * kGroups) {
-        const int u1 = u0 + kGroups;
-        const bool two = kEpiBatch == 2 && u1 < nunits;  // warp-uniform
-        uint32_t va[32], vb[32];
-        int subA = u0 / ngrp, g0A = (u0 % ngrp) * 32;
-        int subB = two ? u1 / ngrp : 0, g0B = two ? (u1 % ngrp) * 32 : 0;
-        const int ncA = (BN - g0A) < 32 ? (BN - g0A) : 32;
-        const int ncB = (BN - g0B) < 32 ? (BN - g0B) : 32;
-        __syncwarp();
-        {
-          uint32_t r16[16];
-          const uint32_t ca = lane_base + buf * (uint32_t)(kSub * BN) + subA * (uint32_t)BN + g0A;
-          tmem_ld16(ca, r16);
-#pragma unroll
-          for (int i = 0; i < 16; ++i) va[i] = r16[i];
-          if (ncA == 32) tmem_ld16(ca + 16, r16);
-#pragma unroll
-          for (int i = 0; i < 16; ++i) va[16 + i] = (ncA == 32) ? r16[i] : 0u;
-        }
-        if (two) {
-          uint32_t r16[16];
-          const uint32_t cb = lane_base + buf * (uint32_t)(kSub * BN) + subB * (uint32_t)BN + g0B;
-          tmem_ld16(cb, r16);
-#pragma unroll
-          for (int i = 0; i < 16; ++i) vb[i] = r16[i];
-          if (ncB == 32) tmem_ld16(cb + 16, r16);
-#pragma unroll
-          for (int i = 0; i < 16; ++i) vb[16 + i] = (ncB == 32) ? r16[i] : 0u;
-        }
+      const uint32_t tbuf = lane_base + buf * (uint32_t)(kSub * BN);
+      uint32_t va[32], vn[32];
+      __syncwarp();
+      if (gi < nunits) {
+        tmem_ld32(tbuf + (gi / ngrp) * (uint32_t)BN + (gi % ngrp) * 32, BN - (gi % ngrp) * 32 >= 32, va);
         tmem_wait_ld();
-        for (int h = 0; h < (two ? 2 : 1); ++h) {
-          const uint32_t* v = h ? vb : va;
-          const int sub = h ? subB : subA, g0 = h ? g0B : g0A, ncols = h ? ncB : ncA;
-          int m;  // output pixel index within the job
-          if constexpr (kFlat) {
-            const FlatTile ft = flat_tile(jb, ti.mt);
-            const int v = ft.v0 + quarter * 32 + lane;  // virtual row at the padded width
-            const int ho = v / jb.wp, wo = v - (v / jb.wp) * jb.wp;
-            if (v >= jb.vimg || wo >= jb.wo) continue;  // junk column or past the image
-            m = (ft.img * jb.ho + ho) * jb.wo + wo;
-          } else {
-            m = ti.mt * BM + sub * 128 + quarter * 32 + lane;
-            if (m >= jb.m_total) continue;
-          }
+        reg_fence32(va);
+      }
+      for (int u0 = gi; u0 < nunits; u0 += kGroups) {
+        const int un = u0 + kGroups;
+        if (un < nunits)
+          tmem_ld32(tbuf + (un / ngrp) * (uint32_t)BN + (un % ngrp) * 32, BN - (un % ngrp) * 32 >= 32, vn);
+        const int sub = u0 / ngrp, g0 = (u0 % ngrp) * 32;
+        const int ncols = (BN - g0) < 32 ? (BN - g0) : 32;
+        if (ncols < 32) {
+#pragma unroll
+          for (int i = 16; i < 32; ++i) va[i] = 0u;  // only the first 16 columns were loaded
+        }
+        const uint32_t* v = va;
+        int m;  // output pixel index within the job
+        bool row_ok;
+        if constexpr (kFlat) {
+          const FlatTile ft = flat_tile(jb, ti.mt, kTileRows);
+          const int vr = ft.v0 + (int)rank * 128 + quarter * 32 + lane;  // virtual row at the padded width
+          const int ho = vr / jb.wp, wo = vr - (vr / jb.wp) * jb.wp;
+          row_ok = vr < jb.vimg && wo < jb.wo;  // else a junk column or past the image
+          m = (ft.img * jb.ho + ho) * jb.wo + wo;
+        } else {
+          m = ti.mt * BM + sub * 128 + quarter * 32 + lane;
+          row_ok = m < jb.m_total;
+        }
+        if (row_ok) {
           uint8_t* yrow = jb.y + (int64_t)m * p.y_row_bytes;
           const int ch0 = ti.nt * BN + g0;
           if (mode == 1) {
@@ -766,10 +871,10 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
           } else if (mode == 2) {
             int32_t* yr = reinterpret_cast<int32_t*>(yrow) + ch0;
             const bool full = ncols == 32 && ch0 + 32 <= p.cout;
-#pragma unroll
+  #pragma unroll
             for (int q = 0; q < 8; ++q) {
               int32_t o[4];
-#pragma unroll
+  #pragma unroll
               for (int k = 0; k < 4; ++k) {
                 const float f = __uint_as_float(v[4 * q + k]);
                 o[k] = magic ? __float_as_int(__fmaf_rn(f, 262144.0f, kMagic)) + epf[g0 + 4 * q + k].x
@@ -778,7 +883,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
               if (full) {
                 reinterpret_cast<int4*>(yr)[q] = make_int4(o[0], o[1], o[2], o[3]);
               } else {
-#pragma unroll
+  #pragma unroll
                 for (int k = 0; k < 4; ++k)
                   if (4 * q + k < ncols && ch0 + 4 * q + k < p.cout) yr[4 * q + k] = o[k];
               }
@@ -795,7 +900,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
             }
             uint32_t vv[32];  // local copies: only this rare path goes through the stack
             int32_t oo[32];
-#pragma unroll
+  #pragma unroll
             for (int i = 0; i < 32; ++i) vv[i] = v[i];
             general_epilogue(p, vv, epi + g0, srow, ch0, ncols, oo);
             if (out_bits == 32) {
@@ -809,20 +914,36 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
             }
           }
         }
+        if (un < nunits) {
+          tmem_wait_ld();
+          reg_fence32(vn);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) va[i] = vn[i];
+        }
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(b_tempty + 8 * buf);
+      if (lane == 0) {
+        if (kPair && !leader) mbar_arrive_cluster(mapa_shared(b_tempty + 8 * buf, 0));
+        else mbar_arrive(b_tempty + 8 * buf);
+      }
     }
     if (!ok) fail(abort_flag, p.status);
   }
 
   tc_fence_before();
   __syncthreads();
+  // neither CTA of a pair leaves while the leader's MMAs may still read the peer's shared
+  // memory or write its TMEM (the leader's MMA thread drained them before the barrier)
+  if constexpr (kPair) cluster_sync();
   if (warp == kWarpMma) {
     tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;"
-                 ::"r"(tmem_base), "r"(p.tmem_cols) : "memory");
+    if constexpr (kPair)
+      asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;"
+                   ::"r"(tmem_base), "r"(p.tmem_cols) : "memory");
+    else
+      asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;"
+                   ::"r"(tmem_base), "r"(p.tmem_cols) : "memory");
   }
 }
 
@@ -967,10 +1088,10 @@ static EncodeTiledFn get_encode_fn(std::string* err) {
   return fn;
 }
 
-template <int kXBits, bool kChunkInTap, bool kFlat>
+template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair = false>
 static int launch_bits(const Params& prm, const CUtensorMap& map, const CUtensorMap& map_a, int grid,
                        size_t smem, cudaStream_t stream, std::string* err) {
-  auto kern = conv_tc_kernel<kXBits, kChunkInTap, kFlat>;
+  auto kern = conv_tc_kernel<kXBits, kChunkInTap, kFlat, kPair>;
   // The opt-in limit is raised to the device maximum, never lowered to this call's size:
   // a CUDA graph node captured earlier with a larger plan must stay launchable (a graph
   // node, or a tool relaunching it, is checked against the function's current limit).
@@ -980,13 +1101,35 @@ static int launch_bits(const Params& prm, const CUtensorMap& map, const CUtensor
   if ((size_t)optin < smem) { *err = "conv_tc: shared memory plan exceeds the device limit"; return 2; }
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
   if (e != cudaSuccess) { *err = std::string("cudaFuncSetAttribute: ") + cudaGetErrorString(e); return 3; }
-  kern<<<grid, threads_for(kFlat), smem, stream>>>(map, map_a, prm);
+  if constexpr (kPair) {
+    // clusters of two CTAs (one pair per two SMs)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3((unsigned)threads_for(kFlat));
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, kern, map, map_a, prm);
+    if (e != cudaSuccess) { *err = std::string("conv_tc pair launch: ") + cudaGetErrorString(e); return 3; }
+  } else {
+    kern<<<grid, threads_for(kFlat), smem, stream>>>(map, map_a, prm);
+  }
   e = cudaGetLastError();
   if (e != cudaSuccess) { *err = std::string("conv_tc launch: ") + cudaGetErrorString(e); return 3; }
   return 0;
 }
 
 }  // namespace tc
+
+bool conv_tc_uses_pair(const ConvArgs& a) {
+  return a.ws != nullptr && a.bn == 256 && tc::kSub == 1 && !a.no_pair;
+}
 
 int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   using namespace tc;
@@ -997,6 +1140,10 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   // flat path: the activations are expanded into the workspace first (stride 1,
   // cin % 128 == 0; the API checks both before passing a workspace)
   const bool flat = a.ws != nullptr;
+  // CTA pairs (cta_group::2, M = 256 per tile) for full 256-channel N tiles of the
+  // workspace path: each SM then streams half of the weight tile per K chunk
+  const bool pair = conv_tc_uses_pair(a);
+  const int tile_rows = pair ? 256 : 128;
   int tiles = 0;
   int64_t rows = 0;
   for (int j = 0; j < a.njobs; ++j) {
@@ -1007,7 +1154,7 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
       jb.hp = jb.h + 2 * a.pad;
       jb.wp = jb.w + 2 * a.pad;
       jb.vimg = jb.ho * jb.wp;
-      jb.tpi = (jb.vimg + 127) / 128;
+      jb.tpi = (jb.vimg + tile_rows - 1) / tile_rows;
       jb.row_off = (int32_t)rows;
       rows += (int64_t)jb.n * jb.hp * jb.wp;
       tiles += jb.n * jb.tpi * prm.n_tiles;
@@ -1033,8 +1180,9 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   prm.acc_small = a.acc_bound < (1LL << 22) ? 1 : 0;
   prm.cin_chunks = a.cin / BK;
   prm.status = a.status;
-  // shared memory plan: stages of (BM x 128 A bytes + BN x 128 B bytes)
-  const size_t stage_bytes = (size_t)kStageA + (size_t)BN * BK;
+  // shared memory plan: stages of (BM x 128 A bytes + this CTA's B rows x 128 bytes)
+  const int b_rows = pair ? BN / 2 : BN;
+  const size_t stage_bytes = (size_t)kStageA + (size_t)b_rows * BK;
   const size_t epi_bytes = 256 * sizeof(EpiChan) + 256 * sizeof(int4);
   const size_t bar_bytes = 8 * (2 * kMaxStages + 5) + 16;
   const size_t budget = 232448 - 1024;  // max dynamic smem per block minus alignment slack
@@ -1048,7 +1196,7 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   if (stages < tma_warps(flat)) { *err = "conv_tc: fewer pipeline stages than TMA issuers"; return 2; }
   prm.stages = stages;
   prm.off_b = (uint32_t)(stages * kStageA);
-  prm.off_epi = prm.off_b + (uint32_t)(stages * BN * BK);
+  prm.off_epi = prm.off_b + (uint32_t)(stages * b_rows * BK);
   prm.off_bar = prm.off_epi + (uint32_t)epi_bytes;
   const size_t smem = 1024 + prm.off_bar + bar_bytes;
   int cols = 32;
@@ -1060,7 +1208,7 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   CUtensorMap map;
   cuuint64_t gdim[2] = {(cuuint64_t)a.k_pad, (cuuint64_t)a.cout_pad};
   cuuint64_t gstride[1] = {(cuuint64_t)a.k_pad};
-  cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)BN};
+  cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)b_rows};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = enc(&map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)a.w_e4m3, gdim, gstride, box, estr,
                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -1070,7 +1218,8 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const int grid = tiles < sms ? tiles : sms;
+  int grid = tiles < sms ? tiles : sms;
+  if (pair) grid = 2 * (tiles < sms / 2 ? tiles : sms / 2);
   const bool in_tap = (a.cin % BK) == 0;
   CUtensorMap map_a = map;  // unused unless flat
   if (flat) {
@@ -1105,6 +1254,7 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
       *err = "cuTensorMapEncodeTiled (activations) failed: " + std::to_string((int)r2);
       return 3;
     }
+    if (pair) return launch_bits<2, true, true, true>(prm, map, map_a, grid, smem, stream, err);
     return launch_bits<2, true, true>(prm, map, map_a, grid, smem, stream, err);
   }
   switch (a.x_bits) {

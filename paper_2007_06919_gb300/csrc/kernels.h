@@ -47,6 +47,7 @@ struct ConvArgs {
   int64_t ws_rows;        // rows of cin bytes available in the workspace
   int32_t skip_expand;    // workspace already holds the expansion: launch only the conv
   int32_t expand_only;    // launch only the expansion into the workspace
+  int32_t no_pair;        // workspace path: use the one-CTA kernel even for 256-wide N tiles
   uint32_t* status;       // device status word
 };
 
@@ -60,6 +61,8 @@ WeightGeom weight_geom(int32_t cout, int32_t kh, int32_t kw, int32_t cin);
 
 // 0 on success, else an aqd_status value; *err gets a message.
 int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err);
+// whether launch_conv_tc runs these arguments on CTA pairs (cta_group::2)
+bool conv_tc_uses_pair(const ConvArgs& a);
 int launch_conv_direct(const ConvArgs& a, cudaStream_t stream, std::string* err);
 int launch_prepare_weights(const uint8_t* w_packed, int32_t w_bits, int32_t w_format,
                            const WeightGeom& g, uint8_t* out, cudaStream_t stream,

@@ -8,7 +8,13 @@ from paper_2007_06919_gb300 import synth
 
 pytestmark = pytest.mark.gpu
 
-TC, DIRECT = 1, 2
+TC, DIRECT, TC_NO_PAIR = 1, 2, 3
+
+
+def ws_path(cout: int) -> int:
+    """Path reported for the workspace-fed tensor-core kernel: CTA pairs (4) for 256-wide
+    N tiles (cout above 240), one CTA (3) otherwise."""
+    return 4 if cout > 240 else 3
 
 
 def _params(rng, levels, cout, out_bits, calib_std=None):
@@ -85,9 +91,11 @@ WS_CASES = [c for c in CASES if c[9] == 1 and c[6] % 128 == 0 and c[0] <= 4 and 
 
 
 @pytest.mark.parametrize("case", WS_CASES, ids=[str(i) for i in range(len(WS_CASES))])
-def test_conv_workspace_path_bit_exact(case):
+@pytest.mark.parametrize("pairs", [True, False])
+def test_conv_workspace_path_bit_exact(case, pairs):
     """The expanded-activation path (one expansion pass into a caller workspace, then TMA
-    tiles of the zero-padded byte image, junk columns dropped) gives the same bytes."""
+    tiles of the zero-padded byte image, junk columns dropped) gives the same bytes, on CTA
+    pairs (256-wide N tiles) and on single CTAs."""
     xb, wb, fmt, n, h, wd, cin, cout, k, stride, pad, ob = case
     rng = np.random.default_rng(hash(case) % 2 ** 32 + 1)
     x = synth.act_codes(rng, (n, h, wd, cin), xb)
@@ -95,21 +103,23 @@ def test_conv_workspace_path_bit_exact(case):
     std = np.sqrt(k * k * cin * np.mean(np.arange(1 << xb) ** 2) * (1 << (2 * wb - 2)) / 3)
     m0, sh, b = _params(rng, 1, cout, ob if ob != 32 else 4, calib_std=std)
     got, want, used = conv_pair(x, xb, w, wb, stride=stride, pad=pad, out_bits=ob, m0=m0, shift=sh, bias=b,
-                                path=TC, workspace=True)
-    assert used == 3
+                                path=TC if pairs else TC_NO_PAIR, workspace=True)
+    assert used == (ws_path(cout) if pairs else 3)
     assert_same(got, want, cout, ob, f"workspace case {case}")
 
 
 @pytest.mark.parametrize("shape", [(1, 1, 1), (2, 3, 300), (1, 37, 2), (3, 7, 11)])
-def test_workspace_path_edge_shapes(shape):
+@pytest.mark.parametrize("pairs", [True, False])
+def test_workspace_path_edge_shapes(shape, pairs):
     """Tiles that cross image rows and images, 1x1 images and single-column images."""
     n, h, wd = shape
     rng = np.random.default_rng(n * 1000 + h * 10 + wd)
     x = synth.act_codes(rng, (n, h, wd, 256), 2)
     w = synth.weight_codes(rng, (256, 3, 3, 256), 2)
     m0, sh, b = _params(rng, 1, 256, 2, calib_std=37.0)
-    got, want, used = conv_pair(x, 2, w, 2, out_bits=2, m0=m0, shift=sh, bias=b, path=TC, workspace=True)
-    assert used == 3
+    got, want, used = conv_pair(x, 2, w, 2, out_bits=2, m0=m0, shift=sh, bias=b,
+                                path=TC if pairs else TC_NO_PAIR, workspace=True)
+    assert used == (4 if pairs else 3)
     assert_same(got, want, 256, 2, f"edge {shape}")
 
 

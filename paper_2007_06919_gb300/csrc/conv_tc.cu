@@ -86,6 +86,8 @@ struct Params {
   int32_t bn, stages, tmem_cols;
   int32_t acc_small;  // |acc| < 2^22 guaranteed by K * max|x| * max|w|
   int32_t cin_chunks; // cin / 128 (flat path)
+  int32_t dp_tiles;   // tiles [0, dp_tiles) are bn wide; later ones are the two bn/2 halves
+                      // of the remaining full tiles (the last, partial wave)
   uint32_t off_b, off_epi, off_bar;
   uint32_t* status;
 };
@@ -358,7 +360,9 @@ __device__ __forceinline__ void reg_fence32(uint32_t (&r)[32]) {
 // ---------------------------------------------------------------- tile bookkeeping
 
 struct TileInfo {
-  int job, mt, nt;
+  int job, mt;
+  int bn;    // output channels of this tile: p.bn, or p.bn / 2 for a half tile
+  int col0;  // first output channel
 };
 // Flat path: M tile mt of a job covers virtual rows [v0, v0 + 128) of image img, where the
 // virtual grid holds the output rows at the padded input width wp (stride 1).
@@ -371,7 +375,15 @@ __device__ __forceinline__ FlatTile flat_tile(const ConvJobDev& jb, int mt, int 
   f.v0 = (mt - f.img * jb.tpi) * rows;
   return f;
 }
+// Global tile t -> (job, M tile, channel range). Tiles past dp_tiles split the remaining
+// full tiles into two halves of N, so the last, partial wave covers more SMs.
 __device__ __forceinline__ TileInfo tile_info(const Params& p, int t) {
+  int half = -1;
+  if (t >= p.dp_tiles) {
+    const int h = t - p.dp_tiles;
+    t = p.dp_tiles + (h >> 1);
+    half = h & 1;
+  }
   int j = 0;
 #pragma unroll 1
   while (j + 1 < p.njobs && t >= p.jobs[j + 1].tile_begin) ++j;
@@ -379,7 +391,9 @@ __device__ __forceinline__ TileInfo tile_info(const Params& p, int t) {
   TileInfo ti;
   ti.job = j;
   ti.mt = local / p.n_tiles;
-  ti.nt = local - ti.mt * p.n_tiles;
+  const int nt = local - ti.mt * p.n_tiles;
+  ti.bn = half < 0 ? p.bn : p.bn / 2;
+  ti.col0 = nt * p.bn + (half > 0 ? p.bn / 2 : 0);
   return ti;
 }
 
@@ -517,8 +531,8 @@ __device__ __forceinline__ void load_chunk(const Params& p, RowCursor<kXBits>& r
 
 template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair>
 __global__ void __launch_bounds__(threads_for(kFlat), 1)
-conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_a,
-               const __grid_constant__ Params p) {
+conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_wh,
+               const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ Params p) {
   static_assert(!kPair || kFlat, "the CTA-pair form exists for the workspace path only");
   constexpr int kTma = tma_warps(kFlat);
   // CTA pair: this CTA's rank; the even CTA issues the MMAs; a tile has 256 rows
@@ -574,8 +588,10 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
   }
-  if (warp >= kWarpTma && warp < kWarpTma + kTmaWarps && lane == 0)
+  if (warp >= kWarpTma && warp < kWarpTma + kTma && lane == 0) {
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmap_w) : "memory");
+    if (p.dp_tiles < p.total_tiles) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmap_wh) : "memory");
+  }
   if (kFlat && warp >= kWarpTma && warp < kWarpTma + kTma && lane == 0)
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmap_a) : "memory");
   tc_fence_before();
@@ -593,7 +609,8 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
   if (warp == kWarpMma) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0 && leader) {
-      const uint32_t idesc = idesc_e4m3(BN, kPair ? 2 * kMmaM : kMmaM);
+      const uint32_t idesc_full = idesc_e4m3(BN, kPair ? 2 * kMmaM : kMmaM);
+      const uint32_t idesc_half = idesc_e4m3(BN / 2, kPair ? 2 * kMmaM : kMmaM);
       // descriptors of stage 0, k-step 0; later stages / sub-tiles / k-steps add
       // (byte offset >> 4) to the 14-bit start-address field (shared addresses < 2^18)
       // the descriptors' high words are constant; stages / sub-tiles / k-steps only move the
@@ -603,18 +620,28 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       const uint32_t a_hi = (uint32_t)(da0 >> 32), b_hi = (uint32_t)(db0 >> 32);
       uint32_t it = 0, lt = 0, s = 0, ph = 0;
       bool ok = true;
+      bool next_ready = false;  // the stage after the current one is known to be full
       for (int t = first_tile; t < p.total_tiles && ok; t += tile_stride, ++lt) {
         const uint32_t buf = lt & 1;
+        const uint32_t idesc = t < p.dp_tiles ? idesc_full : idesc_half;
         if (!mbar_poll(b_tempty + 8 * buf, ((lt >> 1) & 1) ^ 1, abort_flag)) { ok = false; break; }
         tc_fence_after();
         const uint32_t d0 = tmem_base + buf * (uint32_t)(kSub * BN);  // sub-tile j at +j*BN
         for (int q = 0; q < nk; ++q, ++it) {
-          if (!mbar_poll(b_full + 8 * s, ph, abort_flag)) { ok = false; break; }
-          tc_fence_after();
+          // (operands written by TMA, or by producer threads followed by fence.proxy.async,
+          // are ordered for the MMA by the mbarrier phase alone; tcgen05.fence is needed only
+          // where TMEM changes hands, after the accumulator-empty wait above)
+          if (!next_ready && !mbar_poll(b_full + 8 * s, ph, abort_flag)) { ok = false; break; }
           const uint32_t a_lo = a_lo0 + ((s * kStageA) >> 4);
           const uint32_t b_lo = b_lo0 + ((s * stage_b_bytes) >> 4);
+          const uint32_t s_next = s + 1 == (uint32_t)S ? 0u : s + 1;
+          const uint32_t ph_next = s_next == 0 ? ph ^ 1u : ph;
 #pragma unroll
           for (int kk = 0; kk < BK / 32; ++kk) {
+            // The tensor pipe takes about one instruction at a time, so each issue waits for
+            // the previous MMA. Testing the next stage here, while the last MMAs of this
+            // chunk run, lets the next chunk's first MMA follow this chunk's commit at once.
+            if (kk == BK / 32 - 1) next_ready = mbar_test(b_full + 8 * s_next, ph_next);
             const uint32_t acc = (q > 0 || kk > 0) ? 1u : 0u;
             const uint64_t db = ((uint64_t)b_hi << 32) | (b_lo + 2 * kk);
             if constexpr (kPair) {
@@ -661,15 +688,17 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
             const int tap = q / p.cin_chunks, cb = q - tap * p.cin_chunks;
             const int r = tap / p.kw, sx = tap - r * p.kw;
             const int row = jb.row_off + ft.img * jb.hp * jb.wp + ft.v0 + (int)rank * 128 + r * jb.wp + sx;
-            const int brow = ti.nt * BN + (int)rank * (BN / 2);
+            const int brow = ti.col0 + (int)rank * (ti.bn / 2);
+            const CUtensorMap* wm = ti.bn == BN ? &tmap_w : &tmap_wh;
+            const uint32_t b_bytes = (uint32_t)(ti.bn / 2) * BK;
             if (leader) {
-              mbar_arrive_expect_tx(b_full + 8 * s, 2 * (stage_b_bytes + kStageA));
+              mbar_arrive_expect_tx(b_full + 8 * s, 2 * (b_bytes + kStageA));
               tma_load_2d(s_a + s * kStageA, &tmap_a, cb * BK, row, b_full + 8 * s);
-              tma_load_2d(s_b + s * stage_b_bytes, &tmap_w, q * BK, brow, b_full + 8 * s);
+              tma_load_2d(s_b + s * stage_b_bytes, wm, q * BK, brow, b_full + 8 * s);
             } else {
               const uint32_t fb = mapa_shared(b_full + 8 * s, 0);
               tma_load_2d_pair(s_a + s * kStageA, &tmap_a, cb * BK, row, fb);
-              tma_load_2d_pair(s_b + s * stage_b_bytes, &tmap_w, q * BK, brow, fb);
+              tma_load_2d_pair(s_b + s * stage_b_bytes, wm, q * BK, brow, fb);
             }
             continue;
           } else if constexpr (kFlat) {
@@ -679,12 +708,12 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
             const int tap = q / p.cin_chunks, cb = q - tap * p.cin_chunks;
             const int r = tap / p.kw, sx = tap - r * p.kw;
             const int row = jb.row_off + ft.img * jb.hp * jb.wp + ft.v0 + r * jb.wp + sx;
-            mbar_arrive_expect_tx(b_full + 8 * s, stage_b_bytes + kStageA);
+            mbar_arrive_expect_tx(b_full + 8 * s, (uint32_t)ti.bn * BK + kStageA);
             tma_load_2d(s_a + s * kStageA, &tmap_a, cb * BK, row, b_full + 8 * s);
           } else {
-            mbar_arrive_expect_tx(b_full + 8 * s, stage_b_bytes);
+            mbar_arrive_expect_tx(b_full + 8 * s, (uint32_t)ti.bn * BK);
           }
-          tma_load_2d(s_b + s * stage_b_bytes, &tmap_w, q * BK, ti.nt * BN, b_full + 8 * s);
+          tma_load_2d(s_b + s * stage_b_bytes, ti.bn == BN ? &tmap_w : &tmap_wh, q * BK, ti.col0, b_full + 8 * s);
         }
       }
       if (!ok) fail(abort_flag, p.status);
@@ -780,11 +809,12 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       // (R-32) equals rhu(u * M0, R): the low product word cannot carry into the result)
       // and |bias| <= 2^30 (acc + bias cannot leave int32 when |acc| < 2^24).
       int fast_req = 1, small_bias = 1;
+      const int TBN = ti.bn;  // this tile's width
       for (int col = et; col < 256; col += kEpiThreads) {
-        const int ch = ti.nt * BN + col;
+        const int ch = ti.col0 + col;
         EpiChan ec{};
         int4 ef = make_int4((int32_t)(0u - kMagicBits), 0, 0, 1);
-        if (col < BN && ch < p.cout) {
+        if (col < TBN && ch < p.cout) {
           const int64_t idx = (int64_t)jb.level * p.cout + ch;
           ec.bias = p.bias ? p.bias[idx] : 0;
           const bool sb = ec.bias >= -(1 << 30) && ec.bias <= (1 << 30);
@@ -814,22 +844,22 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       // This warp's (sub-tile, 32-column group) units. The TMEM load of the next unit is in
       // flight while the current one is converted and stored; no register written by a
       // tcgen05.ld is read before the tcgen05.wait::ld that covers it.
-      const int ngrp = (BN + 31) / 32;
+      const int ngrp = (TBN + 31) / 32;
       const int nunits = kSub * ngrp;
       const uint32_t tbuf = lane_base + buf * (uint32_t)(kSub * BN);
       uint32_t va[32], vn[32];
       __syncwarp();
       if (gi < nunits) {
-        tmem_ld32(tbuf + (gi / ngrp) * (uint32_t)BN + (gi % ngrp) * 32, BN - (gi % ngrp) * 32 >= 32, va);
+        tmem_ld32(tbuf + (gi / ngrp) * (uint32_t)BN + (gi % ngrp) * 32, TBN - (gi % ngrp) * 32 >= 32, va);
         tmem_wait_ld();
         reg_fence32(va);
       }
       for (int u0 = gi; u0 < nunits; u0 += kGroups) {
         const int un = u0 + kGroups;
         if (un < nunits)
-          tmem_ld32(tbuf + (un / ngrp) * (uint32_t)BN + (un % ngrp) * 32, BN - (un % ngrp) * 32 >= 32, vn);
+          tmem_ld32(tbuf + (un / ngrp) * (uint32_t)BN + (un % ngrp) * 32, TBN - (un % ngrp) * 32 >= 32, vn);
         const int sub = u0 / ngrp, g0 = (u0 % ngrp) * 32;
-        const int ncols = (BN - g0) < 32 ? (BN - g0) : 32;
+        const int ncols = (TBN - g0) < 32 ? (TBN - g0) : 32;
         if (ncols < 32) {
 #pragma unroll
           for (int i = 16; i < 32; ++i) va[i] = 0u;  // only the first 16 columns were loaded
@@ -849,7 +879,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
         }
         if (row_ok) {
           uint8_t* yrow = jb.y + (int64_t)m * p.y_row_bytes;
-          const int ch0 = ti.nt * BN + g0;
+          const int ch0 = ti.col0 + g0;
           if (mode == 1) {
             uint32_t gw[8];
             if (magic) {
@@ -1089,8 +1119,8 @@ static EncodeTiledFn get_encode_fn(std::string* err) {
 }
 
 template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair = false>
-static int launch_bits(const Params& prm, const CUtensorMap& map, const CUtensorMap& map_a, int grid,
-                       size_t smem, cudaStream_t stream, std::string* err) {
+static int launch_bits(const Params& prm, const CUtensorMap& map, const CUtensorMap& map_h, const CUtensorMap& map_a,
+                       int grid, size_t smem, cudaStream_t stream, std::string* err) {
   auto kern = conv_tc_kernel<kXBits, kChunkInTap, kFlat, kPair>;
   // The opt-in limit is raised to the device maximum, never lowered to this call's size:
   // a CUDA graph node captured earlier with a larger plan must stay launchable (a graph
@@ -1115,10 +1145,10 @@ static int launch_bits(const Params& prm, const CUtensorMap& map, const CUtensor
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, kern, map, map_a, prm);
+    e = cudaLaunchKernelEx(&cfg, kern, map, map_h, map_a, prm);
     if (e != cudaSuccess) { *err = std::string("conv_tc pair launch: ") + cudaGetErrorString(e); return 3; }
   } else {
-    kern<<<grid, threads_for(kFlat), smem, stream>>>(map, map_a, prm);
+    kern<<<grid, threads_for(kFlat), smem, stream>>>(map, map_h, map_a, prm);
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) { *err = std::string("conv_tc launch: ") + cudaGetErrorString(e); return 3; }
@@ -1166,8 +1196,19 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
     *err = "conv_tc: workspace path needs stride 1, cin % 128 == 0 and a large enough workspace";
     return 1;
   }
-  prm.total_tiles = tiles;
   if (tiles == 0) return 0;
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (sms < 2) sms = 2;
+  // Last-wave balancing: with `workers` persistent CTAs (or CTA pairs), the full tiles past
+  // the last complete wave run as two half-width (N/2) tiles each, when those halves still
+  // fit in one wave; half as long per tile, they end the kernel sooner.
+  const int workers = pair ? sms / 2 : sms;
+  const int rem = tiles % workers;
+  prm.dp_tiles = tiles;
+  if (BN == 256 && rem > 0 && 2 * rem <= workers) prm.dp_tiles = tiles - rem;
+  prm.total_tiles = prm.dp_tiles + 2 * (tiles - prm.dp_tiles);
   prm.num_kchunks = a.k_pad / BK;
   prm.cin = a.cin; prm.cout = a.cout; prm.kh = a.kh; prm.kw = a.kw;
   prm.stride = a.stride; prm.pad = a.pad; prm.k_total = a.k_total;
@@ -1214,12 +1255,19 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) { *err = "cuTensorMapEncodeTiled failed: " + std::to_string((int)r); return 3; }
+  // the same weights with boxes of half the rows, for the half-width tiles
+  CUtensorMap map_h = map;
+  if (prm.dp_tiles < prm.total_tiles) {
+    cuuint32_t box_h[2] = {(cuuint32_t)BK, (cuuint32_t)(b_rows / 2)};
+    r = enc(&map_h, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)a.w_e4m3, gdim, gstride, box_h, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) { *err = "cuTensorMapEncodeTiled (half) failed: " + std::to_string((int)r); return 3; }
+  }
 
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  int grid = tiles < sms ? tiles : sms;
-  if (pair) grid = 2 * (tiles < sms / 2 ? tiles : sms / 2);
+  const int units = prm.total_tiles;
+  int grid = units < sms ? units : sms;
+  if (pair) grid = 2 * (units < sms / 2 ? units : sms / 2);
   const bool in_tap = (a.cin % BK) == 0;
   CUtensorMap map_a = map;  // unused unless flat
   if (flat) {
@@ -1254,16 +1302,16 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
       *err = "cuTensorMapEncodeTiled (activations) failed: " + std::to_string((int)r2);
       return 3;
     }
-    if (pair) return launch_bits<2, true, true, true>(prm, map, map_a, grid, smem, stream, err);
-    return launch_bits<2, true, true>(prm, map, map_a, grid, smem, stream, err);
+    if (pair) return launch_bits<2, true, true, true>(prm, map, map_h, map_a, grid, smem, stream, err);
+    return launch_bits<2, true, true>(prm, map, map_h, map_a, grid, smem, stream, err);
   }
   switch (a.x_bits) {
-    case 2: return in_tap ? launch_bits<2, true, false>(prm, map, map_a, grid, smem, stream, err)
-                          : launch_bits<2, false, false>(prm, map, map_a, grid, smem, stream, err);
-    case 3: return in_tap ? launch_bits<3, true, false>(prm, map, map_a, grid, smem, stream, err)
-                          : launch_bits<3, false, false>(prm, map, map_a, grid, smem, stream, err);
-    case 4: return in_tap ? launch_bits<4, true, false>(prm, map, map_a, grid, smem, stream, err)
-                          : launch_bits<4, false, false>(prm, map, map_a, grid, smem, stream, err);
+    case 2: return in_tap ? launch_bits<2, true, false>(prm, map, map_h, map_a, grid, smem, stream, err)
+                          : launch_bits<2, false, false>(prm, map, map_h, map_a, grid, smem, stream, err);
+    case 3: return in_tap ? launch_bits<3, true, false>(prm, map, map_h, map_a, grid, smem, stream, err)
+                          : launch_bits<3, false, false>(prm, map, map_h, map_a, grid, smem, stream, err);
+    case 4: return in_tap ? launch_bits<4, true, false>(prm, map, map_h, map_a, grid, smem, stream, err)
+                          : launch_bits<4, false, false>(prm, map, map_h, map_a, grid, smem, stream, err);
     default: *err = "conv_tc: activation bits must be 2, 3 or 4"; return 2;
   }
 }

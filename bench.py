@@ -35,7 +35,8 @@ METRIC = "int-only conv TOPS & % of INT8 tensor peak; detector-head images/s at 
 # DRAM bytes (read + write) of one workspace-fed tower-layer conv_tc launch, taken from an
 # ncu capture of this kernel on this workload (dram__bytes_read.sum + dram__bytes_write.sum).
 # Re-measure (or set to None) whenever conv_tc_kernel changes.
-TOWER_CONV_DRAM_BYTES = 12_687_360
+TOWER_CONV_DRAM_BYTES = None
+KREP = 16  # tower-layer convs per timed kernel graph (16 x 12 MB workspaces > 129 MB L2)
 WORKLOAD = "retina_head_800x1333_b2_2bit"
 
 
@@ -270,13 +271,22 @@ def main():
     with torch.cuda.graph(graph, stream=stream):
         step()
     # the dominant kernel alone: the tensor-core conv of one grouped 256->256 tower layer over
-    # all levels, fed from a workspace expanded beforehand (outside the timed graph)
+    # all levels, fed from workspaces expanded beforehand (outside the timed graph). One graph
+    # replays KREP launches back to back, each reading its own workspace, so the launches'
+    # combined working set (KREP x 12 MB) exceeds L2 and one graph-launch overhead is spread
+    # over KREP kernels.
     kjobs = [(xs[l], bufs[0][l], None, l) for l in range(nl)]
     kgraph = torch.cuda.CUDAGraph()
+    krep = KREP if ws is not None else 1
     if ws is not None:
-        aqd.conv_expand_input(kjobs, tower_w[0], 1, 1, ws, stream=stream)
+        kws = [aqd.workspace_for(kjobs, tower_w[0], 1, 1, device=dev) for _ in range(krep)]
+        with torch.cuda.stream(stream):
+            for w_ in kws:
+                aqd.conv_expand_input(kjobs, tower_w[0], 1, 1, w_, stream=stream)
+        stream.synchronize()
         with torch.cuda.graph(kgraph, stream=stream):
-            aqd.conv_int_grouped_expanded(kjobs, tower_w[0], 1, 1, rq=tower_rq[0], workspace=ws, stream=stream)
+            for w_ in kws:
+                aqd.conv_int_grouped_expanded(kjobs, tower_w[0], 1, 1, rq=tower_rq[0], workspace=w_, stream=stream)
     else:
         with torch.cuda.graph(kgraph, stream=stream):
             aqd.conv_int_grouped(kjobs, tower_w[0], 1, 1, rq=tower_rq[0], stream=stream)
@@ -337,7 +347,7 @@ def main():
 
     peaks, src = measured_peaks()
     fp8_peak = 2.0 * peaks["bf16_tflops"]
-    kern_avg_ms = statistics.mean(kern_ms)
+    kern_avg_ms = statistics.mean(kern_ms) / krep
     achieved = ops[0] / (kern_avg_ms * 1e-3) / 1e12
     line = {
         "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": world, "steps": args.steps,
@@ -353,14 +363,15 @@ def main():
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": fp8_peak, "unit": "TFLOP/s",
                      "frac": achieved / fp8_peak, "traffic": TOWER_CONV_DRAM_BYTES if ws is not None else None,
                      "kernel": "conv_tc_kernel: one 3x3 256->256 tower layer, all 5 levels grouped" +
-                               (" (workspace expanded beforehand)" if ws is not None else ""),
+                               (f" (workspace expanded beforehand; {krep} launches per timed graph, each on "
+                                "its own workspace, working set > L2)" if ws is not None else ""),
                      "algorithmic_ops_per_launch": ops[0],
                      "peak_source": f"{src} bf16 dense burst x 2 (nominal e4m3/bf16 ratio)",
                      "avg_launch_ms": kern_avg_ms},
         "e2e": {"value": e2e_val, "unit": "TOPS", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_ms},
         "clocks": clk.summary(),
-        "gpu_launches": launches_per_step * args.steps + max(50, args.steps // 4),
+        "gpu_launches": launches_per_step * args.steps + krep * max(50, args.steps // 4),
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         ops_c, t_c = oracle_tower_sample(wl)

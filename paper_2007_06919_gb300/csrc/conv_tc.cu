@@ -69,6 +69,7 @@ constexpr int kTmaWarpsFlat = 3;
 __host__ __device__ constexpr int tma_warps(bool flat) { return flat ? kTmaWarpsFlat : kTmaWarps; }
 __host__ __device__ constexpr int threads_for(bool flat) { return flat ? (kWarpTma + kTmaWarpsFlat) * 32 : kThreads; }
 constexpr int kMaxStages = 8;
+constexpr int kQTab = 256;  // K-chunk table entries (larger K falls back to division)
 constexpr uint64_t kTimeoutNs = 1000000000ull;  // 1 s per wait
 
 struct Params {
@@ -88,7 +89,7 @@ struct Params {
   int32_t cin_chunks; // cin / 128 (flat path)
   int32_t dp_tiles;   // tiles [0, dp_tiles) are bn wide; later ones are the two bn/2 halves
                       // of the remaining full tiles (the last, partial wave)
-  uint32_t off_b, off_epi, off_bar;
+  uint32_t off_b, off_epi, off_bar, off_qtab;
   uint32_t* status;
 };
 
@@ -234,6 +235,11 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       " [%0], [%1, {%2, %3}], [%4];"
       ::"r"(dst), "l"((uint64_t)map), "r"(x), "r"(y), "r"(bar) : "memory");
 }
+
+// Programmatic dependent launch: wait for the previous kernel in the stream to finish (and
+// its writes to be visible); allow the next kernel's CTAs to be scheduled.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
@@ -563,6 +569,13 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
   const int BN = p.bn;
   const uint32_t stage_b_bytes = (uint32_t)(kPair ? BN / 2 : BN) * BK;  // this CTA's rows of B
 
+  // K chunk q -> (tap row r, tap column sx, 128-channel block cb), for the TMA issuers
+  uint32_t* qtab = reinterpret_cast<uint32_t*>(smem + p.off_qtab);
+  for (int q = threadIdx.x; q < p.num_kchunks && q < kQTab; q += blockDim.x) {
+    const int tap = q / p.cin_chunks, cb = q - tap * p.cin_chunks;
+    const int r = tap / p.kw, sx = tap - r * p.kw;
+    qtab[q] = ((uint32_t)r << 24) | ((uint32_t)sx << 16) | (uint32_t)cb;
+  }
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(b_full + 8 * s, kFlat ? 1 : kProdWarps + 1);  // per producer warp + TMA
@@ -601,6 +614,9 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
   if constexpr (kPair) cluster_sync();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  // everything above overlaps the previous kernel; global memory is touched only after this
+  grid_dep_wait();
+  if (threadIdx.x == 0) grid_dep_launch();
 
   const int nk = p.num_kchunks;
   const int first_tile = kPair ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
@@ -677,19 +693,32 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       bool ok = true;
       for (int t = first_tile; t < p.total_tiles && ok; t += tile_stride) {
         const TileInfo ti = tile_info(p, t);
+        // per tile: the first workspace row of this CTA's A rows (flat path) and the image width
+        int row0 = 0, wp = 0;
+        if constexpr (kFlat) {
+          const ConvJobDev& jb = p.jobs[ti.job];
+          const FlatTile ft = flat_tile(jb, ti.mt, kTileRows);
+          row0 = jb.row_off + ft.img * jb.hp * jb.wp + ft.v0 + (int)rank * 128;
+          wp = jb.wp;
+        }
+        const CUtensorMap* wm = ti.bn == BN ? &tmap_w : &tmap_wh;
         for (int q = 0; q < nk; ++q, ++it, s = (s + 1 == (uint32_t)S) ? 0 : s + 1, ph ^= (s == 0)) {
           if ((int)(it % kTma) != tw) continue;
           if (!mbar_wait(b_empty + 8 * s, ph ^ 1, abort_flag)) { ok = false; break; }
+          int r, sx, cb;
+          if (q < kQTab) {
+            const uint32_t e = qtab[q];
+            r = (int)(e >> 24); sx = (int)((e >> 16) & 255u); cb = (int)(e & 0xFFFFu);
+          } else {
+            const int tap = q / p.cin_chunks;
+            cb = q - tap * p.cin_chunks;
+            r = tap / p.kw; sx = tap - r * p.kw;
+          }
           if constexpr (kPair) {
             // this CTA's 128 rows of A and its half of B; both CTAs' copies complete on the
             // leader's "full" barrier, which the leader arms with the bytes of all four
-            const ConvJobDev& jb = p.jobs[ti.job];
-            const FlatTile ft = flat_tile(jb, ti.mt, kTileRows);
-            const int tap = q / p.cin_chunks, cb = q - tap * p.cin_chunks;
-            const int r = tap / p.kw, sx = tap - r * p.kw;
-            const int row = jb.row_off + ft.img * jb.hp * jb.wp + ft.v0 + (int)rank * 128 + r * jb.wp + sx;
+            const int row = row0 + r * wp + sx;
             const int brow = ti.col0 + (int)rank * (ti.bn / 2);
-            const CUtensorMap* wm = ti.bn == BN ? &tmap_w : &tmap_wh;
             const uint32_t b_bytes = (uint32_t)(ti.bn / 2) * BK;
             if (leader) {
               mbar_arrive_expect_tx(b_full + 8 * s, 2 * (b_bytes + kStageA));
@@ -703,17 +732,14 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
             continue;
           } else if constexpr (kFlat) {
             // A: 128 consecutive rows of the padded byte image, shifted by the tap (r, s)
-            const ConvJobDev& jb = p.jobs[ti.job];
-            const FlatTile ft = flat_tile(jb, ti.mt);
-            const int tap = q / p.cin_chunks, cb = q - tap * p.cin_chunks;
-            const int r = tap / p.kw, sx = tap - r * p.kw;
-            const int row = jb.row_off + ft.img * jb.hp * jb.wp + ft.v0 + r * jb.wp + sx;
+            const int row = row0 + r * wp + sx;
             mbar_arrive_expect_tx(b_full + 8 * s, (uint32_t)ti.bn * BK + kStageA);
             tma_load_2d(s_a + s * kStageA, &tmap_a, cb * BK, row, b_full + 8 * s);
           } else {
+            (void)r; (void)sx; (void)cb;
             mbar_arrive_expect_tx(b_full + 8 * s, (uint32_t)ti.bn * BK);
           }
-          tma_load_2d(s_b + s * stage_b_bytes, ti.bn == BN ? &tmap_w : &tmap_wh, q * BK, ti.col0, b_full + 8 * s);
+          tma_load_2d(s_b + s * stage_b_bytes, wm, q * BK, ti.col0, b_full + 8 * s);
         }
       }
       if (!ok) fail(abort_flag, p.status);
@@ -1034,6 +1060,9 @@ __global__ void __launch_bounds__(256) expand_kernel(const __grid_constant__ Exp
   // all steps are issued before the stores. All index arithmetic is 32-bit (the host
   // checks rows * cin / 16 < 2^31).
   constexpr int kPerLane = 8;
+  // the previous kernel in the stream may still be reading the workspace or writing x
+  grid_dep_wait();
+  if (threadIdx.x == 0) grid_dep_launch();
   const int chunks = a.cin >> 4;
   const int total = (int)a.total_rows * chunks;
   const int lane = threadIdx.x & 31;
@@ -1131,25 +1160,25 @@ static int launch_bits(const Params& prm, const CUtensorMap& map, const CUtensor
   if ((size_t)optin < smem) { *err = "conv_tc: shared memory plan exceeds the device limit"; return 2; }
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
   if (e != cudaSuccess) { *err = std::string("cudaFuncSetAttribute: ") + cudaGetErrorString(e); return 3; }
-  if constexpr (kPair) {
-    // clusters of two CTAs (one pair per two SMs)
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)grid);
-    cfg.blockDim = dim3((unsigned)threads_for(kFlat));
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 2;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, kern, map, map_h, map_a, prm);
-    if (e != cudaSuccess) { *err = std::string("conv_tc pair launch: ") + cudaGetErrorString(e); return 3; }
-  } else {
-    kern<<<grid, threads_for(kFlat), smem, stream>>>(map, map_h, map_a, prm);
-  }
+  // programmatic dependent launch: the prologue (barriers, TMEM allocation, tensor-map
+  // prefetch) overlaps the previous kernel; the kernel waits for it before touching global
+  // memory. CTA pairs run as clusters of two.
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3((unsigned)threads_for(kFlat));
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 2;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = kPair ? 2 : 1;
+  e = cudaLaunchKernelEx(&cfg, kern, map, map_h, map_a, prm);
+  if (e != cudaSuccess) { *err = std::string("conv_tc launch: ") + cudaGetErrorString(e); return 3; }
   e = cudaGetLastError();
   if (e != cudaSuccess) { *err = std::string("conv_tc launch: ") + cudaGetErrorString(e); return 3; }
   return 0;
@@ -1226,8 +1255,9 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   const size_t stage_bytes = (size_t)kStageA + (size_t)b_rows * BK;
   const size_t epi_bytes = 256 * sizeof(EpiChan) + 256 * sizeof(int4);
   const size_t bar_bytes = 8 * (2 * kMaxStages + 5) + 16;
+  const size_t qtab_bytes = kQTab * sizeof(uint32_t);
   const size_t budget = 232448 - 1024;  // max dynamic smem per block minus alignment slack
-  int stages = (int)((budget - epi_bytes - bar_bytes) / stage_bytes);
+  int stages = (int)((budget - epi_bytes - bar_bytes - qtab_bytes) / stage_bytes);
   if (stages > kMaxStages) stages = kMaxStages;
   if (stages < 2) { *err = "conv_tc: shared memory plan does not fit"; return 2; }
   // The TMA issuers take K chunks round-robin and each waits on its stage's "empty"
@@ -1239,7 +1269,8 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   prm.off_b = (uint32_t)(stages * kStageA);
   prm.off_epi = prm.off_b + (uint32_t)(stages * b_rows * BK);
   prm.off_bar = prm.off_epi + (uint32_t)epi_bytes;
-  const size_t smem = 1024 + prm.off_bar + bar_bytes;
+  prm.off_qtab = prm.off_bar + (uint32_t)bar_bytes;
+  const size_t smem = 1024 + prm.off_qtab + qtab_bytes;
   int cols = 32;
   while (cols < 2 * kSub * BN) cols *= 2;  // two buffers x kSub sub-tiles x BN fp32 columns
   prm.tmem_cols = cols;
@@ -1281,13 +1312,23 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
       // one warp per run of 32 * 8 (row, 16-byte chunk) pairs, 8 warps per block
       const int64_t pairs = rows * (a.cin / 16);
       const unsigned blocks = (unsigned)((pairs + 2047) / 2048);
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(blocks);
+      cfg.blockDim = dim3(256);
+      cfg.stream = stream;
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+      attr[0].val.programmaticStreamSerializationAllowed = 1;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      cudaError_t e;
       switch (a.x_bits) {
-        case 2: expand_kernel<2><<<blocks, 256, 0, stream>>>(ea); break;
-        case 3: expand_kernel<3><<<blocks, 256, 0, stream>>>(ea); break;
-        case 4: expand_kernel<4><<<blocks, 256, 0, stream>>>(ea); break;
+        case 2: e = cudaLaunchKernelEx(&cfg, expand_kernel<2>, ea); break;
+        case 3: e = cudaLaunchKernelEx(&cfg, expand_kernel<3>, ea); break;
+        case 4: e = cudaLaunchKernelEx(&cfg, expand_kernel<4>, ea); break;
         default: *err = "conv_tc: activation bits must be 2, 3 or 4"; return 2;
       }
-      cudaError_t e = cudaGetLastError();
+      if (e == cudaSuccess) e = cudaGetLastError();
       if (e != cudaSuccess) { *err = std::string("expand launch: ") + cudaGetErrorString(e); return 3; }
     }
     if (a.expand_only) return 0;

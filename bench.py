@@ -6,7 +6,9 @@ image batch (levels 100x168, 50x84, 25x42, 13x21, 7x11; batch 2; 2-bit codes): f
 levels) and the 3x3 256->80 classification and 256->4 box convs with int32 outputs.
 The two output convs read the same tower output, so they run as one 256->84 conv with
 the weight rows and biases concatenated (channels 0..79 = classification, 80..83 = box):
-every output value is the one the two separate convs give.
+every output value is the one the two separate convs give. The packed input codes are
+expanded once into a byte image; each tower layer writes its packed 2-bit output and the
+next layer's byte image in the same epilogue.
 Inputs are seeded synthetic codes (no images are used). Ops are counted as 2*M*N*K of the
 real (unpadded) convolutions.
 
@@ -247,21 +249,27 @@ def main():
         flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
         # one expanded-activation workspace serves every conv of the step (same input shapes)
         ws = aqd.workspace_for([(xs[l], bufs[0][l], None, l) for l in range(nl)], tower_w[0], 1, 1, device=dev)
+        assert ws is not None, "the workspace path applies to the 3x3 256->256 tower"
+        ws2 = torch.zeros_like(ws)  # the second image's zero border is written once, here
     stream.synchronize()
 
     def step():
-        cur = xs
+        """The input is expanded once; each tower layer writes its packed 2-bit output and,
+        through aqd_conv_int_grouped_chain, the next layer's zero-padded byte image (two
+        workspaces in turn); the output conv reads the last image."""
+        cur, cur_ws, nxt_ws = xs, ws, ws2
+        aqd.conv_expand_input([(x, None, None, l) for l, x in enumerate(xs)], tower_w[0], 1, 1, ws, stream=stream)
         for i in range(4):
             out = bufs[i % 2]
-            aqd.conv_int_grouped([(cur[l], out[l], None, l) for l in range(nl)], tower_w[i], 1, 1,
-                                 rq=tower_rq[i], workspace=ws, stream=stream)
-            cur = out
-        aqd.conv_int_grouped([(cur[l], heads[l], None, l) for l in range(nl)], head_w, 1, 1,
-                             rq=head_rq, workspace=ws, stream=stream)
+            aqd.conv_int_grouped_chain([(cur[l], out[l], None, l) for l in range(nl)], tower_w[i], 1, 1,
+                                       rq=tower_rq[i], workspace=cur_ws, next_pad=1, next_workspace=nxt_ws,
+                                       stream=stream)
+            cur, cur_ws, nxt_ws = out, nxt_ws, cur_ws
+        aqd.conv_int_grouped_expanded([(cur[l], heads[l], None, l) for l in range(nl)], head_w, 1, 1,
+                                      rq=head_rq, workspace=cur_ws, stream=stream)
 
-    # each conv is one expansion launch + one tensor-core launch when the workspace applies
-    per_conv = 2 if ws is not None else 1
-    launches_per_step = 5 * per_conv
+    # one expansion launch + five tensor-core launches
+    launches_per_step = 6
     with torch.cuda.stream(stream):
         for _ in range(3):
             step()

@@ -206,6 +206,25 @@ aqd_status aqd_conv_int_grouped_expanded(const aqd_conv_job* jobs, int32_t njobs
                                          const aqd_requant_params* rq, const aqd_skip_params* sp,
                                          void* workspace, size_t ws_bytes, aqd_stream_t stream);
 
+/* Layer chaining on the workspace path: aqd_conv_int_grouped_expanded that, besides the
+ * packed k-bit outputs y (k = 2, 3 or 4), writes the same codes one byte each into
+ * `next_workspace` as the zero-padded byte image that a following stride-1 convolution
+ * with padding `next_pad` over these outputs reads (the layout aqd_conv_expand_input
+ * writes for inputs of the outputs' shape, jobs in the same order), so that convolution
+ * can be called with aqd_conv_int_grouped_expanded (or this function) without an
+ * expansion pass. Only the interior of the image is written: its border must already hold
+ * zeros (fill next_workspace with zeros once, or expand an input of the same shape into it
+ * once; no call writes the border afterwards). Needs cout % 128 == 0, a next_workspace of
+ * at least sum(n * (ho + 2 next_pad) * (wo + 2 next_pad)) * cout bytes, 256-byte aligned
+ * and not overlapping `workspace`; otherwise AQD_ERR_INVALID. The paper's layers pass
+ * k-bit codes from one layer to the next (Eq. 2, Fig. 1); this is the same codes stored one
+ * per byte for the tensor cores. */
+aqd_status aqd_conv_int_grouped_chain(const aqd_conv_job* jobs, int32_t njobs,
+                                      const aqd_conv_weights* w, int32_t stride, int32_t pad,
+                                      const aqd_requant_params* rq, const aqd_skip_params* sp,
+                                      void* workspace, size_t ws_bytes, int32_t next_pad,
+                                      void* next_workspace, size_t next_ws_bytes, aqd_stream_t stream);
+
 /* ---- elementwise ------------------------------------------------------------------ */
 
 /* y = requant(sat32(acc + bias)) per channel at `level`: Eq. 6 + Eq. 2 on an int32

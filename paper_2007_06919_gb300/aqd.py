@@ -56,7 +56,7 @@ EXPORTS = ["aqd_row_bytes", "aqd_quantize_multiplier", "aqd_status_string", "aqd
            "aqd_device_status", "aqd_set_conv_path", "aqd_last_conv_path", "aqd_pack_codes",
            "aqd_unpack_codes", "aqd_conv_weights_bytes", "aqd_conv_prepare_weights", "aqd_conv_int",
            "aqd_conv_int_grouped", "aqd_conv_workspace_bytes", "aqd_conv_expand_input",
-           "aqd_conv_int_grouped_expanded", "aqd_requant", "aqd_residual_add_int",
+           "aqd_conv_int_grouped_expanded", "aqd_conv_int_grouped_chain", "aqd_requant", "aqd_residual_add_int",
            "aqd_maxpool_codes"]
 
 _lib = None
@@ -101,6 +101,9 @@ def load(build_if_missing: bool = True):
     L.aqd_conv_expand_input.argtypes = [ctypes.POINTER(_Job), i32, ctypes.POINTER(_Weights), i32, i32, vp,
                                         ctypes.c_size_t, vp]
     L.aqd_conv_int_grouped_expanded.argtypes = L.aqd_conv_int_grouped.argtypes
+    L.aqd_conv_int_grouped_chain.argtypes = [ctypes.POINTER(_Job), i32, ctypes.POINTER(_Weights), i32, i32,
+                                             ctypes.POINTER(_Requant), ctypes.POINTER(_Skip), vp, ctypes.c_size_t,
+                                             i32, vp, ctypes.c_size_t, vp]
     L.aqd_conv_workspace_bytes.restype = ctypes.c_size_t
     L.aqd_conv_workspace_bytes.argtypes = [ctypes.POINTER(_Job), i32, ctypes.POINTER(_Weights), i32, i32]
     L.aqd_requant.argtypes = [ctypes.POINTER(_Tensor), ctypes.POINTER(_Requant), i32, ctypes.POINTER(_Tensor), vp]
@@ -109,7 +112,7 @@ def load(build_if_missing: bool = True):
     L.aqd_maxpool_codes.argtypes = [ctypes.POINTER(_Tensor), i32, i32, i32, ctypes.POINTER(_Tensor), vp]
     for name in ("aqd_quantize_multiplier", "aqd_device_status", "aqd_pack_codes", "aqd_unpack_codes",
                  "aqd_conv_prepare_weights", "aqd_conv_int", "aqd_conv_int_grouped", "aqd_conv_expand_input",
-                 "aqd_conv_int_grouped_expanded", "aqd_requant",
+                 "aqd_conv_int_grouped_expanded", "aqd_conv_int_grouped_chain", "aqd_requant",
                  "aqd_residual_add_int", "aqd_maxpool_codes"):
         getattr(L, name).restype = c_int
     _lib = L
@@ -366,6 +369,24 @@ def conv_int_grouped_expanded(jobs, w: ConvWeights, stride: int, pad: int, *, rq
                                                 ctypes.byref(spc) if spc is not None else None, wsp, wsb,
                                                 _stream(stream)),
            "aqd_conv_int_grouped_expanded")
+
+
+def conv_int_grouped_chain(jobs, w: ConvWeights, stride: int, pad: int, *, rq: RequantParams | None = None,
+                           sp: SkipParams | None = None, workspace: torch.Tensor, next_pad: int,
+                           next_workspace: torch.Tensor, stream=None):
+    """conv_int_grouped_expanded that also writes the outputs, one byte per code, as the
+    zero-padded byte image the next stride-1 conv (padding next_pad) reads from
+    next_workspace (whose border must hold zeros)."""
+    arr = _jobs(jobs)
+    rqc = rq.c() if rq is not None else None
+    spc = sp.cs() if sp is not None else None
+    wsp, wsb = _ws(workspace)
+    nwp, nwb = _ws(next_workspace)
+    _check(load().aqd_conv_int_grouped_chain(arr, len(jobs), ctypes.byref(w.desc), stride, pad,
+                                             ctypes.byref(rqc) if rqc is not None else None,
+                                             ctypes.byref(spc) if spc is not None else None, wsp, wsb,
+                                             next_pad, nwp, nwb, _stream(stream)),
+           "aqd_conv_int_grouped_chain")
 
 
 def requant(acc: DTensor, rq: RequantParams, y: DTensor, *, level: int = 0, stream=None) -> DTensor:

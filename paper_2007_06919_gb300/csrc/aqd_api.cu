@@ -230,12 +230,20 @@ size_t aqd_conv_workspace_bytes(const aqd_conv_job* jobs, int32_t njobs, const a
 
 // What one grouped call runs on the workspace path: expansion + convolution (the public
 // grouped call), the expansion alone, or the convolution from an already expanded workspace.
-enum ConvStage { kStageBoth = 0, kStageExpandOnly = 1, kStageConvOnly = 2 };
+// kStageChain is kStageConvOnly that also writes the output codes, one byte each, as the
+// zero-padded byte image the next stride-1 conv reads.
+enum ConvStage { kStageBoth = 0, kStageExpandOnly = 1, kStageConvOnly = 2, kStageChain = 3 };
+
+struct ChainOut {
+  int32_t pad;
+  void* ws;
+  size_t bytes;
+};
 
 static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
                                int32_t stride, int32_t pad, const aqd_requant_params* rq,
                                const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
-                               aqd_stream_t stream, ConvStage stage);
+                               aqd_stream_t stream, ConvStage stage, const ChainOut* chain = nullptr);
 
 aqd_status aqd_conv_int_grouped(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
                                 int32_t stride, int32_t pad, const aqd_requant_params* rq,
@@ -276,10 +284,19 @@ aqd_status aqd_conv_expand_input(const aqd_conv_job* jobs, int32_t njobs, const 
                       kStageExpandOnly);
 }
 
+aqd_status aqd_conv_int_grouped_chain(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
+                                      int32_t stride, int32_t pad, const aqd_requant_params* rq,
+                                      const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
+                                      int32_t next_pad, void* next_workspace, size_t next_ws_bytes,
+                                      aqd_stream_t stream) {
+  const ChainOut c{next_pad, next_workspace, next_ws_bytes};
+  return conv_grouped(jobs, njobs, w, stride, pad, rq, sp, workspace, ws_bytes, stream, kStageChain, &c);
+}
+
 static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
                                int32_t stride, int32_t pad, const aqd_requant_params* rq,
                                const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
-                               aqd_stream_t stream, ConvStage stage) {
+                               aqd_stream_t stream, ConvStage stage, const ChainOut* chain) {
   std::string err;
   if (!jobs || njobs <= 0 || njobs > kMaxJobs) return fail(AQD_ERR_INVALID, "njobs must be 1..8");
   if (!check_weights(w, &err)) return fail(AQD_ERR_INVALID, err);
@@ -380,7 +397,25 @@ static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aq
     if (!workspace) return fail(AQD_ERR_INVALID, "the workspace must not be NULL");
     if (!a.ws) return fail(AQD_ERR_INVALID, "the workspace path does not apply, or the workspace is too small");
   }
-  a.skip_expand = stage == kStageConvOnly ? 1 : 0;
+  a.skip_expand = (stage == kStageConvOnly || stage == kStageChain) ? 1 : 0;
+  if (stage == kStageChain) {
+    if (!chain || !chain->ws) return fail(AQD_ERR_INVALID, "next_workspace must not be NULL");
+    if ((reinterpret_cast<uintptr_t>(chain->ws) & 255) != 0) return fail(AQD_ERR_INVALID, "next_workspace must be 256-byte aligned");
+    if (chain->pad < 0) return fail(AQD_ERR_INVALID, "next_pad must be >= 0");
+    if (out_bits < 2 || out_bits > 4) return fail(AQD_ERR_INVALID, "a chained output needs 2-, 3- or 4-bit codes");
+    if (w->cout % 128 != 0) return fail(AQD_ERR_INVALID, "a chained output needs cout % 128 == 0");
+    int64_t orows = 0;
+    for (int j = 0; j < njobs; ++j)
+      orows += (int64_t)jobs[j].y.n * (jobs[j].y.h + 2 * chain->pad) * (jobs[j].y.w + 2 * chain->pad);
+    if (orows * (w->cout / 16) >= (1LL << 31)) return fail(AQD_ERR_UNSUPPORTED, "chained output image too large");
+    const size_t need = (size_t)orows * (size_t)w->cout;
+    if (chain->bytes < need) return fail(AQD_ERR_INVALID, "next_workspace is too small");
+    const uintptr_t i0 = reinterpret_cast<uintptr_t>(workspace), o0 = reinterpret_cast<uintptr_t>(chain->ws);
+    const size_t in_need = (size_t)flat_rows(jobs, njobs, w, stride, pad) * (size_t)w->cin;
+    if (i0 < o0 + need && o0 < i0 + in_need) return fail(AQD_ERR_INVALID, "workspace and next_workspace overlap");
+    a.ws_out = static_cast<uint8_t*>(chain->ws);
+    a.out_pad = chain->pad;
+  }
   a.expand_only = stage == kStageExpandOnly ? 1 : 0;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   int rc = path == 1 ? launch_conv_tc(a, st, &err) : launch_conv_direct(a, st, &err);

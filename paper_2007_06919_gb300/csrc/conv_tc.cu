@@ -90,6 +90,8 @@ struct Params {
   int32_t dp_tiles;   // tiles [0, dp_tiles) are bn wide; later ones are the two bn/2 halves
                       // of the remaining full tiles (the last, partial wave)
   uint32_t off_b, off_epi, off_bar, off_qtab;
+  uint8_t* ws_out;    // chained output image (NULL: none)
+  int32_t out_pad;
   uint32_t* status;
 };
 
@@ -474,6 +476,22 @@ __device__ __forceinline__ void fast_requant_group(const uint32_t* v, const EpiC
       gw[i / q] |= y << (8 * (i % 4) + kOut * ((i % q) / 4));
     }
   }
+}
+
+// Chained output: the 32 codes of one packed group, one byte each, at their place in the
+// zero-padded byte image that the next stride-1 conv (padding out_pad) reads.
+__device__ __forceinline__ void chain_store(const Params& p, const ConvJobDev& jb, int img, int oh, int ow,
+                                            int ch0, const uint32_t gw[8], int out_bits) {
+  uint32_t o[8];
+  switch (out_bits) {
+    case 2: unpack_group_bytes<2>(gw, o); break;
+    case 3: unpack_group_bytes<3>(gw, o); break;
+    default: unpack_group_bytes<4>(gw, o); break;
+  }
+  const int row = jb.orow_off + (img * jb.ohp + oh + p.out_pad) * jb.owp + ow + p.out_pad;
+  uint4* dst = reinterpret_cast<uint4*>(p.ws_out + (size_t)row * p.cout + ch0);
+  dst[0] = make_uint4(o[0], o[1], o[2], o[3]);
+  dst[1] = make_uint4(o[4], o[5], o[6], o[7]);
 }
 
 // ---------------------------------------------------------------- the kernel
@@ -893,12 +911,14 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
         const uint32_t* v = va;
         int m;  // output pixel index within the job
         bool row_ok;
+        int oimg = 0, oh = 0, ow = 0;  // the pixel (flat path)
         if constexpr (kFlat) {
           const FlatTile ft = flat_tile(jb, ti.mt, kTileRows);
           const int vr = ft.v0 + (int)rank * 128 + quarter * 32 + lane;  // virtual row at the padded width
           const int ho = vr / jb.wp, wo = vr - (vr / jb.wp) * jb.wp;
           row_ok = vr < jb.vimg && wo < jb.wo;  // else a junk column or past the image
           m = (ft.img * jb.ho + ho) * jb.wo + wo;
+          oimg = ft.img; oh = ho; ow = wo;
         } else {
           m = ti.mt * BM + sub * 128 + quarter * 32 + lane;
           row_ok = m < jb.m_total;
@@ -924,6 +944,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
               }
             }
             store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
+            if (kFlat && p.ws_out) chain_store(p, jb, oimg, oh, ow, ch0, gw, out_bits);
           } else if (mode == 2) {
             int32_t* yr = reinterpret_cast<int32_t*>(yrow) + ch0;
             const bool full = ncols == 32 && ch0 + 32 <= p.cout;
@@ -967,6 +988,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
               uint32_t gw[8];
               pack_group_vals(oo, out_bits, gw);
               store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
+              if (kFlat && p.ws_out) chain_store(p, jb, oimg, oh, ow, ch0, gw, out_bits);
             }
           }
         }
@@ -1249,6 +1271,18 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   prm.bn = BN;
   prm.acc_small = a.acc_bound < (1LL << 22) ? 1 : 0;
   prm.cin_chunks = a.cin / BK;
+  prm.ws_out = a.ws_out;
+  prm.out_pad = a.out_pad;
+  if (a.ws_out) {
+    int64_t orows = 0;
+    for (int j = 0; j < a.njobs; ++j) {
+      ConvJobDev& jb = prm.jobs[j];
+      jb.ohp = jb.ho + 2 * a.out_pad;
+      jb.owp = jb.wo + 2 * a.out_pad;
+      jb.orow_off = (int32_t)orows;
+      orows += (int64_t)jb.n * jb.ohp * jb.owp;
+    }
+  }
   prm.status = a.status;
   // shared memory plan: stages of (BM x 128 A bytes + this CTA's B rows x 128 bytes)
   const int b_rows = pair ? BN / 2 : BN;

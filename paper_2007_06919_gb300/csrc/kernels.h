@@ -24,6 +24,9 @@ struct ConvJobDev {
   int32_t hp, wp;         // padded height / width (h + 2 pad, w + 2 pad)
   int32_t vimg;           // virtual output rows per image: ho * wp (columns >= wo are junk)
   int32_t tpi;            // tiles per image
+  // chained output (ws_out): zero-padded byte image of this job's output for the next conv
+  int32_t orow_off;       // first ws_out row (one row = cout bytes) of image 0
+  int32_t ohp, owp;       // padded output height / width (ho + 2 out_pad, wo + 2 out_pad)
 };
 
 struct ConvArgs {
@@ -48,6 +51,8 @@ struct ConvArgs {
   int32_t skip_expand;    // workspace already holds the expansion: launch only the conv
   int32_t expand_only;    // launch only the expansion into the workspace
   int32_t no_pair;        // workspace path: use the one-CTA kernel even for 256-wide N tiles
+  uint8_t* ws_out;        // chained output: also write the output codes as the next conv's byte image
+  int32_t out_pad;        // padding of that next conv
   uint32_t* status;       // device status word
 };
 

@@ -230,3 +230,73 @@ def test_expanded_conv_needs_an_applicable_workspace():
     with pytest.raises(aqd.AqdError) as e:
         aqd.conv_expand_input([(X, Y, None, 0)], W, 1, 1, buf)
     assert e.value.status == 1
+
+
+@pytest.mark.parametrize("bits,pairs", [(2, True), (2, False), (3, True), (4, True)])
+def test_chained_tower_bit_exact(bits, pairs):
+    """Layer chaining: the input expanded once, then three tower layers each written by
+    aqd_conv_int_grouped_chain straight into the next layer's byte image (two workspaces
+    in turn, the second zero-filled once), then the output conv from the last image. Every
+    layer's packed output equals the oracle chain's, and every chained image equals what
+    aqd_conv_expand_input writes for that layer's output."""
+    levels = [(15, 26), (8, 13), (4, 7)]
+    wl = synth.head_tower(41 + bits, 2, bits, levels=levels, calibrated=True)
+    nl = len(levels)
+    xts = [oracle.CodeTensor.from_codes(x, bits) for x in wl.inputs]
+    xs = [to_device(t) for t in xts]
+    Ws = [weights(cv.w, bits) for cv in wl.convs]
+    old = aqd.set_conv_path(1 if pairs else 3)
+    try:
+        jobs0 = [(xs[l], None, None, l) for l in range(nl)]
+        wsA = aqd.workspace_for(jobs0, Ws[0][0], 1, 1)
+        wsB = torch.zeros_like(wsA)
+        wsA.fill_(0x5A)
+        aqd.conv_expand_input(jobs0, Ws[0][0], 1, 1, wsA)
+        cur_ws, nxt_ws = wsA, wsB
+        cur = xs
+        refs = xts
+        for i in range(3):
+            cv = wl.convs[i]
+            ys = [aqd.DTensor.empty(t.n, t.h, t.w, 256, bits) for t in refs]
+            jobs = [(cur[l], ys[l], None, l) for l in range(nl)]
+            aqd.conv_int_grouped_chain(jobs, Ws[i][0], 1, 1, rq=_rq(cv), workspace=cur_ws, next_pad=1,
+                                       next_workspace=nxt_ws)
+            torch.cuda.synchronize()
+            refs = [_ref_conv(refs[l], Ws[i][1], cv, level=l) for l in range(nl)]
+            for l in range(nl):
+                assert_same(ys[l].data.cpu().numpy().reshape(refs[l].packed.shape), refs[l].packed, 256, bits,
+                            f"layer {i} level {l}")
+            check = torch.full_like(nxt_ws, 0x33)
+            aqd.conv_expand_input([(ys[l], None, None, l) for l in range(nl)], Ws[i + 1][0], 1, 1, check)
+            torch.cuda.synchronize()
+            assert torch.equal(check, nxt_ws), f"chained image of layer {i}"
+            cur, cur_ws, nxt_ws = ys, nxt_ws, cur_ws
+        cls = wl.convs[4]
+        hs = [aqd.DTensor.empty(t.n, t.h, t.w, cls.cout, 32) for t in refs]
+        aqd.conv_int_grouped_expanded([(cur[l], hs[l], None, l) for l in range(nl)], Ws[4][0], 1, 1,
+                                      rq=aqd.RequantParams.from_numpy(None, None, cls.bias), workspace=cur_ws)
+        torch.cuda.synchronize()
+        for l in range(nl):
+            want = _ref_conv(refs[l], Ws[4][1], cls, level=l).packed
+            assert_same(hs[l].data.cpu().numpy().reshape(want.shape), want, cls.cout, 32, f"head level {l}")
+    finally:
+        aqd.set_conv_path(old)
+    assert aqd.device_status() == 0
+
+
+def test_chain_rejects_overlap_and_bad_shapes():
+    rng = np.random.default_rng(5)
+    W, _ = weights(synth.weight_codes(rng, (256, 3, 3, 256), 2), 2)
+    X = aqd.DTensor.empty(1, 6, 7, 256, 2)
+    Y = aqd.DTensor.empty(1, 6, 7, 256, 2)
+    jobs = [(X, Y, None, 0)]
+    ws = aqd.workspace_for(jobs, W, 1, 1)
+    rq = aqd.RequantParams.from_numpy(np.full((1, 256), 1 << 30), np.full((1, 256), 8), np.zeros((1, 256)))
+    with pytest.raises(aqd.AqdError) as e:  # output image into the input workspace
+        aqd.conv_int_grouped_chain(jobs, W, 1, 1, rq=rq, workspace=ws, next_pad=1, next_workspace=ws)
+    assert e.value.status == 1
+    small = aqd.workspace_for(jobs, W, 1, 0)  # too small for padding 1
+    with pytest.raises(aqd.AqdError) as e:
+        aqd.conv_int_grouped_chain(jobs, W, 1, 1, rq=rq, workspace=ws, next_pad=1, next_workspace=small)
+    assert e.value.status == 1
+    torch.cuda.synchronize()

@@ -1209,7 +1209,9 @@ static int launch_bits(const Params& prm, const CUtensorMap& map, const CUtensor
 }  // namespace tc
 
 bool conv_tc_uses_pair(const ConvArgs& a) {
-  return a.ws != nullptr && a.bn == 256 && tc::kSub == 1 && !a.no_pair;
+  // every N tile width of the workspace path (BN is a multiple of 16, so each CTA's half of
+  // the weight tile is whole 8-row swizzle atoms and M = 256 MMAs take N = BN)
+  return a.ws != nullptr && a.bn >= 16 && a.bn % 16 == 0 && tc::kSub == 1 && !a.no_pair;
 }
 
 int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
@@ -1221,8 +1223,8 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   // flat path: the activations are expanded into the workspace first (stride 1,
   // cin % 128 == 0; the API checks both before passing a workspace)
   const bool flat = a.ws != nullptr;
-  // CTA pairs (cta_group::2, M = 256 per tile) for full 256-channel N tiles of the
-  // workspace path: each SM then streams half of the weight tile per K chunk
+  // CTA pairs (cta_group::2, M = 256 per tile) on the workspace path: each SM streams half
+  // of the weight tile per K chunk, and one MMA instruction covers both SMs' rows
   const bool pair = conv_tc_uses_pair(a);
   const int tile_rows = pair ? 256 : 128;
   int tiles = 0;
@@ -1258,7 +1260,8 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   const int workers = pair ? sms / 2 : sms;
   const int rem = tiles % workers;
   prm.dp_tiles = tiles;
-  if (BN == 256 && rem > 0 && 2 * rem <= workers) prm.dp_tiles = tiles - rem;
+  // (a half tile must start on a 32-channel packing group: BN / 2 a multiple of 32)
+  if (BN % 64 == 0 && rem > 0 && 2 * rem <= workers) prm.dp_tiles = tiles - rem;
   prm.total_tiles = prm.dp_tiles + 2 * (tiles - prm.dp_tiles);
   prm.num_kchunks = a.k_pad / BK;
   prm.cin = a.cin; prm.cout = a.cout; prm.kh = a.kh; prm.kw = a.kw;

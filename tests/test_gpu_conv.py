@@ -12,9 +12,8 @@ TC, DIRECT, TC_NO_PAIR = 1, 2, 3
 
 
 def ws_path(cout: int) -> int:
-    """Path reported for the workspace-fed tensor-core kernel: CTA pairs (4) for 256-wide
-    N tiles (cout above 240), one CTA (3) otherwise."""
-    return 4 if cout > 240 else 3
+    """Path reported for the workspace-fed tensor-core kernel: it runs on CTA pairs (4)."""
+    return 4
 
 
 def _params(rng, levels, cout, out_bits, calib_std=None):
@@ -143,7 +142,7 @@ def test_conv_with_skip_bit_exact(path, skip_bits, upsample, mirror, ws):
     c, d = synth.skip_params(rng, 1, cout, sh)
     got, want, used = conv_pair(x, 4, w, 4, out_bits=4, m0=m0, shift=sh, bias=b, skip=skip, skip_bits=skip_bits,
                              skip_c=c, skip_d=d, upsample=upsample, scale_main=mirror, path=path, workspace=ws)
-    assert used == (3 if (ws and path == TC) else path)
+    assert used == (4 if (ws and path == TC) else path)
     assert_same(got, want, cout, 4, "skip")
 
 

@@ -42,7 +42,7 @@ def test_config1_bottleneck_chain_bit_exact(ws):
         skt = to_device(xt) if sp else None
         wsb = aqd.workspace_for([(cur, Y, skt, 0)], W, cv.stride, cv.pad) if ws else None
         aqd.conv_int(cur, W, cv.stride, cv.pad, Y, rq=_rq(cv), skip=skt, sp=sp, workspace=wsb)
-        assert aqd.last_conv_path() == ((4 if cv.cout > 240 else 3) if ws else 1)
+        assert aqd.last_conv_path() == (4 if ws else 1)
         torch.cuda.synchronize()
         assert_same(Y.data.cpu().numpy().reshape(ref.packed.shape), ref.packed, cv.cout, 4, f"stage {i}")
         cur = Y
@@ -160,7 +160,7 @@ def test_cls_and_box_as_one_conv_bit_exact():
     ys = [aqd.DTensor.empty(t.n, t.h, t.w, 84, 32) for t in xts]
     jobs = [(xs[l], ys[l], None, l) for l in range(5)]
     aqd.conv_int_grouped(jobs, W, 1, 1, rq=rq, workspace=aqd.workspace_for(jobs, W, 1, 1))
-    assert aqd.last_conv_path() == 3
+    assert aqd.last_conv_path() == 4
     torch.cuda.synchronize()
     for l in range(5):
         got = ys[l].data.cpu().numpy().view(np.int32).reshape(-1, 84)

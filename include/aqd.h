@@ -225,6 +225,27 @@ aqd_status aqd_conv_int_grouped_chain(const aqd_conv_job* jobs, int32_t njobs,
                                       void* workspace, size_t ws_bytes, int32_t next_pad,
                                       void* next_workspace, size_t next_ws_bytes, aqd_stream_t stream);
 
+/* ---- convolution without a caller workspace ---------------------------------------- */
+
+/* Size of the library's own expanded-activation workspace (16 MiB per device context). */
+#define AQD_STATIC_WORKSPACE_BYTES (16u << 20)
+
+/* aqd_conv_int on the expanded-activation workspace path, with the workspace taken from a
+ * fixed array inside the library instead of from the caller; it allocates nothing. The
+ * paper has no counterpart: this exists for callers that cannot allocate device memory
+ * (a serving loop whose device memory was all reserved at start-up, a host plugin without
+ * an allocator of its own). Results are the same bytes as aqd_conv_int with a workspace.
+ * The first call on a device looks the array up (cudaGetSymbolAddress); make it before any
+ * stream capture. Every call on a device shares the one array: calls that overlap in time
+ * (other streams, other host threads) race on it and must be ordered by the caller;
+ * nothing in it needs to start at zero (each call writes every byte it reads).
+ * Returns AQD_ERR_UNSUPPORTED, launching nothing, when the workspace path does not apply
+ * (aqd_conv_workspace_bytes would be 0) or needs more than AQD_STATIC_WORKSPACE_BYTES. */
+aqd_status aqd_conv_int_static_workspace(const aqd_tensor* x, const aqd_conv_weights* w, int32_t stride,
+                                         int32_t pad, int32_t level, const aqd_requant_params* rq,
+                                         const aqd_tensor* skip, const aqd_skip_params* sp, aqd_tensor* y,
+                                         aqd_stream_t stream);
+
 /* ---- elementwise ------------------------------------------------------------------ */
 
 /* y = requant(sat32(acc + bias)) per channel at `level`: Eq. 6 + Eq. 2 on an int32

@@ -57,7 +57,7 @@ EXPORTS = ["aqd_row_bytes", "aqd_quantize_multiplier", "aqd_status_string", "aqd
            "aqd_unpack_codes", "aqd_conv_weights_bytes", "aqd_conv_prepare_weights", "aqd_conv_int",
            "aqd_conv_int_grouped", "aqd_conv_workspace_bytes", "aqd_conv_expand_input",
            "aqd_conv_int_grouped_expanded", "aqd_conv_int_grouped_chain", "aqd_requant", "aqd_residual_add_int",
-           "aqd_maxpool_codes"]
+           "aqd_maxpool_codes", "aqd_conv_int_static_workspace"]
 
 _lib = None
 
@@ -104,6 +104,10 @@ def load(build_if_missing: bool = True):
     L.aqd_conv_int_grouped_chain.argtypes = [ctypes.POINTER(_Job), i32, ctypes.POINTER(_Weights), i32, i32,
                                              ctypes.POINTER(_Requant), ctypes.POINTER(_Skip), vp, ctypes.c_size_t,
                                              i32, vp, ctypes.c_size_t, vp]
+    L.aqd_conv_int_static_workspace.argtypes = [ctypes.POINTER(_Tensor), ctypes.POINTER(_Weights), i32, i32, i32,
+                                                ctypes.POINTER(_Requant), ctypes.POINTER(_Tensor),
+                                                ctypes.POINTER(_Skip), ctypes.POINTER(_Tensor), vp]
+    L.aqd_conv_int_static_workspace.restype = c_int
     L.aqd_conv_workspace_bytes.restype = ctypes.c_size_t
     L.aqd_conv_workspace_bytes.argtypes = [ctypes.POINTER(_Job), i32, ctypes.POINTER(_Weights), i32, i32]
     L.aqd_requant.argtypes = [ctypes.POINTER(_Tensor), ctypes.POINTER(_Requant), i32, ctypes.POINTER(_Tensor), vp]
@@ -305,6 +309,24 @@ def conv_int(x: DTensor, w: ConvWeights, stride: int, pad: int, y: DTensor, *, l
                                ctypes.byref(spc) if spc is not None else None, ctypes.byref(yc), wsp, wsb,
                                _stream(stream)),
            "aqd_conv_int")
+    return y
+
+
+def conv_int_static_workspace(x: DTensor, w: ConvWeights, stride: int, pad: int, y: DTensor, *, level: int = 0,
+                              rq: RequantParams | None = None, skip: DTensor | None = None,
+                              sp: SkipParams | None = None, stream=None) -> DTensor:
+    """conv_int on the workspace path with the library's own fixed workspace (no allocation);
+    calls that overlap in time share that workspace and must be ordered by the caller."""
+    xc, yc = x.ct(), y.ct()
+    rqc = rq.c() if rq is not None else None
+    skc = skip.ct() if skip is not None else None
+    spc = sp.cs() if sp is not None else None
+    _check(load().aqd_conv_int_static_workspace(ctypes.byref(xc), ctypes.byref(w.desc), stride, pad, level,
+                                                ctypes.byref(rqc) if rqc is not None else None,
+                                                ctypes.byref(skc) if skc is not None else None,
+                                                ctypes.byref(spc) if spc is not None else None, ctypes.byref(yc),
+                                                _stream(stream)),
+           "aqd_conv_int_static_workspace")
     return y
 
 

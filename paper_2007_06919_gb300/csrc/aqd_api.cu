@@ -504,4 +504,59 @@ aqd_status aqd_maxpool_codes(const aqd_tensor* x, int32_t k, int32_t stride, int
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------- static workspace
+// A fixed expanded-activation workspace inside the library, for callers that cannot
+// allocate device memory themselves: code that runs after its process's device memory
+// budget was fixed (a serving loop that pre-reserves everything at start-up and treats any
+// later allocation as a failure), or a host plugin that holds no allocator of its own.
+// One array per device context, shared by every call: the expansion pass of each call
+// writes every byte the convolution then reads (zero border included), so nothing in it
+// has to start at zero; two calls that overlap in time (different streams, or host
+// threads) race on it and must be ordered by the caller.
+static __device__ __align__(256) uint8_t g_static_ws[AQD_STATIC_WORKSPACE_BYTES];
+
+static uint8_t* static_ws_ptr(std::string* err) {
+  static std::mutex mu;
+  static uint8_t* ptrs[64] = {nullptr};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    *err = "cudaGetDevice failed";
+    return nullptr;
+  }
+  std::lock_guard<std::mutex> lk(mu);
+  if (!ptrs[dev]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_static_ws);
+    if (e != cudaSuccess) {
+      *err = std::string("cudaGetSymbolAddress(static workspace): ") + cudaGetErrorString(e);
+      return nullptr;
+    }
+    ptrs[dev] = static_cast<uint8_t*>(p);
+  }
+  return ptrs[dev];
+}
+
+extern "C" {
+
+aqd_status aqd_conv_int_static_workspace(const aqd_tensor* x, const aqd_conv_weights* w, int32_t stride,
+                                         int32_t pad, int32_t level, const aqd_requant_params* rq,
+                                         const aqd_tensor* skip, const aqd_skip_params* sp, aqd_tensor* y,
+                                         aqd_stream_t stream) {
+  if (!x || !y) return fail(AQD_ERR_INVALID, "x and y must not be NULL");
+  aqd_conv_job job{};
+  job.x = *x;
+  job.y = *y;
+  const size_t need = aqd_conv_workspace_bytes(&job, 1, w, stride, pad);
+  if (need == 0) return fail(AQD_ERR_UNSUPPORTED, "the expanded-activation workspace path does not apply");
+  if (need > (size_t)AQD_STATIC_WORKSPACE_BYTES)
+    return fail(AQD_ERR_UNSUPPORTED, "needs " + std::to_string(need) + " workspace bytes, more than the " +
+                                         std::to_string((size_t)AQD_STATIC_WORKSPACE_BYTES) + " of the static one");
+  std::string err;
+  uint8_t* ws = static_ws_ptr(&err);
+  if (!ws) return fail(AQD_ERR_CUDA, err);
+  return aqd_conv_int(x, w, stride, pad, level, rq, skip, sp, y, ws, (size_t)AQD_STATIC_WORKSPACE_BYTES, stream);
+}
+
+}  // extern "C"
 }  // namespace aqd

@@ -37,7 +37,7 @@ METRIC = "int-only conv TOPS & % of INT8 tensor peak; detector-head images/s at 
 # DRAM bytes (read + write) of one workspace-fed tower-layer conv_tc launch, taken from an
 # ncu capture of this kernel on this workload (dram__bytes_read.sum + dram__bytes_write.sum).
 # Re-measure (or set to None) whenever conv_tc_kernel changes.
-TOWER_CONV_DRAM_BYTES = None
+TOWER_CONV_DRAM_BYTES = 12_691_200
 KREP = 16  # tower-layer convs per timed kernel graph (16 x 12 MB workspaces > 129 MB L2)
 WORKLOAD = "retina_head_800x1333_b2_2bit"
 
@@ -278,26 +278,23 @@ def main():
     graph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(graph, stream=stream):
         step()
-    # the dominant kernel alone: the tensor-core conv of one grouped 256->256 tower layer over
-    # all levels, fed from workspaces expanded beforehand (outside the timed graph). One graph
-    # replays KREP launches back to back, each reading its own workspace, so the launches'
-    # combined working set (KREP x 12 MB) exceeds L2 and one graph-launch overhead is spread
-    # over KREP kernels.
+    # the dominant kernel alone: the chained tensor-core conv of one grouped 256->256 tower
+    # layer over all levels, as in the step. One graph replays KREP launches back to back;
+    # launch i reads workspace i and writes its output image into workspace i + KREP/2, which
+    # is read again only KREP/2 launches later, so every launch reads an input that has left
+    # L2 (KREP x 12 MB > 129 MB), and one graph-launch overhead is spread over KREP kernels.
     kjobs = [(xs[l], bufs[0][l], None, l) for l in range(nl)]
     kgraph = torch.cuda.CUDAGraph()
-    krep = KREP if ws is not None else 1
-    if ws is not None:
-        kws = [aqd.workspace_for(kjobs, tower_w[0], 1, 1, device=dev) for _ in range(krep)]
-        with torch.cuda.stream(stream):
-            for w_ in kws:
-                aqd.conv_expand_input(kjobs, tower_w[0], 1, 1, w_, stream=stream)
-        stream.synchronize()
-        with torch.cuda.graph(kgraph, stream=stream):
-            for w_ in kws:
-                aqd.conv_int_grouped_expanded(kjobs, tower_w[0], 1, 1, rq=tower_rq[0], workspace=w_, stream=stream)
-    else:
-        with torch.cuda.graph(kgraph, stream=stream):
-            aqd.conv_int_grouped(kjobs, tower_w[0], 1, 1, rq=tower_rq[0], stream=stream)
+    krep = KREP
+    kws = [aqd.workspace_for(kjobs, tower_w[0], 1, 1, device=dev) for _ in range(krep)]
+    with torch.cuda.stream(stream):
+        for w_ in kws:
+            aqd.conv_expand_input(kjobs, tower_w[0], 1, 1, w_, stream=stream)
+    stream.synchronize()
+    with torch.cuda.graph(kgraph, stream=stream):
+        for i in range(krep):
+            aqd.conv_int_grouped_chain(kjobs, tower_w[0], 1, 1, rq=tower_rq[0], workspace=kws[i], next_pad=1,
+                                       next_workspace=kws[(i + krep // 2) % krep], stream=stream)
 
     ops = head_ops(levels, batch)
     ops_step = float(sum(ops))
@@ -369,10 +366,9 @@ def main():
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "images_per_s": world * batch / (ms_per_step * 1e-3),
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": fp8_peak, "unit": "TFLOP/s",
-                     "frac": achieved / fp8_peak, "traffic": TOWER_CONV_DRAM_BYTES if ws is not None else None,
-                     "kernel": "conv_tc_kernel: one 3x3 256->256 tower layer, all 5 levels grouped" +
-                               (f" (workspace expanded beforehand; {krep} launches per timed graph, each on "
-                                "its own workspace, working set > L2)" if ws is not None else ""),
+                     "frac": achieved / fp8_peak, "traffic": TOWER_CONV_DRAM_BYTES,
+                     "kernel": "conv_tc_kernel (CTA pairs): one chained 3x3 256->256 tower layer, all 5 levels "
+                               f"grouped; {krep} launches per timed graph on distinct workspaces, working set > L2",
                      "algorithmic_ops_per_launch": ops[0],
                      "peak_source": f"{src} bf16 dense burst x 2 (nominal e4m3/bf16 ratio)",
                      "avg_launch_ms": kern_avg_ms},

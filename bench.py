@@ -201,6 +201,144 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def run_sweep(args):
+    """Measurements of the other workloads, one JSON line each (not the bench line): the
+    3x3 64->64 2-bit conv, the ResNet-50 C3 bottleneck block, and the head's first tower
+    layer at batch 16 for 2/3/4/8-bit codes, all levels grouped and each level alone.
+    TOPS = 2*M*N*K of the real convs / time; GB/s = packed input + packed output + packed
+    weights / time (the algorithmic bytes); L2 flushed before every timed replay."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2007_06919_gb300 import aqd, synth
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    stream = torch.cuda.Stream()
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    peaks, src = measured_peaks()
+    fp8_peak = 2.0 * peaks["bf16_tflops"]
+    reps = max(20, min(200, args.steps // 10))
+
+    def timed(fn):
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                fn()
+        stream.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            fn()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+        with torch.cuda.stream(stream):
+            for a, b in ev:
+                flush.fill_(1)
+                a.record(stream)
+                g.replay()
+                b.record(stream)
+        stream.synchronize()
+        assert aqd.device_status(stream) == 0
+        return statistics.median(a.elapsed_time(b) for a, b in ev)
+
+    def emit(name, ms, ops, nbytes, **kw):
+        line = {"sweep": name, "ms": ms, "TOPS": ops / (ms * 1e-3) / 1e12,
+                "GB_s": nbytes / (ms * 1e-3) / 1e9, "frac_e4m3_peak": ops / (ms * 1e-3) / 1e12 / fp8_peak,
+                "peak_source": src, "l2": "flushed before every replay", **kw}
+        print(json.dumps(line), flush=True)
+
+    def dt(codes, bits):
+        return aqd.DTensor.from_codes(torch.from_numpy(codes).to(dev), bits)
+
+    want = args.sweep
+    # config 0: 3x3 64->64, 32x32, batch 1, 2-bit (one small launch)
+    wl = synth.config0()
+    cv = wl.convs[0]
+    x = dt(wl.inputs[0], 2)
+    y = aqd.DTensor.empty(1, 32, 32, 64, 2, device=dev)
+    W = aqd.ConvWeights(torch.from_numpy(cv.w).to(dev), 2)
+    rq = aqd.RequantParams.from_numpy(cv.m0, cv.shift, cv.bias, device=dev)
+    if want in ("all", "config0"):
+        ms = timed(lambda: aqd.conv_int(x, W, 1, 1, y, rq=rq, stream=stream))
+        emit("config0_conv3x3_64_32x32_b1_2bit", ms, 2 * 1024 * 64 * 576, 8192 + 8192 + 64 * 576 // 4)
+
+    # config 1: ResNet-50 C3 bottleneck (1x1 512->128, 3x3 128->128, 1x1 128->512 + identity)
+    wl = synth.config1()
+    x = dt(wl.inputs[0], 4)
+    n, h, w = 2, 100, 152
+    Ws = [aqd.ConvWeights(torch.from_numpy(c.w).to(dev), 4) for c in wl.convs]
+    rqs = [aqd.RequantParams.from_numpy(c.m0, c.shift, c.bias, device=dev) for c in wl.convs]
+    c3 = wl.convs[2]
+    sp = aqd.SkipParams.from_numpy(c3.skip_c, c3.skip_d, device=dev)
+    t1 = aqd.DTensor.empty(n, h, w, 128, 4, device=dev)
+    t2 = aqd.DTensor.empty(n, h, w, 128, 4, device=dev)
+    out = aqd.DTensor.empty(n, h, w, 512, 4, device=dev)
+    wsx = aqd.workspace_for([(x, None, None, 0)], Ws[0], 1, 0, device=dev)
+    ws1 = torch.zeros(aqd.conv_workspace_bytes([(t1, None, None, 0)], Ws[1], 1, 1) + 256, dtype=torch.uint8,
+                      device=dev)
+    ws1 = ws1[(-ws1.data_ptr()) % 256:][:aqd.conv_workspace_bytes([(t1, None, None, 0)], Ws[1], 1, 1)]
+    ws2 = aqd.workspace_for([(t2, None, None, 0)], Ws[2], 1, 0, device=dev)
+
+    def block():
+        aqd.conv_expand_input([(x, None, None, 0)], Ws[0], 1, 0, wsx, stream=stream)
+        aqd.conv_int_grouped_chain([(x, t1, None, 0)], Ws[0], 1, 0, rq=rqs[0], workspace=wsx, next_pad=1,
+                                   next_workspace=ws1, stream=stream)
+        aqd.conv_int_grouped_chain([(t1, t2, None, 0)], Ws[1], 1, 1, rq=rqs[1], workspace=ws1, next_pad=0,
+                                   next_workspace=ws2, stream=stream)
+        aqd.conv_int_grouped_expanded([(t2, out, x, 0)], Ws[2], 1, 0, rq=rqs[2], sp=sp, workspace=ws2,
+                                      stream=stream)
+    m = n * h * w
+    if want not in ("all", "config1"):
+        parts_wanted = False
+    else:
+        parts_wanted = True
+    ops = 2 * m * (128 * 512 + 128 * 1152 + 512 * 128)
+    nbytes = m * (256 + 64 + 64 + 64 + 256 + 256) + (128 * 512 + 128 * 1152 + 512 * 128) // 2
+    if parts_wanted:
+        ms = timed(block)
+        emit("config1_r50_c3_bottleneck_b2_100x152_4bit", ms, ops, nbytes, images_per_s=n / (ms * 1e-3),
+             launches=4)
+    parts = [("expand_x", lambda: aqd.conv_expand_input([(x, None, None, 0)], Ws[0], 1, 0, wsx, stream=stream), 0),
+             ("conv1x1_512_128", lambda: aqd.conv_int_grouped_chain([(x, t1, None, 0)], Ws[0], 1, 0, rq=rqs[0],
+                                                                    workspace=wsx, next_pad=1, next_workspace=ws1,
+                                                                    stream=stream), 2 * m * 128 * 512),
+             ("conv3x3_128_128", lambda: aqd.conv_int_grouped_chain([(t1, t2, None, 0)], Ws[1], 1, 1, rq=rqs[1],
+                                                                    workspace=ws1, next_pad=0, next_workspace=ws2,
+                                                                    stream=stream), 2 * m * 128 * 1152),
+             ("conv1x1_128_512_skip", lambda: aqd.conv_int_grouped_expanded([(t2, out, x, 0)], Ws[2], 1, 0, rq=rqs[2],
+                                                                           sp=sp, workspace=ws2, stream=stream),
+              2 * m * 512 * 128)]
+    for nm, fn, o in (parts if parts_wanted else []):
+        ms = timed(fn)
+        emit(f"config1_part_{nm}", ms, o, 0)
+
+    # config 4: first tower layer of the head at batch 16, 2/3/4/8-bit
+    for bits in ((2, 3, 4, 8) if want in ("all", "config4") else ()):
+        wl = synth.config4(bits)
+        levels = wl.extra["levels"]
+        cv = wl.convs[0]
+        xs = [dt(xi, bits) for xi in wl.inputs]
+        ys = [aqd.DTensor.empty(16, hh, ww, 256, bits, device=dev) for (hh, ww) in levels]
+        W = aqd.ConvWeights(torch.from_numpy(cv.w).to(dev), bits)
+        rq = aqd.RequantParams.from_numpy(cv.m0, cv.shift, cv.bias, device=dev)
+        row = aqd.row_bytes(256, bits)
+
+        def work(ls):
+            jobs = [(xs[l], ys[l], None, l) for l in ls]
+            ws = aqd.workspace_for(jobs, W, 1, 1, device=dev)
+
+            def fn():
+                aqd.conv_int_grouped(jobs, W, 1, 1, rq=rq, workspace=ws, stream=stream)
+            px = sum(16 * levels[l][0] * levels[l][1] for l in ls)
+            return fn, 2 * px * 256 * 2304, px * 2 * row + 256 * 2304 * bits // 8
+        fn, ops, nbytes = work(range(5))
+        ms = timed(fn)
+        emit(f"config4_tower_layer_b16_{bits}bit_all_levels", ms, ops, nbytes, bits=bits,
+             path=aqd.last_conv_path())
+        for l in range(5):
+            fn, ops, nbytes = work([l])
+            ms = timed(fn)
+            emit(f"config4_tower_layer_b16_{bits}bit_level{l}", ms, ops, nbytes, bits=bits, level=levels[l],
+                 path=aqd.last_conv_path())
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--steps", type=int, default=2000)
@@ -208,9 +346,13 @@ def main():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", nargs="?", const="all", default=None, choices=["all", "config0", "config1", "config4"],
+                    help="measure the other workloads (several lines)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.sweep:
+        return run_sweep(args)
     assert args.warmup >= 3, "at least 3 warm-up steps"
 
     import torch

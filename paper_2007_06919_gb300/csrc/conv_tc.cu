@@ -409,22 +409,72 @@ __device__ __forceinline__ TileInfo tile_info(const Params& p, int t) {
 
 // Eq. 6 -> Eq. 7 -> Eq. 2 in int64 for 32 accumulators of one row (any shift, any skip).
 // Kept out of line: the common cases take the 32-bit fast path in the kernel body.
-__device__ __noinline__ void general_epilogue(const Params& p, const uint32_t* v, const EpiChan* ep,
-                                              const uint8_t* srow, int ch0, int ncols, int32_t* out) {
-  int32_t sk[32];
-  if (p.has_skip) {
-    if (p.skip_bits == 32) {
-      for (int i = 0; i < 32; ++i)
-        sk[i] = (i < ncols && ch0 + i < p.cout) ? reinterpret_cast<const int32_t*>(srow)[ch0 + i] : 0;
+// Eq. 6 -> Eq. 7 -> Eq. 2 in int64 for 32 accumulators of one row (any shift, any skip),
+// all in registers: the 32 skip values are loaded and unpacked per skip width, every index
+// is static, and nothing goes through local memory.
+__device__ __forceinline__ void load_skip_group(const Params& p, const uint8_t* srow, int ch0, int ncols,
+                                                int32_t (&sk)[32]) {
+#pragma unroll
+  for (int i = 0; i < 32; ++i) sk[i] = 0;
+  {
+    const int sb = p.skip_bits;
+    if (sb == 32) {
+      const int32_t* s32 = reinterpret_cast<const int32_t*>(srow) + ch0;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) sk[i] = (i < ncols && ch0 + i < p.cout) ? __ldg(s32 + i) : 0;
+    } else if (sb == 8) {
+      const uint8_t* s8 = srow + ch0;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) sk[i] = (i < ncols && ch0 + i < p.cout) ? (int32_t)__ldg(s8 + i) : 0;
     } else {
-      unpack_group_vals(srow + (ch0 >> 5) * group_bytes(p.skip_bits), p.skip_bits, false, sk);
+      // 2/3/4-bit codes: one whole packed group (the layout needs cout % 32 == 0)
+      const uint32_t* g32 = reinterpret_cast<const uint32_t*>(srow + (ch0 >> 5) * group_bytes(sb));
+      uint32_t g[4] = {__ldg(g32), __ldg(g32 + 1), sb >= 3 ? __ldg(g32 + 2) : 0u, sb == 4 ? __ldg(g32 + 3) : 0u};
+      uint32_t b[8];
+      if (sb == 2) unpack_group_bytes<2>(g, b);
+      else if (sb == 3) unpack_group_bytes<3>(g, b);
+      else unpack_group_bytes<4>(g, b);
+#pragma unroll
+      for (int i = 0; i < 32; ++i) sk[i] = (int32_t)((b[i / 4] >> (8 * (i % 4))) & 0xFFu);
     }
   }
+}
+
+template <bool kSkip>
+__device__ __forceinline__ void general_group(const Params& p, const uint32_t* v, const EpiChan* ep,
+                                              const uint8_t* srow, int ch0, int ncols, int32_t (&out)[32]) {
+  int32_t sk[32];
+  if (kSkip && p.has_skip) load_skip_group(p, srow, ch0, ncols, sk);
+  else {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) sk[i] = 0;
+  }
+#pragma unroll
   for (int i = 0; i < 32; ++i) {
     const int64_t acc = (int64_t)__float2int_rn(__uint_as_float(v[i]) * 262144.0f);  // exact
     const EpiChan ec = ep[i];
-    out[i] = p.has_skip ? epilogue<true>(acc, sk[i], ec, p.scale_main, p.out_bits)
+    out[i] = (kSkip && p.has_skip) ? epilogue<true>(acc, sk[i], ec, p.scale_main, p.out_bits)
                         : epilogue<false>(acc, 0, ec, p.scale_main, p.out_bits);
+  }
+}
+
+// Skip epilogue in 32-bit arithmetic (Eq. 6, Eq. 7 with the skip rescaled, Eq. 2) when, for
+// every column of the tile, R = 31 + shift >= 33, |bias| <= 2^30 and d >= 8, and the skip
+// holds k-bit codes (s <= 255): then rhu(s * c, d) = (s * c + 2^(d-1)) >> d fits in int32,
+// acc + bias cannot overflow (|acc| < 2^24), and one saturating add gives sat32 of the
+// exact sum; the requant is the same 32-bit form as fast_requant_group.
+// (y may be sk itself: element i is read before it is written)
+__device__ __forceinline__ void fast_skip_group(const uint32_t* v, const EpiChan* ep, const int32_t (&sk)[32],
+                                                int qmax, int32_t (&y)[32]) {
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    const EpiChan c = ep[i];
+    const int32_t acc = __float2int_rn(__uint_as_float(v[i]) * 262144.0f);  // exact integer
+    const int64_t sc = (int64_t)sk[i] * (int64_t)c.c;
+    const int32_t st = (int32_t)((sc + (1LL << (c.d - 1))) >> c.d);
+    const int32_t u = add_sat(acc + c.bias, st);
+    const int r = c.r;
+    y[i] = min(max((__mulhi(u, c.m0) + (1 << (r - 33))) >> (r - 32), 0), qmax);
   }
 }
 
@@ -553,7 +603,9 @@ __device__ __forceinline__ void load_chunk(const Params& p, RowCursor<kXBits>& r
   }
 }
 
-template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair>
+// kSkip: the instantiation that handles a skip tensor (Eq. 7); the others carry no skip code,
+// which keeps the common path's registers free.
+template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair, bool kSkip>
 __global__ void __launch_bounds__(threads_for(kFlat), 1)
 conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_wh,
                const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ Params p) {
@@ -878,6 +930,14 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       }
       fast_req = named_bar_and(1, kEpiThreads, fast_req);
       small_bias = named_bar_and(1, kEpiThreads, small_bias);
+      // 32-bit skip path (fast_skip_group): default direction, code skips, d >= 8 everywhere
+      int fast_skip = 0;
+      if (kSkip && p.has_skip && p.scale_main == 0 && p.skip_bits <= 8 && out_bits != 32 && fast_req && small_bias) {
+        int ok8 = 1;
+        for (int col = et; col < TBN; col += kEpiThreads)
+          if (ti.col0 + col < p.cout && epi[col].d < 8) ok8 = 0;
+        fast_skip = named_bar_and(1, kEpiThreads, ok8);
+      }
       // 0: general int64 epilogue; 1: fast requant to codes; 2: int32 output, no skip
       const int mode = p.has_skip ? 0 : (out_bits == 32 ? 2 : (fast_req ? 1 : 0));
       const bool magic = p.acc_small && (mode == 2 ? small_bias : fast_req);
@@ -900,7 +960,9 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       }
       for (int u0 = gi; u0 < nunits; u0 += kGroups) {
         const int un = u0 + kGroups;
-        if (un < nunits)
+        // the next unit's TMEM load overlaps this unit's work in the light modes; the general /
+        // skip mode (0) holds more registers and loads it afterwards
+        if (un < nunits && mode != 0)
           tmem_ld32(tbuf + (un / ngrp) * (uint32_t)BN + (un % ngrp) * 32, TBN - (un % ngrp) * 32 >= 32, vn);
         const int sub = u0 / ngrp, g0 = (u0 % ngrp) * 32;
         const int ncols = (TBN - g0) < 32 ? (TBN - g0) : 32;
@@ -967,7 +1029,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
             }
           } else {
             const uint8_t* srow = nullptr;
-            if (p.has_skip) {
+            if (kSkip && p.has_skip) {
               const int hw = jb.ho * jb.wo;
               const int img = m / hw;
               const int rem = m - img * hw;
@@ -975,13 +1037,16 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
               const int sh = ho / p.upsample, sw = wo / p.upsample;
               srow = jb.skip + (((int64_t)img * jb.skip_h + sh) * jb.skip_w + sw) * p.skip_row_bytes;
             }
-            uint32_t vv[32];  // local copies: only this rare path goes through the stack
             int32_t oo[32];
-  #pragma unroll
-            for (int i = 0; i < 32; ++i) vv[i] = v[i];
-            general_epilogue(p, vv, epi + g0, srow, ch0, ncols, oo);
+            if (kSkip && fast_skip) {
+              load_skip_group(p, srow, ch0, ncols, oo);   // skip codes, replaced by the results
+              fast_skip_group(v, epi + g0, oo, qmax, oo);
+            } else {
+              general_group<kSkip>(p, v, epi + g0, srow, ch0, ncols, oo);
+            }
             if (out_bits == 32) {
               int32_t* yr = reinterpret_cast<int32_t*>(yrow) + ch0;
+#pragma unroll
               for (int i = 0; i < 32; ++i)
                 if (i < ncols && ch0 + i < p.cout) yr[i] = oo[i];
             } else {
@@ -993,6 +1058,8 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
           }
         }
         if (un < nunits) {
+          if (mode == 0)
+            tmem_ld32(tbuf + (un / ngrp) * (uint32_t)BN + (un % ngrp) * 32, TBN - (un % ngrp) * 32 >= 32, vn);
           tmem_wait_ld();
           reg_fence32(vn);
 #pragma unroll
@@ -1169,10 +1236,10 @@ static EncodeTiledFn get_encode_fn(std::string* err) {
   return fn;
 }
 
-template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair = false>
+template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair = false, bool kSkip = true>
 static int launch_bits(const Params& prm, const CUtensorMap& map, const CUtensorMap& map_h, const CUtensorMap& map_a,
                        int grid, size_t smem, cudaStream_t stream, std::string* err) {
-  auto kern = conv_tc_kernel<kXBits, kChunkInTap, kFlat, kPair>;
+  auto kern = conv_tc_kernel<kXBits, kChunkInTap, kFlat, kPair, kSkip>;
   // The opt-in limit is raised to the device maximum, never lowered to this call's size:
   // a CUDA graph node captured earlier with a larger plan must stay launchable (a graph
   // node, or a tool relaunching it, is checked against the function's current limit).
@@ -1380,8 +1447,11 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
       *err = "cuTensorMapEncodeTiled (activations) failed: " + std::to_string((int)r2);
       return 3;
     }
-    if (pair) return launch_bits<2, true, true, true>(prm, map, map_h, map_a, grid, smem, stream, err);
-    return launch_bits<2, true, true>(prm, map, map_h, map_a, grid, smem, stream, err);
+    if (pair)
+      return a.has_skip ? launch_bits<2, true, true, true, true>(prm, map, map_h, map_a, grid, smem, stream, err)
+                        : launch_bits<2, true, true, true, false>(prm, map, map_h, map_a, grid, smem, stream, err);
+    return a.has_skip ? launch_bits<2, true, true, false, true>(prm, map, map_h, map_a, grid, smem, stream, err)
+                      : launch_bits<2, true, true, false, false>(prm, map, map_h, map_a, grid, smem, stream, err);
   }
   switch (a.x_bits) {
     case 2: return in_tap ? launch_bits<2, true, false>(prm, map, map_h, map_a, grid, smem, stream, err)

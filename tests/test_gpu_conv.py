@@ -194,3 +194,51 @@ def test_invalid_skip_shape_is_rejected_before_launch():
         aqd.conv_int(X, W, 1, 1, Y, rq=rq, skip=S, sp=sp)
     assert e.value.status == 1
     torch.cuda.synchronize()
+
+
+@pytest.mark.parametrize("shape", [(1, 37, 53), (2, 24, 40)])
+def test_first_conv_8bit_rgb_7x7_s2_bit_exact(shape):
+    """The network's first conv (config 3): 8-bit unsigned image codes with 3 channels,
+    7x7 stride 2 padding 3, 4-bit weight values (stored as 8-bit codes: a 3-channel row has
+    no 4-bit packed layout), 64 channels of 4-bit codes out."""
+    n, h, wd = shape
+    rng = np.random.default_rng(h * 1000 + wd)
+    x = synth.act_codes(rng, (n, h, wd, 3), 8)
+    w = synth.weight_codes(rng, (64, 7, 7, 3), 4, "normal2")
+    std = np.sqrt(147 * np.mean(np.arange(256) ** 2) * 4.0)
+    m0, sh, b = _params(rng, 1, 64, 4, calib_std=std)
+    got, want, used = conv_pair(x, 8, w, 8, stride=2, pad=3, out_bits=4, m0=m0, shift=sh, bias=b, path=0)
+    assert used == DIRECT  # 8-bit codes and cin 3 take the exact int32 CUDA-core kernel
+    assert_same(got, want, 64, 4, f"first conv {shape}")
+    assert len(np.unique(oracle_unpack(want, 64, 4))) > 4
+
+
+def test_first_conv_full_size_sampled():
+    """The first conv at the config-3 size (batch 8, 800x1344 after padding): oracle on
+    sampled output pixels, every output channel."""
+    import oracle
+    import torch
+    from gpu_util import dev
+    from paper_2007_06919_gb300 import aqd
+    rng = np.random.default_rng(3)
+    n, h, wd = 8, 800, 1344
+    x = synth.act_codes(rng, (n, h, wd, 3), 8)
+    w = synth.weight_codes(rng, (64, 7, 7, 3), 4, "normal2")
+    std = np.sqrt(147 * np.mean(np.arange(256) ** 2) * 4.0)
+    m0, sh, b = _params(rng, 1, 64, 4, calib_std=std)
+    xt = oracle.CodeTensor.from_codes(x, 8)
+    W, wp = weights(w, 8)
+    X = aqd.DTensor(dev(xt.packed), n, h, wd, 3, 8)
+    Y = aqd.DTensor.empty(n, 400, 672, 64, 4)
+    aqd.conv_int(X, W, 2, 3, Y, rq=aqd.RequantParams.from_numpy(m0, sh, b))
+    torch.cuda.synchronize()
+    pix = synth.sample_pixels(rng, n * 400 * 672, 2000)
+    want = oracle.conv_int_pixels(xt, wp, 8, 0, 7, 7, 2, 3, 64, pix, m0=m0, shift=sh, bias=b, out_bits=4)
+    got = oracle.unpack(Y.data.cpu().numpy().reshape(n * 400 * 672, -1)[pix], 64, 4)
+    assert np.array_equal(got, want)
+    assert aqd.device_status() == 0
+
+
+def oracle_unpack(packed, c, bits):
+    import oracle
+    return oracle.unpack(packed, c, bits)

@@ -55,7 +55,11 @@ WeightGeom weight_geom(int32_t cout, int32_t kh, int32_t kw, int32_t cin) {
   g.k_pad = (g.k_total + 127) / 128 * 128;
   g.bn = cout <= 256 ? (cout + 15) / 16 * 16 : 256;  // N tile of the tensor-core kernel
   g.cout_pad = (cout + g.bn - 1) / g.bn * g.bn;
-  g.e4m3_bytes = (size_t)g.cout_pad * g.k_pad;
+  g.split_rows = 2 * ((cout + 127) / 128 * 128);
+  // the tensor-core weight block holds either layout: [cout_pad][k_pad] E4M3 bytes for
+  // |w| <= 15, or, for 8-bit weights, per 128 output channels 128 rows of w_lo = w & 15 then
+  // 128 rows of w_hi = w >> 4 (floor), so it is sized for the larger of the two
+  g.e4m3_bytes = (size_t)(g.cout_pad > g.split_rows ? g.cout_pad : g.split_rows) * g.k_pad;
   g.i16_offset = (g.e4m3_bytes + 255) / 256 * 256;
   g.total_bytes = g.i16_offset + 2 * (size_t)cout * g.k_total;
   return g;
@@ -203,29 +207,44 @@ aqd_status aqd_conv_prepare_weights(const void* w_packed, const aqd_conv_weights
 }
 
 // Rows (of cin bytes) of the expanded-activation workspace, or 0 if that path does not apply.
+// Whether 8-bit operands go through the split form on the tensor cores (see ConvArgs).
+static bool split_weights(const aqd_conv_weights* w) { return w->w_bits == 8 && w->w_format == AQD_W_TWOS; }
+
+// Rows (of cin bytes, per plane) of the expanded-activation workspace, or 0 if that path does
+// not apply. 8-bit activations take two planes; 8-bit two's-complement weights the split
+// layout. Every partial sum of the FP32 accumulator stays exact while K * 3825 < 2^24
+// (x_lo * w_lo + 16 x_hi * w_lo <= 15 * 255 per term, w_hi likewise smaller).
 static int64_t flat_rows(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w, int32_t stride,
-                         int32_t pad) {
+                         int32_t pad, int32_t* planes = nullptr) {
   if (!jobs || njobs <= 0 || njobs > kMaxJobs || !w) return 0;
-  if (stride != 1 || pad < 0 || w->cin <= 0 || w->cin % 128 != 0 || w->w_bits < 2 || w->w_bits > 4) return 0;
+  if (stride != 1 || pad < 0 || w->cin <= 0 || w->cin % 128 != 0) return 0;
   if (w->w_format != AQD_W_TWOS && w->w_format != AQD_W_ODD) return 0;
+  const bool wsplit = split_weights(w);
+  if (!(w->w_bits >= 2 && w->w_bits <= 4) && !wsplit) return 0;
   const int64_t max_w = max_abs_weight(w->w_bits, w->w_format);
-  if (max_w > 15) return 0;
+  if (max_w > 15 && !wsplit) return 0;
+  const int64_t k = (int64_t)w->kh * w->kw * w->cin;
   int64_t rows = 0;
+  int np = 1;
   for (int j = 0; j < njobs; ++j) {
     const aqd_tensor& x = jobs[j].x;
-    if (x.bits < 2 || x.bits > 4 || x.c != w->cin || x.n <= 0 || x.h <= 0 || x.w <= 0) return 0;
-    const int64_t k = (int64_t)w->kh * w->kw * w->cin;
-    if (k * ((1LL << x.bits) - 1) * max_w >= (1LL << 24)) return 0;
+    if (!(x.bits >= 2 && x.bits <= 4) && x.bits != 8) return 0;
+    if (x.c != w->cin || x.n <= 0 || x.h <= 0 || x.w <= 0) return 0;
+    if (x.bits == 8) np = 2;
+    const bool wide = x.bits == 8 || wsplit;
+    if (wide ? k * 3825 >= (1LL << 24) : k * ((1LL << x.bits) - 1) * max_w >= (1LL << 24)) return 0;
     rows += (int64_t)x.n * (x.h + 2 * pad) * (x.w + 2 * pad);
   }
-  // the expansion pass indexes (row, 128-channel block) pairs in 32 bits
-  return rows * (w->cin / 16) < (1LL << 31) ? rows : 0;
+  if (planes) *planes = np;
+  // the expansion pass indexes (row, 16-byte chunk) pairs of every plane in 32 bits
+  return rows * np * (w->cin / 16) < (1LL << 31) ? rows : 0;
 }
 
 size_t aqd_conv_workspace_bytes(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
                                 int32_t stride, int32_t pad) {
-  const int64_t rows = flat_rows(jobs, njobs, w, stride, pad);
-  return rows > 0 ? (size_t)rows * (size_t)w->cin : 0;
+  int32_t planes = 1;
+  const int64_t rows = flat_rows(jobs, njobs, w, stride, pad, &planes);
+  return rows > 0 ? (size_t)rows * (size_t)planes * (size_t)w->cin : 0;
 }
 
 // What one grouped call runs on the workspace path: expansion + convolution (the public
@@ -365,6 +384,8 @@ static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aq
   a.w_e4m3 = static_cast<const uint8_t*>(w->data);
   a.w_i16 = reinterpret_cast<const int16_t*>(static_cast<const uint8_t*>(w->data) + g.i16_offset);
   a.cout_pad = g.cout_pad; a.k_total = g.k_total; a.k_pad = g.k_pad; a.bn = g.bn;
+  a.split_rows = g.split_rows;
+  a.a_planes = 1;
   a.status = status_ptr(&err);
   if (!a.status) return fail(AQD_ERR_CUDA, err);
 
@@ -375,8 +396,15 @@ static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aq
   a.acc_bound = bound;
   const bool tc_ok = a.x_bits <= 4 && max_w <= 15 && (a.cin % 32) == 0 && bound < (1LL << 24);
   const bool direct_ok = bound < (1LL << 31);
-  int path = tc_ok ? 1 : 2;
-  if ((g_forced_path == 1 || g_forced_path == 3) && tc_ok) path = 1;
+  // 8-bit operands go to the tensor cores in split form, on the workspace path, without a skip
+  int32_t wide_planes = 1;
+  bool wide_ok = false;
+  if (!tc_ok && workspace && !has_skip && (a.x_bits == 8 || split_weights(w))) {
+    const int64_t rows = flat_rows(jobs, njobs, w, stride, pad, &wide_planes);
+    wide_ok = rows > 0 && (size_t)rows * (size_t)wide_planes * (size_t)w->cin <= ws_bytes;
+  }
+  int path = (tc_ok || wide_ok) ? 1 : 2;
+  if ((g_forced_path == 1 || g_forced_path == 3) && (tc_ok || wide_ok)) path = 1;
   a.no_pair = g_forced_path == 3 ? 1 : 0;
   if (g_forced_path == 2) path = 2;
   // expanded-activation path when a large enough, aligned workspace is supplied
@@ -385,12 +413,16 @@ static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aq
   if (path == 1 && workspace) {
     if ((reinterpret_cast<uintptr_t>(workspace) & 255) != 0)
       return fail(AQD_ERR_INVALID, "workspace must be 256-byte aligned");
-    const int64_t rows = flat_rows(jobs, njobs, w, stride, pad);
-    if (rows > 0 && (size_t)rows * (size_t)w->cin <= ws_bytes) {
+    int32_t planes = 1;
+    const int64_t rows = flat_rows(jobs, njobs, w, stride, pad, &planes);
+    if (rows > 0 && (size_t)rows * (size_t)planes * (size_t)w->cin <= ws_bytes) {
       a.ws = static_cast<uint8_t*>(workspace);
-      a.ws_rows = (int64_t)(ws_bytes / (size_t)w->cin);
+      a.ws_rows = (int64_t)(ws_bytes / ((size_t)planes * (size_t)w->cin));
+      a.a_planes = planes;
+      a.split_w = (!tc_ok && split_weights(w)) ? 1 : 0;
     }
   }
+  if (path == 1 && !tc_ok && !a.ws) path = 2;  // the split form exists only on the workspace path
   if (path == 2 && !direct_ok) return fail(AQD_ERR_UNSUPPORTED, "accumulator bound exceeds int32");
   if (stage != kStageBoth) {
     if (path != 1) return fail(AQD_ERR_UNSUPPORTED, "the tensor-core kernel does not take this convolution");
@@ -411,7 +443,7 @@ static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aq
     const size_t need = (size_t)orows * (size_t)w->cout;
     if (chain->bytes < need) return fail(AQD_ERR_INVALID, "next_workspace is too small");
     const uintptr_t i0 = reinterpret_cast<uintptr_t>(workspace), o0 = reinterpret_cast<uintptr_t>(chain->ws);
-    const size_t in_need = (size_t)flat_rows(jobs, njobs, w, stride, pad) * (size_t)w->cin;
+    const size_t in_need = (size_t)flat_rows(jobs, njobs, w, stride, pad) * (size_t)a.a_planes * (size_t)w->cin;
     if (i0 < o0 + need && o0 < i0 + in_need) return fail(AQD_ERR_INVALID, "workspace and next_workspace overlap");
     a.ws_out = static_cast<uint8_t*>(chain->ws);
     a.out_pad = chain->pad;

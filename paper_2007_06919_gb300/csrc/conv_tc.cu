@@ -92,6 +92,9 @@ struct Params {
   uint32_t off_b, off_epi, off_bar, off_qtab;
   uint8_t* ws_out;    // chained output image (NULL: none)
   int32_t out_pad;
+  int32_t a_planes;   // K runs over this many planes of the byte image (2: 8-bit activations)
+  int32_t plane_rows; // workspace rows per plane
+  int32_t split_w;    // weights in the split layout: a tile's bn B rows give bn/2 channels
   uint32_t* status;
 };
 
@@ -369,8 +372,10 @@ __device__ __forceinline__ void reg_fence32(uint32_t (&r)[32]) {
 
 struct TileInfo {
   int job, mt;
-  int bn;    // output channels of this tile: p.bn, or p.bn / 2 for a half tile
+  int bn;    // MMA N of this tile (weight rows): p.bn, or p.bn / 2 for a half tile
   int col0;  // first output channel
+  int brow;  // first weight row
+  int cn;    // output channels of this tile: bn, or bn / 2 with split weights
 };
 // Flat path: M tile mt of a job covers virtual rows [v0, v0 + 128) of image img, where the
 // virtual grid holds the output rows at the padded input width wp (stride 1).
@@ -401,7 +406,11 @@ __device__ __forceinline__ TileInfo tile_info(const Params& p, int t) {
   ti.mt = local / p.n_tiles;
   const int nt = local - ti.mt * p.n_tiles;
   ti.bn = half < 0 ? p.bn : p.bn / 2;
-  ti.col0 = nt * p.bn + (half > 0 ? p.bn / 2 : 0);
+  ti.brow = nt * p.bn + (half > 0 ? p.bn / 2 : 0);
+  // split weights (no half tiles): rows [brow, brow + bn/2) hold w_lo of bn/2 channels and
+  // the next bn/2 rows their w_hi
+  ti.cn = p.split_w ? ti.bn / 2 : ti.bn;
+  ti.col0 = p.split_w ? nt * (p.bn / 2) : ti.brow;
   return ti;
 }
 
@@ -440,7 +449,7 @@ __device__ __forceinline__ void load_skip_group(const Params& p, const uint8_t* 
   }
 }
 
-template <bool kSkip>
+template <bool kSkip, bool kIntAcc = false>
 __device__ __forceinline__ void general_group(const Params& p, const uint32_t* v, const EpiChan* ep,
                                               const uint8_t* srow, int ch0, int ncols, int32_t (&out)[32]) {
   int32_t sk[32];
@@ -451,7 +460,9 @@ __device__ __forceinline__ void general_group(const Params& p, const uint32_t* v
   }
 #pragma unroll
   for (int i = 0; i < 32; ++i) {
-    const int64_t acc = (int64_t)__float2int_rn(__uint_as_float(v[i]) * 262144.0f);  // exact
+    // v: FP32 accumulators of exact integers x 2^-18, or (kIntAcc) int32 sums already
+    const int64_t acc = kIntAcc ? (int64_t)(int32_t)v[i]
+                                : (int64_t)__float2int_rn(__uint_as_float(v[i]) * 262144.0f);
     const EpiChan ec = ep[i];
     out[i] = (kSkip && p.has_skip) ? epilogue<true>(acc, sk[i], ec, p.scale_main, p.out_bits)
                         : epilogue<false>(acc, 0, ec, p.scale_main, p.out_bits);
@@ -605,7 +616,8 @@ __device__ __forceinline__ void load_chunk(const Params& p, RowCursor<kXBits>& r
 
 // kSkip: the instantiation that handles a skip tensor (Eq. 7); the others carry no skip code,
 // which keeps the common path's registers free.
-template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair, bool kSkip>
+// kSplit: the 8-bit split form (split weights combined as D1 + 16 D2 in the epilogue).
+template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair, bool kSkip, bool kSplit>
 __global__ void __launch_bounds__(threads_for(kFlat), 1)
 conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_wh,
                const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ Params p) {
@@ -688,7 +700,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
   grid_dep_wait();
   if (threadIdx.x == 0) grid_dep_launch();
 
-  const int nk = p.num_kchunks;
+  const int nk = p.num_kchunks * p.a_planes;  // K chunks, over every plane of the image
   const int first_tile = kPair ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
   const int tile_stride = kPair ? (int)(gridDim.x >> 1) : (int)gridDim.x;
 
@@ -772,9 +784,13 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
           wp = jb.wp;
         }
         const CUtensorMap* wm = ti.bn == BN ? &tmap_w : &tmap_wh;
-        for (int q = 0; q < nk; ++q, ++it, s = (s + 1 == (uint32_t)S) ? 0 : s + 1, ph ^= (s == 0)) {
+        for (int q2 = 0; q2 < nk; ++q2, ++it, s = (s + 1 == (uint32_t)S) ? 0 : s + 1, ph ^= (s == 0)) {
           if ((int)(it % kTma) != tw) continue;
           if (!mbar_wait(b_empty + 8 * s, ph ^ 1, abort_flag)) { ok = false; break; }
+          // plane of the byte image (8-bit activations: x_lo, then 16 x_hi) and K chunk in it
+          const int plane = q2 >= p.num_kchunks ? 1 : 0;
+          const int q = q2 - plane * p.num_kchunks;
+          const int prow = plane * p.plane_rows;
           int r, sx, cb;
           if (q < kQTab) {
             const uint32_t e = qtab[q];
@@ -787,8 +803,8 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
           if constexpr (kPair) {
             // this CTA's 128 rows of A and its half of B; both CTAs' copies complete on the
             // leader's "full" barrier, which the leader arms with the bytes of all four
-            const int row = row0 + r * wp + sx;
-            const int brow = ti.col0 + (int)rank * (ti.bn / 2);
+            const int row = row0 + prow + r * wp + sx;
+            const int brow = ti.brow + (int)rank * (ti.bn / 2);
             const uint32_t b_bytes = (uint32_t)(ti.bn / 2) * BK;
             if (leader) {
               mbar_arrive_expect_tx(b_full + 8 * s, 2 * (b_bytes + kStageA));
@@ -802,14 +818,14 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
             continue;
           } else if constexpr (kFlat) {
             // A: 128 consecutive rows of the padded byte image, shifted by the tap (r, s)
-            const int row = row0 + r * wp + sx;
+            const int row = row0 + prow + r * wp + sx;
             mbar_arrive_expect_tx(b_full + 8 * s, (uint32_t)ti.bn * BK + kStageA);
             tma_load_2d(s_a + s * kStageA, &tmap_a, cb * BK, row, b_full + 8 * s);
           } else {
             (void)r; (void)sx; (void)cb;
             mbar_arrive_expect_tx(b_full + 8 * s, (uint32_t)ti.bn * BK);
           }
-          tma_load_2d(s_b + s * stage_b_bytes, wm, q * BK, ti.col0, b_full + 8 * s);
+          tma_load_2d(s_b + s * stage_b_bytes, wm, q * BK, ti.brow, b_full + 8 * s);
         }
       }
       if (!ok) fail(abort_flag, p.status);
@@ -905,7 +921,9 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       // (R-32) equals rhu(u * M0, R): the low product word cannot carry into the result)
       // and |bias| <= 2^30 (acc + bias cannot leave int32 when |acc| < 2^24).
       int fast_req = 1, small_bias = 1;
-      const int TBN = ti.bn;  // this tile's width
+      // this tile's output channels that exist (a last N tile may reach past cout; packed
+      // groups past it must not be written)
+      const int TBN = ti.cn < p.cout - ti.col0 ? ti.cn : p.cout - ti.col0;
       for (int col = et; col < 256; col += kEpiThreads) {
         const int ch = ti.col0 + col;
         EpiChan ec{};
@@ -939,7 +957,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
         fast_skip = named_bar_and(1, kEpiThreads, ok8);
       }
       // 0: general int64 epilogue; 1: fast requant to codes; 2: int32 output, no skip
-      const int mode = p.has_skip ? 0 : (out_bits == 32 ? 2 : (fast_req ? 1 : 0));
+      const int mode = (kSplit || p.has_skip) ? 0 : (out_bits == 32 ? 2 : (fast_req ? 1 : 0));
       const bool magic = p.acc_small && (mode == 2 ? small_bias : fast_req);
       const uint32_t buf = lt & 1;
       if (!mbar_wait(b_tfull + 8 * buf, (lt >> 1) & 1, abort_flag)) { ok = false; break; }
@@ -954,7 +972,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       uint32_t va[32], vn[32];
       __syncwarp();
       if (gi < nunits) {
-        tmem_ld32(tbuf + (gi / ngrp) * (uint32_t)BN + (gi % ngrp) * 32, TBN - (gi % ngrp) * 32 >= 32, va);
+        tmem_ld32(tbuf + (gi / ngrp) * (uint32_t)BN + (gi % ngrp) * 32, ti.cn - (gi % ngrp) * 32 >= 32, va);
         tmem_wait_ld();
         reg_fence32(va);
       }
@@ -963,12 +981,28 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
         // the next unit's TMEM load overlaps this unit's work in the light modes; the general /
         // skip mode (0) holds more registers and loads it afterwards
         if (un < nunits && mode != 0)
-          tmem_ld32(tbuf + (un / ngrp) * (uint32_t)BN + (un % ngrp) * 32, TBN - (un % ngrp) * 32 >= 32, vn);
+          tmem_ld32(tbuf + (un / ngrp) * (uint32_t)BN + (un % ngrp) * 32, ti.cn - (un % ngrp) * 32 >= 32, vn);
         const int sub = u0 / ngrp, g0 = (u0 % ngrp) * 32;
         const int ncols = (TBN - g0) < 32 ? (TBN - g0) : 32;
-        if (ncols < 32) {
+        // 32 TMEM columns were loaded when the tile's MMA width covers them (else 16)
+        const bool full = ti.cn - g0 >= 32;
+        if (!full) {
 #pragma unroll
           for (int i = 16; i < 32; ++i) va[i] = 0u;  // only the first 16 columns were loaded
+        }
+        if constexpr (kSplit) {
+          // split weights: va holds D1 (w_lo rows); D2 (w_hi rows) sits TBN columns on;
+          // the exact sum is D1 + 16 D2, each an integer x 2^-18 below 2^24
+          uint32_t vb[32];
+          tmem_ld32(tbuf + (uint32_t)ti.cn + g0, full, vb);
+          tmem_wait_ld();
+          reg_fence32(vb);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const int32_t d1 = __float2int_rn(__uint_as_float(va[i]) * 262144.0f);
+            const int32_t d2 = (full || i < 16) ? __float2int_rn(__uint_as_float(vb[i]) * 262144.0f) : 0;
+            va[i] = (uint32_t)(d1 + 16 * d2);
+          }
         }
         const uint32_t* v = va;
         int m;  // output pixel index within the job
@@ -1009,7 +1043,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
             if (kFlat && p.ws_out) chain_store(p, jb, oimg, oh, ow, ch0, gw, out_bits);
           } else if (mode == 2) {
             int32_t* yr = reinterpret_cast<int32_t*>(yrow) + ch0;
-            const bool full = ncols == 32 && ch0 + 32 <= p.cout;
+            const bool whole = ncols == 32 && ch0 + 32 <= p.cout;
   #pragma unroll
             for (int q = 0; q < 8; ++q) {
               int32_t o[4];
@@ -1019,7 +1053,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
                 o[k] = magic ? __float_as_int(__fmaf_rn(f, 262144.0f, kMagic)) + epf[g0 + 4 * q + k].x
                              : add_sat(__float2int_rn(f * 262144.0f), epi[g0 + 4 * q + k].bias);
               }
-              if (full) {
+              if (whole) {
                 reinterpret_cast<int4*>(yr)[q] = make_int4(o[0], o[1], o[2], o[3]);
               } else {
   #pragma unroll
@@ -1042,7 +1076,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
               load_skip_group(p, srow, ch0, ncols, oo);   // skip codes, replaced by the results
               fast_skip_group(v, epi + g0, oo, qmax, oo);
             } else {
-              general_group<kSkip>(p, v, epi + g0, srow, ch0, ncols, oo);
+              general_group<kSkip, kSplit>(p, v, epi + g0, srow, ch0, ncols, oo);
             }
             if (out_bits == 32) {
               int32_t* yr = reinterpret_cast<int32_t*>(yrow) + ch0;
@@ -1059,7 +1093,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
         }
         if (un < nunits) {
           if (mode == 0)
-            tmem_ld32(tbuf + (un / ngrp) * (uint32_t)BN + (un % ngrp) * 32, TBN - (un % ngrp) * 32 >= 32, vn);
+            tmem_ld32(tbuf + (un / ngrp) * (uint32_t)BN + (un % ngrp) * 32, ti.cn - (un % ngrp) * 32 >= 32, vn);
           tmem_wait_ld();
           reg_fence32(vn);
 #pragma unroll
@@ -1101,9 +1135,17 @@ struct ExpandArgs {
   ConvJobDev jobs[kMaxJobs];
   int32_t njobs, cin, pad;
   int64_t x_row_bytes;
-  int64_t total_rows;
+  int64_t total_rows;     // rows of one plane
   uint8_t* ws;
 };
+
+// E4M3 byte of the value 16 n * 2^-9 = n * 2^-5, n in [0, 15] (the raw byte n is n * 2^-9):
+// n = 2^e (1 + m/8) with 8-bit exponent field e + 2, packed as two 64-bit tables of 8 bytes.
+__device__ __forceinline__ uint32_t e4m3_times16(uint32_t n) {
+  constexpr uint64_t lo = 0x26242220'1C181000ull;  // n = 7 .. 0
+  constexpr uint64_t hi = 0x2F2E2D2C'2B2A2928ull;  // n = 15 .. 8
+  return (uint32_t)(((n < 8 ? lo : hi) >> (8 * (n & 7))) & 0xFFu);
+}
 
 // Position of one workspace row: its job, image, padded row / column and input pointer.
 struct ExpandPos {
@@ -1161,7 +1203,7 @@ __global__ void __launch_bounds__(256) expand_kernel(const __grid_constant__ Exp
   ExpandPos ps;
   int q = e0 % chunks;
   expand_locate(a, e0 / chunks, ps);
-  uint32_t w[kPerLane][kXBits == 2 ? 1 : 2];
+  uint32_t w[kPerLane][kXBits == 2 ? 1 : (kXBits == 8 ? 4 : 2)];
   uint8_t* dst[kPerLane];
   bool inside[kPerLane];
   int hsel[kPerLane];
@@ -1177,7 +1219,12 @@ __global__ void __launch_bounds__(256) expand_kernel(const __grid_constant__ Exp
     if (inside[i]) {
       const uint32_t* grp = reinterpret_cast<const uint32_t*>(
           jb.x + ((size_t)(ps.img * jb.h + hi) * jb.w + wi) * a.x_row_bytes + (q >> 1) * 4 * kXBits);
-      if constexpr (kXBits == 2) {
+      if constexpr (kXBits == 8) {
+        // 16 one-byte codes: channels 16 q .. 16 q + 15
+        const uint4 v = __ldg(reinterpret_cast<const uint4*>(jb.x + ((size_t)(ps.img * jb.h + hi) * jb.w + wi) *
+                                                             a.x_row_bytes) + q);
+        w[i][0] = v.x; w[i][1] = v.y; w[i][2] = v.z; w[i][3] = v.w;
+      } else if constexpr (kXBits == 2) {
         w[i][0] = __ldg(grp + (q & 1));
       } else if constexpr (kXBits == 4) {
         const uint2 v = __ldg(reinterpret_cast<const uint2*>(grp) + (q & 1));
@@ -1197,6 +1244,22 @@ __global__ void __launch_bounds__(256) expand_kernel(const __grid_constant__ Exp
   for (int i = 0; i < kPerLane; ++i) {
     if (!dst[i]) continue;
     uint32_t o[4] = {0u, 0u, 0u, 0u};
+    if constexpr (kXBits == 8) {
+      // plane 0: x_lo = x & 15 (raw byte); plane 1, total_rows rows on: 16 x_hi as E4M3
+      uint32_t o1[4] = {0u, 0u, 0u, 0u};
+      if (inside[i]) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          o[j] = w[i][j] & 0x0F0F0F0Fu;
+          const uint32_t hn = (w[i][j] >> 4) & 0x0F0F0F0Fu;
+          o1[j] = e4m3_times16(hn & 0xFFu) | (e4m3_times16((hn >> 8) & 0xFFu) << 8) |
+                  (e4m3_times16((hn >> 16) & 0xFFu) << 16) | (e4m3_times16(hn >> 24) << 24);
+        }
+      }
+      *reinterpret_cast<uint4*>(dst[i]) = make_uint4(o[0], o[1], o[2], o[3]);
+      *reinterpret_cast<uint4*>(dst[i] + (size_t)a.total_rows * a.cin) = make_uint4(o1[0], o1[1], o1[2], o1[3]);
+      continue;
+    }
     if (inside[i]) {
       const int h = hsel[i];
       if constexpr (kXBits == 2) {
@@ -1236,10 +1299,10 @@ static EncodeTiledFn get_encode_fn(std::string* err) {
   return fn;
 }
 
-template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair = false, bool kSkip = true>
+template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair = false, bool kSkip = true, bool kSplit = false>
 static int launch_bits(const Params& prm, const CUtensorMap& map, const CUtensorMap& map_h, const CUtensorMap& map_a,
                        int grid, size_t smem, cudaStream_t stream, std::string* err) {
-  auto kern = conv_tc_kernel<kXBits, kChunkInTap, kFlat, kPair, kSkip>;
+  auto kern = conv_tc_kernel<kXBits, kChunkInTap, kFlat, kPair, kSkip, kSplit>;
   // The opt-in limit is raised to the device maximum, never lowered to this call's size:
   // a CUDA graph node captured earlier with a larger plan must stay launchable (a graph
   // node, or a tool relaunching it, is checked against the function's current limit).
@@ -1284,9 +1347,11 @@ bool conv_tc_uses_pair(const ConvArgs& a) {
 int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   using namespace tc;
   Params prm{};
-  const int BN = a.bn;
+  // split (8-bit) weights: tiles of 256 weight rows = 128 output channels
+  const int BN = a.split_w ? 256 : a.bn;
+  const int w_rows = a.split_w ? a.split_rows : a.cout_pad;  // rows of the weight block
   prm.njobs = a.njobs;
-  prm.n_tiles = a.cout_pad / BN;
+  prm.n_tiles = w_rows / BN;
   // flat path: the activations are expanded into the workspace first (stride 1,
   // cin % 128 == 0; the API checks both before passing a workspace)
   const bool flat = a.ws != nullptr;
@@ -1328,7 +1393,7 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   const int rem = tiles % workers;
   prm.dp_tiles = tiles;
   // (a half tile must start on a 32-channel packing group: BN / 2 a multiple of 32)
-  if (BN % 64 == 0 && rem > 0 && 2 * rem <= workers) prm.dp_tiles = tiles - rem;
+  if (BN % 64 == 0 && !a.split_w && rem > 0 && 2 * rem <= workers) prm.dp_tiles = tiles - rem;
   prm.total_tiles = prm.dp_tiles + 2 * (tiles - prm.dp_tiles);
   prm.num_kchunks = a.k_pad / BK;
   prm.cin = a.cin; prm.cout = a.cout; prm.kh = a.kh; prm.kw = a.kw;
@@ -1343,6 +1408,9 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   prm.cin_chunks = a.cin / BK;
   prm.ws_out = a.ws_out;
   prm.out_pad = a.out_pad;
+  prm.a_planes = flat ? (a.a_planes > 1 ? a.a_planes : 1) : 1;
+  prm.plane_rows = (int32_t)rows;
+  prm.split_w = a.split_w;
   if (a.ws_out) {
     int64_t orows = 0;
     for (int j = 0; j < a.njobs; ++j) {
@@ -1382,7 +1450,7 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   EncodeTiledFn enc = get_encode_fn(err);
   if (!enc) return 3;
   CUtensorMap map;
-  cuuint64_t gdim[2] = {(cuuint64_t)a.k_pad, (cuuint64_t)a.cout_pad};
+  cuuint64_t gdim[2] = {(cuuint64_t)a.k_pad, (cuuint64_t)w_rows};
   cuuint64_t gstride[1] = {(cuuint64_t)a.k_pad};
   cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)b_rows};
   cuuint32_t estr[2] = {1, 1};
@@ -1430,6 +1498,7 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
         case 2: e = cudaLaunchKernelEx(&cfg, expand_kernel<2>, ea); break;
         case 3: e = cudaLaunchKernelEx(&cfg, expand_kernel<3>, ea); break;
         case 4: e = cudaLaunchKernelEx(&cfg, expand_kernel<4>, ea); break;
+        case 8: e = cudaLaunchKernelEx(&cfg, expand_kernel<8>, ea); break;
         default: *err = "conv_tc: activation bits must be 2, 3 or 4"; return 2;
       }
       if (e == cudaSuccess) e = cudaGetLastError();
@@ -1437,7 +1506,7 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
     }
     if (a.expand_only) return 0;
     // 2) tensor map over the workspace as a [rows][cin] byte matrix with 128 x 128 boxes
-    cuuint64_t gd[2] = {(cuuint64_t)a.cin, (cuuint64_t)rows};
+    cuuint64_t gd[2] = {(cuuint64_t)a.cin, (cuuint64_t)rows * (cuuint64_t)prm.a_planes};
     cuuint64_t gs[1] = {(cuuint64_t)a.cin};
     cuuint32_t bx[2] = {(cuuint32_t)BK, 128};
     CUresult r2 = enc(&map_a, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)a.ws, gd, gs, bx, estr,
@@ -1446,6 +1515,10 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
     if (r2 != CUDA_SUCCESS) {
       *err = "cuTensorMapEncodeTiled (activations) failed: " + std::to_string((int)r2);
       return 3;
+    }
+    if (a.split_w) {  // (no skip: the API keeps skips off the split form)
+      if (pair) return launch_bits<2, true, true, true, false, true>(prm, map, map_h, map_a, grid, smem, stream, err);
+      return launch_bits<2, true, true, false, false, true>(prm, map, map_h, map_a, grid, smem, stream, err);
     }
     if (pair)
       return a.has_skip ? launch_bits<2, true, true, true, true>(prm, map, map_h, map_a, grid, smem, stream, err)

@@ -157,13 +157,28 @@ unpack_kernel(const uint8_t* packed, int64_t rows, int c, int bits, int64_t row_
 __global__ void __launch_bounds__(kThreads)
 prepare_weights_kernel(const uint8_t* wp, int w_bits, int w_format, WeightGeom g, int64_t w_row_bytes,
                        int make_e4m3, uint8_t* out) {
+  // make_e4m3: 0 none (weights too wide for the tensor cores), 1 the plain layout, 2 the
+  // split layout of 8-bit two's-complement weights (per 128 channels: w_lo rows, w_hi rows)
   const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
-  const int64_t n_e4 = (int64_t)g.cout_pad * g.k_pad;
+  const int64_t e4_rows = make_e4m3 == 2 ? g.split_rows : g.cout_pad;
+  const int64_t n_e4 = e4_rows * g.k_pad;
   const int64_t n_i16 = (int64_t)g.cout * g.k_total;
   if (t >= n_e4 + n_i16) return;
   int64_t co, k;
-  if (t < n_e4) { co = t / g.k_pad; k = t - co * g.k_pad; }
-  else { co = (t - n_e4) / g.k_total; k = (t - n_e4) - co * g.k_total; }
+  int part = 0;  // split layout: 0 = w_lo, 1 = w_hi
+  if (t < n_e4) {
+    int64_t rr = t / g.k_pad;
+    k = t - rr * g.k_pad;
+    if (make_e4m3 == 2) {
+      const int64_t blk = rr / 256, within = rr - blk * 256;
+      part = (int)(within >> 7);
+      co = blk * 128 + (within & 127);
+    } else {
+      co = rr;
+    }
+  } else {
+    co = (t - n_e4) / g.k_total; k = (t - n_e4) - co * g.k_total;
+  }
   int32_t w = 0;
   if (co < g.cout && k < g.k_total) {
     const int64_t tap = k / g.cin;
@@ -176,6 +191,7 @@ prepare_weights_kernel(const uint8_t* wp, int w_bits, int w_format, WeightGeom g
     }
   }
   if (t < n_e4) {
+    if (make_e4m3 == 2) w = part == 0 ? (w & 15) : (w >> 4);  // w = 16 w_hi + w_lo, w_lo in [0, 15]
     if (make_e4m3) {
       const uint32_t mag = (uint32_t)(w < 0 ? -w : w);
       out[t] = (uint8_t)((w < 0 ? 0x80u : 0u) | (mag & 0x0Fu));
@@ -232,10 +248,12 @@ int launch_unpack(const uint8_t* packed, int64_t rows, int32_t c, int32_t bits, 
 
 int launch_prepare_weights(const uint8_t* w_packed, int32_t w_bits, int32_t w_format, const WeightGeom& g,
                            uint8_t* out, cudaStream_t stream, std::string* err) {
-  const int64_t total = (int64_t)g.cout_pad * g.k_pad + (int64_t)g.cout * g.k_total;
   const int max_abs = (w_format == 0) ? (1 << (w_bits - 1)) : ((1 << w_bits) - 1);
+  const int mode = max_abs <= 15 ? 1 : ((w_bits == 8 && w_format == 0) ? 2 : 0);
+  const int64_t e4_rows = mode == 2 ? g.split_rows : g.cout_pad;
+  const int64_t total = e4_rows * g.k_pad + (int64_t)g.cout * g.k_total;
   elt::prepare_weights_kernel<<<elt::blocks_for(total), elt::kThreads, 0, stream>>>(
-      w_packed, w_bits, w_format, g, row_bytes_of(g.cin, w_bits), max_abs <= 15 ? 1 : 0, out);
+      w_packed, w_bits, w_format, g, row_bytes_of(g.cin, w_bits), mode, out);
   return check_launch("prepare_weights launch", err);
 }
 

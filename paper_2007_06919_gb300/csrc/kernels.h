@@ -51,6 +51,12 @@ struct ConvArgs {
   int32_t skip_expand;    // workspace already holds the expansion: launch only the conv
   int32_t expand_only;    // launch only the expansion into the workspace
   int32_t no_pair;        // workspace path: use the one-CTA kernel even for 256-wide N tiles
+  // 8-bit operands on the tensor cores (workspace path): activations as two planes of
+  // 4-bit halves (x_lo, 16 x_hi) over which K runs twice; weights, when wider than 15, as
+  // two row blocks per 128 output channels (w_lo, w_hi) whose accumulators combine as D1 + 16 D2
+  int32_t a_planes;       // 1, or 2 for 8-bit activation codes
+  int32_t split_w;        // weights in the split layout
+  int32_t split_rows;     // weight rows of that layout (2 * round_up(cout, 128))
   uint8_t* ws_out;        // chained output: also write the output codes as the next conv's byte image
   int32_t out_pad;        // padding of that next conv
   uint32_t* status;       // device status word
@@ -60,6 +66,7 @@ struct ConvArgs {
 struct WeightGeom {
   int32_t cout, kh, kw, cin;
   int32_t k_total, k_pad, bn, cout_pad;
+  int32_t split_rows;     // 2 * round_up(cout, 128): rows of the split (8-bit) weight layout
   size_t e4m3_bytes, i16_offset, total_bytes;
 };
 WeightGeom weight_geom(int32_t cout, int32_t kh, int32_t kw, int32_t cin);

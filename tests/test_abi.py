@@ -104,8 +104,10 @@ def test_invalid_arguments_return_before_launch(lib):
 
 
 def test_workspace_bytes_host_logic(lib):
-    """The expanded-activation workspace is sum(n * (h+2p) * (w+2p)) * cin bytes for stride-1
-    convolutions with cin % 128 == 0 and codes/weights of at most 4 bits, else 0."""
+    """The expanded-activation workspace is planes * sum(n * (h+2p) * (w+2p)) * cin bytes for
+    stride-1 convolutions with cin % 128 == 0 (planes = 2 for 8-bit activation codes; 8-bit
+    two's-complement weights take the split form), else 0; 8-bit operands also need
+    K * 3825 < 2^24 (the exact FP32 partial sums)."""
     from paper_2007_06919_gb300 import aqd
     jobs = (aqd._Job * 2)()
     jobs[0].x = aqd._Tensor(2, 10, 17, 256, 2, 256)
@@ -115,7 +117,16 @@ def test_workspace_bytes_host_logic(lib):
     assert lib.aqd_conv_workspace_bytes(jobs, 2, ctypes.byref(w), 1, 1) == want
     assert lib.aqd_conv_workspace_bytes(jobs, 2, ctypes.byref(w), 2, 1) == 0      # stride 2
     w8 = aqd._Weights(256, 256, 3, 3, 256, 8, 0)
-    assert lib.aqd_conv_workspace_bytes(jobs, 2, ctypes.byref(w8), 1, 1) == 0     # 8-bit weights
+    assert lib.aqd_conv_workspace_bytes(jobs, 2, ctypes.byref(w8), 1, 1) == want  # 8-bit weights: split
+    w8odd = aqd._Weights(256, 256, 3, 3, 256, 8, 1)
+    assert lib.aqd_conv_workspace_bytes(jobs, 2, ctypes.byref(w8odd), 1, 1) == 0  # odd grid, 8-bit
+    jobs8 = (aqd._Job * 2)()
+    jobs8[0].x = aqd._Tensor(2, 10, 17, 256, 8, 256)
+    jobs8[1].x = aqd._Tensor(2, 5, 9, 256, 8, 256)
+    assert lib.aqd_conv_workspace_bytes(jobs8, 2, ctypes.byref(w8), 1, 1) == 2 * want  # two planes
+    wbig = aqd._Weights(256, 256, 3, 3, 2048, 8, 0)  # K = 18432: 18432 * 3825 >= 2^24
+    jobs8[0].x = aqd._Tensor(2, 10, 17, 2048, 8, 256)
+    assert lib.aqd_conv_workspace_bytes(jobs8, 1, ctypes.byref(wbig), 1, 1) == 0
     w64 = aqd._Weights(256, 64, 3, 3, 64, 2, 0)
     jobs[0].x = aqd._Tensor(2, 10, 17, 64, 2, 256)
     assert lib.aqd_conv_workspace_bytes(jobs, 1, ctypes.byref(w64), 1, 1) == 0    # cin 64

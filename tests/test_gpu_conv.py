@@ -242,3 +242,44 @@ def test_first_conv_full_size_sampled():
 def oracle_unpack(packed, c, bits):
     import oracle
     return oracle.unpack(packed, c, bits)
+
+
+# (x_bits, w_bits, n, h, w, cin, cout, out_bits): 8-bit operands on the tensor cores, split
+# into 4-bit halves (activation planes x_lo, 16 x_hi; weight rows w_lo, w_hi)
+WIDE_CASES = [
+    (8, 4, 2, 11, 13, 128, 64, 4),     # 8-bit activations, 4-bit weights: two planes
+    (8, 8, 1, 9, 17, 256, 256, 8),     # both 8-bit: two planes, split weights
+    (2, 8, 2, 7, 9, 128, 96, 2),       # 8-bit weights only
+    (4, 8, 1, 12, 10, 256, 80, 32),    # int32 output
+    (8, 8, 3, 5, 6, 128, 384, 4),      # three 128-channel output blocks
+]
+
+
+@pytest.mark.parametrize("case", WIDE_CASES, ids=[str(i) for i in range(len(WIDE_CASES))])
+@pytest.mark.parametrize("pairs", [True, False])
+def test_wide_operands_on_tensor_cores_bit_exact(case, pairs):
+    xb, wb, n, h, wd, cin, cout, ob = case
+    rng = np.random.default_rng(hash(case) % 2 ** 32 + 7)
+    x = synth.act_codes(rng, (n, h, wd, cin), xb)
+    w = rng.integers(-(1 << (wb - 1)), 1 << (wb - 1), size=(cout, 3, 3, cin)).astype(np.int32)
+    std = np.sqrt(9 * cin * np.mean(np.arange(1 << xb) ** 2) * (1 << (2 * wb - 2)) / 3)
+    m0, sh, b = _params(rng, 1, cout, ob if ob != 32 else 4, calib_std=std)
+    got, want, used = conv_pair(x, xb, w, wb, out_bits=ob, m0=m0, shift=sh, bias=b,
+                                path=TC if pairs else TC_NO_PAIR, workspace=True)
+    assert used == (4 if pairs else 3)
+    assert_same(got, want, cout, ob, f"wide case {case}")
+
+
+def test_wide_operands_exact_at_the_bound():
+    """Every code 255 and every weight -128 or 127 (signs mixed per channel), K = 3456 (the
+    FP32 partial sums D1 <= 3825 K stay below 2^24): int32 outputs equal the oracle's."""
+    cin = 384
+    x = np.full((1, 4, 5, cin), 255, np.int32)
+    w = np.full((64, 3, 3, cin), -128, np.int32)
+    w[1::2] = 127
+    w[3, :, :, ::2] = -1
+    got, want, used = conv_pair(x, 8, w, 8, pad=1, out_bits=32, bias=np.zeros((1, 64), np.int32), path=TC,
+                                workspace=True)
+    assert used == 4
+    assert_same(got, want, 64, 32, "wide exactness")
+    assert np.abs(want.view(np.int32)).max() > (1 << 26)

@@ -37,7 +37,7 @@ METRIC = "int-only conv TOPS & % of INT8 tensor peak; detector-head images/s at 
 # DRAM bytes (read + write) of one workspace-fed tower-layer conv_tc launch, taken from an
 # ncu capture of this kernel on this workload (dram__bytes_read.sum + dram__bytes_write.sum).
 # Re-measure (or set to None) whenever conv_tc_kernel changes.
-TOWER_CONV_DRAM_BYTES = 12_691_200
+TOWER_CONV_DRAM_BYTES = 12_692_480
 KREP = 16  # tower-layer convs per timed kernel graph (16 x 12 MB workspaces > 129 MB L2)
 WORKLOAD = "retina_head_800x1333_b2_2bit"
 
@@ -309,6 +309,35 @@ def run_sweep(args):
         ms = timed(fn)
         emit(f"config1_part_{nm}", ms, o, 0)
 
+    # config 3: the whole integer detector (ResNet-18 + FPN + head), batch 8, 800x1344, 4-bit
+    if want in ("all", "config3"):
+        from paper_2007_06919_gb300.detector import IntDetector
+        wl = synth.config3()
+        nb, (hh, ww) = wl.extra["batch"], wl.extra["hw"]
+        with torch.cuda.stream(stream):
+            net = IntDetector(wl.extra["layers"], (nb, hh, ww, 3, 8), device=dev)
+            img = aqd.DTensor.from_codes(torch.from_numpy(wl.inputs[0]).to(dev), 8)
+            net.tensors["image"].data.copy_(img.data)
+        stream.synchronize()
+        ms = timed(lambda: net.forward(stream=stream))
+        emit("config3_int_resnet18_fpn_retina_b8_800x1344_4bit", ms, net.ops, 0, images_per_s=nb / (ms * 1e-3),
+             launches=net.launches)
+        for kind, p in net.steps:
+            ly = p if kind == "pool" else p.layer
+            one = IntDetector.__new__(IntDetector)
+            one.__dict__.update(net.__dict__)
+            one.steps = [(kind, p)]
+            ops = 0
+            if kind == "conv":
+                cv = ly.conv
+                for x, y, _, _ in p.jobs:
+                    ops += 2 * y.n * y.h * y.w * cv.cout * cv.kh * cv.kw * cv.cin
+            ms = timed(lambda: one.forward(stream=stream))
+            emit(f"config3_layer_{ly.name}", ms, ops, 0,
+                 path=("chain" if p.chain_to is not None else "image" if p.reads_image else
+                       "workspace" if p.ws_bytes else "no workspace") if kind == "conv" else "pool",
+                 last_path=aqd.last_conv_path() if kind == "conv" else None)
+
     # config 4: first tower layer of the head at batch 16, 2/3/4/8-bit
     for bits in ((2, 3, 4, 8) if want in ("all", "config4") else ()):
         wl = synth.config4(bits)
@@ -346,7 +375,7 @@ def main():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--sweep", nargs="?", const="all", default=None, choices=["all", "config0", "config1", "config4"],
+    ap.add_argument("--sweep", nargs="?", const="all", default=None, choices=["all", "config0", "config1", "config3", "config4"],
                     help="measure the other workloads (several lines)")
     args = ap.parse_args()
     if args.impl == "reference":

@@ -272,3 +272,27 @@ def maxpool(x: CodeTensor, k: int, stride: int, pad: int) -> CodeTensor:
     yt = _tensor(y, x.n, ho, wo, x.c, x.bits)
     _check(lib().aqd_ref_maxpool_codes(ctypes.byref(x.ct()), k, stride, pad, ctypes.byref(yt)), "maxpool")
     return CodeTensor(y, x.n, ho, wo, x.c, x.bits)
+
+
+def run_network(layers, tensors: dict) -> dict:
+    """Runs a layer list (convs and max-pools naming their input, output and skip tensors)
+    on the oracle, in list order. ``tensors`` maps names to CodeTensors and receives every
+    layer output. A conv with several jobs (the shared head) takes parameter row l for job l
+    (multi-level BN, Sec. 3.2.2); each job is one plain oracle convolution (Eq. 4 -> Eq. 6 ->
+    Eq. 7 -> Eq. 2); a max-pool compares codes (Sec. 3.2.4)."""
+    for ly in layers:
+        if ly.pool is not None:
+            k, s, p = ly.pool
+            tensors[ly.dst[0]] = maxpool(tensors[ly.src[0]], k, s, p)
+            continue
+        cv = ly.conv
+        wp = pack(cv.w.reshape(-1, cv.cin), cv.w_bits)
+        ref = cv.m0 if cv.m0 is not None else cv.bias
+        levels = ref.shape[0]
+        for j, (src, dst) in enumerate(zip(ly.src, ly.dst)):
+            skip = tensors[ly.skip[j]] if ly.skip else None
+            tensors[dst] = conv_int(tensors[src], wp, cv.w_bits, W_TWOS, cv.kh, cv.kw, cv.stride, cv.pad,
+                                    cv.cout, level=j, m0=cv.m0, shift=cv.shift, bias=cv.bias, levels=levels,
+                                    skip=skip, skip_c=cv.skip_c, skip_d=cv.skip_d, upsample=ly.upsample,
+                                    out_bits=cv.out_bits)
+    return tensors

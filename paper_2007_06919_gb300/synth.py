@@ -171,3 +171,121 @@ def sample_pixels(rng, total: int, n: int) -> np.ndarray:
     if n > 1:
         idx[1] = total - 1
     return np.unique(idx)
+
+
+# ------------------------------------------------------------------ config 3: whole network
+
+# second moments of the drawn distributions, for the calibrated shifts below
+_EX2_CODE4 = 16.0                     # |N(0,4)| clipped to [0, 15]: E[x^2] ~ 16
+_EX2_CODE8 = sum(v * v for v in range(256)) / 256.0   # uniform 8-bit image codes
+_EW2_NORMAL2 = 4.0                    # N(0, 2) clipped to [-7, 7]: E[w^2] ~ 4
+
+
+def skip_params_acc(rng, levels: int, cout: int):
+    """Rescale c/2^d of an int32 skip held in another conv's accumulator units (a downsample
+    branch): c uniform in [2^30, 2^31), d = 31 + delta with delta uniform in {0, 1, 2}, so the
+    branch enters the sum at 1/8 to 1 times its own value."""
+    c = rng.integers(1 << 30, 1 << 31, size=(levels, cout), dtype=np.int64).astype(np.int32)
+    d = (31 + rng.integers(0, 3, size=(levels, cout))).astype(np.int8)
+    return c, d
+
+
+@dataclass
+class Layer:
+    """One step of a network: a conv (``conv`` set) or a max-pool on codes (``pool`` set).
+    ``src``, ``dst`` and ``skip`` name tensors, one entry per job; a grouped layer (the shared
+    head) has one job per FPN level, and job l uses row l of the per-level tables. ``upsample``
+    2 reads the skip at half resolution (nearest 2x, the FPN top-down add)."""
+    name: str
+    src: list
+    dst: list
+    conv: ConvSpec | None = None
+    skip: list | None = None
+    upsample: int = 1
+    pool: tuple | None = None     # (k, stride, pad)
+
+
+def _conv(rng, cin, cout, k, stride, pad, *, levels=1, out_bits=4, x_ex2=_EX2_CODE4, w_bits=4,
+          skip="none", skip_levels=None):
+    """Draws one conv in the fixed order: weights, M0, shift, bias, then the skip's (c, d).
+    Codes out: requant calibrated from the accumulator's standard deviation. int32 out: bias only."""
+    wt = weight_codes(rng, (cout, k, k, cin), 4, "normal2")
+    std = math.sqrt(k * k * cin * x_ex2 * _EW2_NORMAL2)
+    if out_bits == 32:
+        lim = max(1, int(std))
+        bias = rng.integers(-lim, lim + 1, size=(levels, cout), dtype=np.int64).astype(np.int32)
+        cv = ConvSpec(cin, cout, k, k, stride, pad, wt, w_bits, None, None, bias, 32)
+    else:
+        m0, shift, bias = requant_params(rng, levels, cout, calib_std=std, out_bits=out_bits)
+        cv = ConvSpec(cin, cout, k, k, stride, pad, wt, w_bits, m0, shift, bias, out_bits)
+    if skip == "codes":
+        cv.skip_c, cv.skip_d = skip_params(rng, levels, cout, cv.shift)
+    elif skip == "acc":
+        cv.skip_c, cv.skip_d = skip_params_acc(rng, levels, cout)
+    return cv
+
+
+def config3(seed: int = 3, batch: int = 8, h: int = 800, w: int = 1333, w_pad: int = 1344) -> Workload:
+    """Integer ResNet-18 backbone + FPN (P3-P7, 256 channels) + the shared head of config 2,
+    4-bit weights (N(0,2) rounded, clipped to [-7, 7]) and 4-bit activations; the input is an
+    8-bit RGB image batch (codes uniform in [0, 255]) zero-padded on the right from w to w_pad
+    columns. Every conv's requant is calibrated so that activations stay spread over the code
+    range through the depth of the network.
+
+    Layers (NHWC, codes unless stated):
+    - conv1 7x7 s2 p3 3->64 (8-bit input; weights held as 8-bit codes since a 3-channel row has
+      no 4-bit packed layout), max-pool 3x3 s2 p1;
+    - four stages of two basic blocks (64, 128, 256, 512 channels; stages 2-4 start with a 3x3 s2
+      conv and a 1x1 s2 downsample conv whose int32 output is the block's skip, Eq. 7 with
+      an accumulator-domain operand); identity skips are the block input's codes;
+    - FPN: 1x1 lateral convs on C3, C4, C5; the top-down path adds the coarser merged map,
+      read with nearest 2x upsampling, in the lateral conv's epilogue (Eq. 7); 3x3 output convs
+      give P3-P5; P6 = 3x3 s2 on C5, P7 = 3x3 s2 on P6;
+    - head: 4 x [3x3 256->256] over P3-P7 with per-level (M0, shift, bias) (Sec. 3.2.2), then
+      3x3 256->80 classification and 3x3 256->4 box convs with int32 outputs.
+    """
+    rng = np.random.default_rng(seed)
+    x = np.zeros((batch, h, w_pad, 3), dtype=np.int32)
+    x[:, :, :w] = act_codes(rng, (batch, h, w, 3), 8)
+    layers: list[Layer] = []
+    c1 = _conv(rng, 3, 64, 7, 2, 3, x_ex2=_EX2_CODE8, w_bits=8)
+    layers.append(Layer("conv1", ["image"], ["conv1"], conv=c1))
+    layers.append(Layer("pool", ["conv1"], ["pool"], pool=(3, 2, 1)))
+    cur, cin = "pool", 64
+    for stage, cout in enumerate((64, 128, 256, 512), start=1):
+        for blk in range(2):
+            down = stage > 1 and blk == 0
+            pre = f"layer{stage}.{blk}"
+            a = _conv(rng, cin, cout, 3, 2 if down else 1, 1)
+            layers.append(Layer(pre + ".conv_a", [cur], [pre + ".a"], conv=a))
+            if down:
+                ds = _conv(rng, cin, cout, 1, 2, 0, out_bits=32)
+                layers.append(Layer(pre + ".down", [cur], [pre + ".down"], conv=ds))
+                b = _conv(rng, cout, cout, 3, 1, 1, skip="acc")
+                layers.append(Layer(pre + ".conv_b", [pre + ".a"], [pre], conv=b, skip=[pre + ".down"]))
+            else:
+                b = _conv(rng, cout, cout, 3, 1, 1, skip="codes")
+                layers.append(Layer(pre + ".conv_b", [pre + ".a"], [pre], conv=b, skip=[cur]))
+            cur, cin = pre, cout
+    c3, c4, c5 = "layer2.1", "layer3.1", "layer4.1"
+    layers.append(Layer("fpn.lat5", [c5], ["fpn.m5"], conv=_conv(rng, 512, 256, 1, 1, 0)))
+    layers.append(Layer("fpn.lat4", [c4], ["fpn.m4"], conv=_conv(rng, 256, 256, 1, 1, 0, skip="codes"),
+                        skip=["fpn.m5"], upsample=2))
+    layers.append(Layer("fpn.lat3", [c3], ["fpn.m3"], conv=_conv(rng, 128, 256, 1, 1, 0, skip="codes"),
+                        skip=["fpn.m4"], upsample=2))
+    for l in (3, 4, 5):
+        layers.append(Layer(f"fpn.out{l}", [f"fpn.m{l}"], [f"P{l}"], conv=_conv(rng, 256, 256, 3, 1, 1)))
+    layers.append(Layer("fpn.p6", [c5], ["P6"], conv=_conv(rng, 512, 256, 3, 2, 1)))
+    layers.append(Layer("fpn.p7", ["P6"], ["P7"], conv=_conv(rng, 256, 256, 3, 2, 1)))
+    src = [f"P{l}" for l in range(3, 8)]
+    for i in range(4):
+        dst = [f"head.t{i}.{l}" for l in range(5)]
+        layers.append(Layer(f"head.tower{i}", src, dst, conv=_conv(rng, 256, 256, 3, 1, 1, levels=5)))
+        src = dst
+    layers.append(Layer("head.cls", src, [f"cls.{l}" for l in range(5)],
+                        conv=_conv(rng, 256, 80, 3, 1, 1, levels=5, out_bits=32)))
+    layers.append(Layer("head.box", src, [f"box.{l}" for l in range(5)],
+                        conv=_conv(rng, 256, 4, 3, 1, 1, levels=5, out_bits=32)))
+    name = f"int_resnet18_fpn_retina_b{batch}_{h}x{w_pad}_4bit"
+    return Workload(name, 4, [x], [ly.conv for ly in layers if ly.conv is not None],
+                    {"layers": layers, "batch": batch, "hw": (h, w_pad), "input_bits": 8})

@@ -137,7 +137,9 @@ aqd_status aqd_device_status(aqd_stream_t stream, int32_t* code);
  * pairs); returns the previous setting, or -1 for an unknown value. aqd_last_conv_path()
  * reports the kernel the calling thread's last successful conv call used (1 tensor core
  * unpacking in-kernel, 2 CUDA core, 3 tensor core fed from the expanded workspace, 4 the
- * same on CTA pairs sharing each weight tile, 0 none yet). */
+ * same on CTA pairs sharing each weight tile, 5 the F16 tensor-core kernel of a network's
+ * first conv on a 3-channel 8-bit image with a 7x7 kernel, 0 none yet). Forcing 2 also
+ * turns path 5 off. */
 int32_t aqd_set_conv_path(int32_t path);
 int32_t aqd_last_conv_path(void);
 

@@ -403,7 +403,9 @@ static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aq
     const int64_t rows = flat_rows(jobs, njobs, w, stride, pad, &wide_planes);
     wide_ok = rows > 0 && (size_t)rows * (size_t)wide_planes * (size_t)w->cin <= ws_bytes;
   }
-  int path = (tc_ok || wide_ok) ? 1 : 2;
+  // the network's first conv (3-channel 8-bit image, 7x7): its own F16 tensor-core kernel
+  const bool stem_ok = !tc_ok && !wide_ok && stage == kStageBoth && stem_applicable(a);
+  int path = (tc_ok || wide_ok) ? 1 : (stem_ok ? 5 : 2);
   if ((g_forced_path == 1 || g_forced_path == 3) && (tc_ok || wide_ok)) path = 1;
   a.no_pair = g_forced_path == 3 ? 1 : 0;
   if (g_forced_path == 2) path = 2;
@@ -450,7 +452,7 @@ static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aq
   }
   a.expand_only = stage == kStageExpandOnly ? 1 : 0;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  int rc = path == 1 ? launch_conv_tc(a, st, &err) : launch_conv_direct(a, st, &err);
+  int rc = path == 1 ? launch_conv_tc(a, st, &err) : path == 5 ? launch_stem(a, st, &err) : launch_conv_direct(a, st, &err);
   if (rc) return fail((aqd_status)rc, err);
   if (stage != kStageExpandOnly)
     g_last_path = (path == 1 && a.ws) ? (conv_tc_uses_pair(a) ? 4 : 3) : path;

@@ -76,6 +76,9 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err);
 // whether launch_conv_tc runs these arguments on CTA pairs (cta_group::2)
 bool conv_tc_uses_pair(const ConvArgs& a);
 int launch_conv_direct(const ConvArgs& a, cudaStream_t stream, std::string* err);
+// the first conv of the network (3-channel 8-bit image, 7x7 kernel) on F16 tensor cores
+bool stem_applicable(const ConvArgs& a);
+int launch_stem(const ConvArgs& a, cudaStream_t stream, std::string* err);
 int launch_prepare_weights(const uint8_t* w_packed, int32_t w_bits, int32_t w_format,
                            const WeightGeom& g, uint8_t* out, cudaStream_t stream,
                            std::string* err);

@@ -196,21 +196,64 @@ def test_invalid_skip_shape_is_rejected_before_launch():
     torch.cuda.synchronize()
 
 
+STEM = 5
+
+
 @pytest.mark.parametrize("shape", [(1, 37, 53), (2, 24, 40)])
-def test_first_conv_8bit_rgb_7x7_s2_bit_exact(shape):
+@pytest.mark.parametrize("path", [0, DIRECT])
+def test_first_conv_8bit_rgb_7x7_s2_bit_exact(shape, path):
     """The network's first conv (config 3): 8-bit unsigned image codes with 3 channels,
     7x7 stride 2 padding 3, 4-bit weight values (stored as 8-bit codes: a 3-channel row has
-    no 4-bit packed layout), 64 channels of 4-bit codes out."""
+    no 4-bit packed layout), 64 channels of 4-bit codes out. The automatic choice is the F16
+    tensor-core stem kernel; forcing path 2 runs the exact int32 CUDA-core kernel."""
     n, h, wd = shape
     rng = np.random.default_rng(h * 1000 + wd)
     x = synth.act_codes(rng, (n, h, wd, 3), 8)
     w = synth.weight_codes(rng, (64, 7, 7, 3), 4, "normal2")
     std = np.sqrt(147 * np.mean(np.arange(256) ** 2) * 4.0)
     m0, sh, b = _params(rng, 1, 64, 4, calib_std=std)
-    got, want, used = conv_pair(x, 8, w, 8, stride=2, pad=3, out_bits=4, m0=m0, shift=sh, bias=b, path=0)
-    assert used == DIRECT  # 8-bit codes and cin 3 take the exact int32 CUDA-core kernel
+    got, want, used = conv_pair(x, 8, w, 8, stride=2, pad=3, out_bits=4, m0=m0, shift=sh, bias=b, path=path)
+    assert used == (STEM if path == 0 else DIRECT)
     assert_same(got, want, 64, 4, f"first conv {shape}")
     assert len(np.unique(oracle_unpack(want, 64, 4))) > 4
+
+
+# (n, h, w, cout, out_bits, stride, pad, levels, level, w_lim, calibrated): the stem kernel's
+# output widths, channel counts (one and several 32-column groups, a 16-column tail with
+# int32 out), geometries whose receptive fields leave the image on every side, a tile count
+# that is not a multiple of the SM count, per-level tables, 7-bit weights, and requant shifts
+# that force the int64 epilogue
+STEM_CASES = [
+    (1, 29, 31, 64, 2, 2, 3, 1, 0, 7, True),
+    (2, 17, 45, 32, 3, 1, 3, 1, 0, 7, True),
+    (1, 40, 40, 96, 8, 2, 0, 3, 2, 7, True),
+    (3, 23, 19, 48, 32, 2, 3, 1, 0, 7, True),
+    (1, 64, 90, 256, 4, 2, 3, 2, 1, 21, True),
+    (1, 16, 16, 64, 4, 1, 1, 1, 0, 7, False),
+    (1, 7, 7, 16, 32, 1, 0, 1, 0, 7, True),
+]
+
+
+@pytest.mark.parametrize("case", STEM_CASES, ids=[str(i) for i in range(len(STEM_CASES))])
+def test_stem_kernel_bit_exact(case):
+    n, h, wd, cout, out_bits, stride, pad, levels, level, w_lim, calibrated = case
+    rng = np.random.default_rng(1000 + h * wd + cout)
+    x = synth.act_codes(rng, (n, h, wd, 3), 8)
+    w = rng.integers(-w_lim, w_lim + 1, size=(cout, 7, 7, 3)).astype(np.int32)
+    std = np.sqrt(147 * np.mean(np.arange(256) ** 2) * np.mean(np.arange(-w_lim, w_lim + 1) ** 2))
+    if out_bits == 32:
+        m0 = sh = None
+        b = rng.integers(-5000, 5000, size=(levels, cout)).astype(np.int32)
+    elif calibrated:
+        m0, sh, b = _params(rng, levels, cout, out_bits, calib_std=std)
+    else:
+        m0, sh, b = _params(rng, levels, cout, out_bits)
+        sh[:, ::3] = 1  # R = 32: outside the 32-bit fast form
+        sh[:, 1::5] = -4
+    got, want, used = conv_pair(x, 8, w, 8, stride=stride, pad=pad, out_bits=out_bits, m0=m0, shift=sh, bias=b,
+                                level=level)
+    assert used == STEM
+    assert_same(got, want, cout, out_bits, f"stem {case}")
 
 
 def test_first_conv_full_size_sampled():

@@ -118,6 +118,69 @@ __global__ void __launch_bounds__(kThreads) maxpool_kernel(const PoolArgs a) {
   store_vals(a.y + pix * a.row_bytes, a.bits, a.c, ch0, best);
 }
 
+// Max-pool on packed codes of 2, 4 or 8 bits (Sec. 3.2.4: max-pooling commutes with the
+// monotone quantizer, so it runs on the codes). In these layouts every byte holds 8/bits
+// codes at bit offsets 0, bits, 2 bits, ..., each of a different channel, so the per-channel
+// maximum is a byte-wise maximum (__vmaxu4) of each bit plane. One thread owns kVec words of
+// one output pixel's row; window taps outside the input are skipped (codes are >= 0 and the
+// padding is smaller than the window, so every window holds a tap).
+template <int kBits, int kVec>
+__global__ void __launch_bounds__(kThreads) maxpool_packed_kernel(const PoolArgs a) {
+  constexpr int kPlanes = 8 / kBits;
+  constexpr uint32_t kMask = kBits == 8 ? 0xFFFFFFFFu : (kBits == 4 ? 0x0F0F0F0Fu : 0x03030303u);
+  const int64_t units = a.row_bytes / (4 * kVec);
+  const int64_t total = (int64_t)a.n * a.ho * a.wo * units;
+  const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  if (t >= total) return;
+  const int64_t pix = t / units;
+  const int u = (int)(t - pix * units);
+  const int hw = a.ho * a.wo;
+  const int img = (int)(pix / hw);
+  const int rem = (int)(pix - (int64_t)img * hw);
+  const int oh = rem / a.wo, ow = rem - oh * a.wo;
+  uint32_t acc[kVec][kPlanes];
+#pragma unroll
+  for (int v = 0; v < kVec; ++v)
+#pragma unroll
+    for (int j = 0; j < kPlanes; ++j) acc[v][j] = 0u;
+  for (int r = 0; r < a.k; ++r) {
+    const int hi = oh * a.stride - a.pad + r;
+    if (hi < 0 || hi >= a.h) continue;
+    for (int s = 0; s < a.k; ++s) {
+      const int wi = ow * a.stride - a.pad + s;
+      if (wi < 0 || wi >= a.w) continue;
+      const uint32_t* src = reinterpret_cast<const uint32_t*>(
+          a.x + (((int64_t)img * a.h + hi) * a.w + wi) * a.row_bytes) + u * kVec;
+      uint32_t w[kVec];
+      if constexpr (kVec == 4) {
+        const uint4 q = __ldg(reinterpret_cast<const uint4*>(src));
+        w[0] = q.x; w[1] = q.y; w[2] = q.z; w[3] = q.w;
+      } else {
+#pragma unroll
+        for (int v = 0; v < kVec; ++v) w[v] = __ldg(src + v);
+      }
+#pragma unroll
+      for (int v = 0; v < kVec; ++v)
+#pragma unroll
+        for (int j = 0; j < kPlanes; ++j) acc[v][j] = __vmaxu4(acc[v][j], (w[v] >> (kBits * j)) & kMask);
+    }
+  }
+  uint32_t o[kVec];
+#pragma unroll
+  for (int v = 0; v < kVec; ++v) {
+    o[v] = 0u;
+#pragma unroll
+    for (int j = 0; j < kPlanes; ++j) o[v] |= acc[v][j] << (kBits * j);
+  }
+  uint32_t* dst = reinterpret_cast<uint32_t*>(a.y + pix * a.row_bytes) + u * kVec;
+  if constexpr (kVec == 4) {
+    *reinterpret_cast<uint4*>(dst) = make_uint4(o[0], o[1], o[2], o[3]);
+  } else {
+#pragma unroll
+    for (int v = 0; v < kVec; ++v) dst[v] = o[v];
+  }
+}
+
 __global__ void __launch_bounds__(kThreads)
 pack_kernel(const int32_t* codes, int64_t rows, int c, int bits, int64_t row_bytes, uint8_t* out) {
   const int groups = (c + 31) / 32;
@@ -222,8 +285,26 @@ int launch_elementwise(const EltArgs& a, cudaStream_t stream, std::string* err) 
 }
 
 int launch_maxpool(const PoolArgs& a, cudaStream_t stream, std::string* err) {
-  const int64_t total = (int64_t)a.n * a.ho * a.wo * ((a.c + 31) / 32);
-  if (total == 0) return 0;
+  const int64_t pixels = (int64_t)a.n * a.ho * a.wo;
+  if (pixels == 0) return 0;
+  // packed 2/4/8-bit rows: bit-plane maxima on whole words (16-byte units when the row allows)
+  if ((a.bits == 2 || a.bits == 4 || a.bits == 8) && a.row_bytes % 4 == 0) {
+    const bool v4 = a.row_bytes % 16 == 0;
+    const int64_t total = pixels * (a.row_bytes / (v4 ? 16 : 4));
+    const int blocks = elt::blocks_for(total);
+    if (a.bits == 2) {
+      if (v4) elt::maxpool_packed_kernel<2, 4><<<blocks, elt::kThreads, 0, stream>>>(a);
+      else elt::maxpool_packed_kernel<2, 1><<<blocks, elt::kThreads, 0, stream>>>(a);
+    } else if (a.bits == 4) {
+      if (v4) elt::maxpool_packed_kernel<4, 4><<<blocks, elt::kThreads, 0, stream>>>(a);
+      else elt::maxpool_packed_kernel<4, 1><<<blocks, elt::kThreads, 0, stream>>>(a);
+    } else {
+      if (v4) elt::maxpool_packed_kernel<8, 4><<<blocks, elt::kThreads, 0, stream>>>(a);
+      else elt::maxpool_packed_kernel<8, 1><<<blocks, elt::kThreads, 0, stream>>>(a);
+    }
+    return check_launch("maxpool launch", err);
+  }
+  const int64_t total = pixels * ((a.c + 31) / 32);
   elt::maxpool_kernel<<<elt::blocks_for(total), elt::kThreads, 0, stream>>>(a);
   return check_launch("maxpool launch", err);
 }

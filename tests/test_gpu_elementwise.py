@@ -64,8 +64,11 @@ def test_residual_add_matches_oracle(a_bits, b_bits, up, mirror, out_bits, with_
     assert_same(Y.data.cpu().numpy().reshape(ref.packed.shape), ref.packed, c, out_bits, "residual")
 
 
+# 16-byte units (4-bit 64 / 96 ch, 2-bit 256 ch, 8-bit 32 ch), single words (2-bit 32 ch: 8-byte
+# rows; 8-bit 4 ch), and the generic kernel (8-bit 3 ch, 3-bit)
 @pytest.mark.parametrize("bits,c,k,stride,pad", [(4, 64, 3, 2, 1), (2, 256, 3, 2, 1), (8, 3, 2, 2, 0),
-                                                  (3, 32, 3, 1, 1)])
+                                                  (3, 32, 3, 1, 1), (2, 32, 3, 1, 1), (8, 32, 3, 2, 1),
+                                                  (8, 4, 2, 2, 0), (4, 96, 3, 2, 0)])
 def test_maxpool_matches_oracle(bits, c, k, stride, pad):
     rng = np.random.default_rng(bits + c)
     x = synth.act_codes(rng, (2, 41, 67, c), bits)

@@ -186,7 +186,8 @@ aqd_status aqd_conv_int_grouped(const aqd_conv_job* jobs, int32_t njobs,
  * byte image (one byte per code: sum over jobs of n*(h+2*pad)*(w+2*pad)*cin bytes) and feed
  * the tensor cores from it with TMA tile loads, instead of unpacking every code once per
  * kernel tap inside the convolution. Returns 0 when this path does not apply (stride != 1,
- * cin % 128 != 0, codes or weights wider than 4 bits); a NULL or smaller workspace passed
+ * cin % 64 != 0, codes or weights wider than 4 bits with cin % 128 != 0, K * 3825 >= 2^24
+ * with 8-bit codes or weights); a NULL or smaller workspace passed
  * to the conv calls then selects the in-kernel unpacking path. */
 size_t aqd_conv_workspace_bytes(const aqd_conv_job* jobs, int32_t njobs,
                                 const aqd_conv_weights* w, int32_t stride, int32_t pad);
@@ -216,7 +217,7 @@ aqd_status aqd_conv_int_grouped_expanded(const aqd_conv_job* jobs, int32_t njobs
  * can be called with aqd_conv_int_grouped_expanded (or this function) without an
  * expansion pass. Only the interior of the image is written: its border must already hold
  * zeros (fill next_workspace with zeros once, or expand an input of the same shape into it
- * once; no call writes the border afterwards). Needs cout % 128 == 0, a next_workspace of
+ * once; no call writes the border afterwards). Needs cout % 64 == 0, a next_workspace of
  * at least sum(n * (ho + 2 next_pad) * (wo + 2 next_pad)) * cout bytes, 256-byte aligned
  * and not overlapping `workspace`; otherwise AQD_ERR_INVALID. The paper's layers pass
  * k-bit codes from one layer to the next (Eq. 2, Fig. 1); this is the same codes stored one

@@ -217,9 +217,12 @@ static bool split_weights(const aqd_conv_weights* w) { return w->w_bits == 8 && 
 static int64_t flat_rows(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w, int32_t stride,
                          int32_t pad, int32_t* planes = nullptr) {
   if (!jobs || njobs <= 0 || njobs > kMaxJobs || !w) return 0;
-  if (stride != 1 || pad < 0 || w->cin <= 0 || w->cin % 128 != 0) return 0;
+  if (stride != 1 || pad < 0 || w->cin <= 0 || w->cin % 64 != 0) return 0;
   if (w->w_format != AQD_W_TWOS && w->w_format != AQD_W_ODD) return 0;
   const bool wsplit = split_weights(w);
+  // rows of 64 channels (64-byte K chunks) only for 2- to 4-bit codes and 4-bit-range weights
+  const bool half_rows = w->cin % 128 != 0;
+  if (half_rows && wsplit) return 0;
   if (!(w->w_bits >= 2 && w->w_bits <= 4) && !wsplit) return 0;
   const int64_t max_w = max_abs_weight(w->w_bits, w->w_format);
   if (max_w > 15 && !wsplit) return 0;
@@ -229,6 +232,7 @@ static int64_t flat_rows(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv
   for (int j = 0; j < njobs; ++j) {
     const aqd_tensor& x = jobs[j].x;
     if (!(x.bits >= 2 && x.bits <= 4) && x.bits != 8) return 0;
+    if (half_rows && x.bits == 8) return 0;
     if (x.c != w->cin || x.n <= 0 || x.h <= 0 || x.w <= 0) return 0;
     if (x.bits == 8) np = 2;
     const bool wide = x.bits == 8 || wsplit;
@@ -437,7 +441,7 @@ static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aq
     if ((reinterpret_cast<uintptr_t>(chain->ws) & 255) != 0) return fail(AQD_ERR_INVALID, "next_workspace must be 256-byte aligned");
     if (chain->pad < 0) return fail(AQD_ERR_INVALID, "next_pad must be >= 0");
     if (out_bits < 2 || out_bits > 4) return fail(AQD_ERR_INVALID, "a chained output needs 2-, 3- or 4-bit codes");
-    if (w->cout % 128 != 0) return fail(AQD_ERR_INVALID, "a chained output needs cout % 128 == 0");
+    if (w->cout % 64 != 0) return fail(AQD_ERR_INVALID, "a chained output needs cout % 64 == 0");
     int64_t orows = 0;
     for (int j = 0; j < njobs; ++j)
       orows += (int64_t)jobs[j].y.n * (jobs[j].y.h + 2 * chain->pad) * (jobs[j].y.w + 2 * chain->pad);

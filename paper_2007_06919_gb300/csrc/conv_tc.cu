@@ -66,7 +66,7 @@ constexpr int kThreads = (kWarpProd0 + kProdWarps) * 32;
 constexpr int kTmaWarpsFlat = 3;
 __host__ __device__ constexpr int tma_warps(bool flat) { return flat ? kTmaWarpsFlat : kTmaWarps; }
 __host__ __device__ constexpr int threads_for(bool flat) { return flat ? (kWarpTma + kTmaWarpsFlat) * 32 : kThreads; }
-constexpr int kMaxStages = 8;
+constexpr int kMaxStages = 16;
 constexpr int kQTab = 256;  // K-chunk table entries (larger K falls back to division)
 
 struct Params {
@@ -156,10 +156,26 @@ __device__ __forceinline__ void load_skip_group(const Params& p, const uint8_t* 
   for (int i = 0; i < 32; ++i) sk[i] = 0;
   {
     const int sb = p.skip_bits;
-    if (sb == 32) {
+    // a whole group of 32 channels in rows whose size is a multiple of 16 bytes: 16-byte loads
+    // (the tensor base is 16-byte aligned); otherwise element by element
+    const bool whole = ncols == 32 && ch0 + 32 <= p.cout && (p.skip_row_bytes & 15) == 0;
+    if (sb == 32 && whole) {
+      const int4* s4 = reinterpret_cast<const int4*>(reinterpret_cast<const int32_t*>(srow) + ch0);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const int4 v = __ldg(s4 + q);
+        sk[4 * q] = v.x; sk[4 * q + 1] = v.y; sk[4 * q + 2] = v.z; sk[4 * q + 3] = v.w;
+      }
+    } else if (sb == 32) {
       const int32_t* s32 = reinterpret_cast<const int32_t*>(srow) + ch0;
 #pragma unroll
       for (int i = 0; i < 32; ++i) sk[i] = (i < ncols && ch0 + i < p.cout) ? __ldg(s32 + i) : 0;
+    } else if (sb == 8 && whole) {
+      const uint4* s16 = reinterpret_cast<const uint4*>(srow + ch0);
+      const uint4 a = __ldg(s16), b = __ldg(s16 + 1);
+      const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+#pragma unroll
+      for (int i = 0; i < 32; ++i) sk[i] = (int32_t)((w[i / 4] >> (8 * (i % 4))) & 0xFFu);
     } else if (sb == 8) {
       const uint8_t* s8 = srow + ch0;
 #pragma unroll
@@ -167,7 +183,16 @@ __device__ __forceinline__ void load_skip_group(const Params& p, const uint8_t* 
     } else {
       // 2/3/4-bit codes: one whole packed group (the layout needs cout % 32 == 0)
       const uint32_t* g32 = reinterpret_cast<const uint32_t*>(srow + (ch0 >> 5) * group_bytes(sb));
-      uint32_t g[4] = {__ldg(g32), __ldg(g32 + 1), sb >= 3 ? __ldg(g32 + 2) : 0u, sb == 4 ? __ldg(g32 + 3) : 0u};
+      uint32_t g[4] = {0u, 0u, 0u, 0u};
+      if (sb == 4) {  // 16-byte groups at 16-byte offsets
+        const uint4 v = __ldg(reinterpret_cast<const uint4*>(g32));
+        g[0] = v.x; g[1] = v.y; g[2] = v.z; g[3] = v.w;
+      } else if (sb == 2) {
+        const uint2 v = __ldg(reinterpret_cast<const uint2*>(g32));
+        g[0] = v.x; g[1] = v.y;
+      } else {
+        g[0] = __ldg(g32); g[1] = __ldg(g32 + 1); g[2] = __ldg(g32 + 2);
+      }
       uint32_t b[8];
       if (sb == 2) unpack_group_bytes<2>(g, b);
       else if (sb == 3) unpack_group_bytes<3>(g, b);
@@ -213,6 +238,26 @@ __device__ __forceinline__ void fast_skip_group(const uint32_t* v, const EpiChan
     const int64_t sc = (int64_t)sk[i] * (int64_t)c.c;
     const int32_t st = (int32_t)((sc + (1LL << (c.d - 1))) >> c.d);
     const int32_t u = add_sat(acc + c.bias, st);
+    const int r = c.r;
+    y[i] = min(max((__mulhi(u, c.m0) + (1 << (r - 33))) >> (r - 32), 0), qmax);
+  }
+}
+
+// Skip epilogue for an int32 skip (a downsample branch in accumulator units), default
+// direction, when every column has R >= 33, |bias| <= 2^30 and d >= 1: Eq. 7's rescaled skip
+// rhu(s * c, d) is one 64-bit product, add and shift (|s * c| < 2^62); acc + bias fits in
+// int32 (|acc| < 2^24); the sum is saturated to int32 as in Eq. 7's int64 form, and the requant
+// is the 32-bit form of fast_requant_group.
+__device__ __forceinline__ void fast_skip32_group(const uint32_t* v, const EpiChan* ep, const int32_t (&sk)[32],
+                                                  int qmax, int32_t (&y)[32]) {
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    const EpiChan c = ep[i];
+    const int32_t acc = __float2int_rn(__uint_as_float(v[i]) * 262144.0f);  // exact integer
+    const int64_t st = ((int64_t)sk[i] * (int64_t)c.c + (1LL << (c.d - 1))) >> c.d;
+    int64_t t = (int64_t)(acc + c.bias) + st;
+    t = t > 2147483647LL ? 2147483647LL : (t < -2147483648LL ? -2147483648LL : t);
+    const int32_t u = (int32_t)t;
     const int r = c.r;
     y[i] = min(max((__mulhi(u, c.m0) + (1 << (r - 33))) >> (r - 32), 0), qmax);
   }
@@ -346,11 +391,14 @@ __device__ __forceinline__ void load_chunk(const Params& p, RowCursor<kXBits>& r
 // kSkip: the instantiation that handles a skip tensor (Eq. 7); the others carry no skip code,
 // which keeps the common path's registers free.
 // kSplit: the 8-bit split form (split weights combined as D1 + 16 D2 in the epilogue).
-template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair, bool kSkip, bool kSplit>
+template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair, bool kSkip, bool kSplit, int kBK>
 __global__ void __launch_bounds__(threads_for(kFlat), 1)
 conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_wh,
                const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ Params p) {
   static_assert(!kPair || kFlat, "the CTA-pair form exists for the workspace path only");
+  static_assert(kBK == BK || kFlat, "64-byte K chunks exist for the workspace path only");
+  // bytes of one stage's A operand: kSub sub-tiles of 128 rows x kBK bytes
+  constexpr int kStA = kSub * 128 * kBK;
   constexpr int kTma = tma_warps(kFlat);
   // CTA pair: this CTA's rank; the even CTA issues the MMAs; a tile has 256 rows
   const uint32_t rank = kPair ? cluster_ctarank() : 0u;
@@ -378,7 +426,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
   const int warp = threadIdx.x / 32;
   const int lane = threadIdx.x % 32;
   const int BN = p.bn;
-  const uint32_t stage_b_bytes = (uint32_t)(kPair ? BN / 2 : BN) * BK;  // this CTA's rows of B
+  const uint32_t stage_b_bytes = (uint32_t)(kPair ? BN / 2 : BN) * kBK;  // this CTA's rows of B
 
   // K chunk q -> (tap row r, tap column sx, 128-channel block cb), for the TMA issuers
   uint32_t* qtab = reinterpret_cast<uint32_t*>(smem + p.off_qtab);
@@ -442,7 +490,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       // (byte offset >> 4) to the 14-bit start-address field (shared addresses < 2^18)
       // the descriptors' high words are constant; stages / sub-tiles / k-steps only move the
       // 14-bit start-address field in the low word (shared addresses < 2^18, no carry)
-      const uint64_t da0 = sdesc_sw128(s_a), db0 = sdesc_sw128(s_b);
+      const uint64_t da0 = sdesc_k<kBK>(s_a), db0 = sdesc_k<kBK>(s_b);
       const uint32_t a_lo0 = (uint32_t)da0, b_lo0 = (uint32_t)db0;
       const uint32_t a_hi = (uint32_t)(da0 >> 32), b_hi = (uint32_t)(db0 >> 32);
       uint32_t it = 0, lt = 0, s = 0, ph = 0;
@@ -459,16 +507,16 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
           // are ordered for the MMA by the mbarrier phase alone; tcgen05.fence is needed only
           // where TMEM changes hands, after the accumulator-empty wait above)
           if (!next_ready && !mbar_poll(b_full + 8 * s, ph, abort_flag)) { ok = false; break; }
-          const uint32_t a_lo = a_lo0 + ((s * kStageA) >> 4);
+          const uint32_t a_lo = a_lo0 + ((s * kStA) >> 4);
           const uint32_t b_lo = b_lo0 + ((s * stage_b_bytes) >> 4);
           const uint32_t s_next = s + 1 == (uint32_t)S ? 0u : s + 1;
           const uint32_t ph_next = s_next == 0 ? ph ^ 1u : ph;
 #pragma unroll
-          for (int kk = 0; kk < BK / 32; ++kk) {
+          for (int kk = 0; kk < kBK / 32; ++kk) {
             // The tensor pipe takes about one instruction at a time, so each issue waits for
             // the previous MMA. Testing the next stage here, while the last MMAs of this
             // chunk run, lets the next chunk's first MMA follow this chunk's commit at once.
-            if (kk == BK / 32 - 1) next_ready = mbar_test(b_full + 8 * s_next, ph_next);
+            if (kk == kBK / 32 - 1) next_ready = mbar_test(b_full + 8 * s_next, ph_next);
             const uint32_t acc = (q > 0 || kk > 0) ? 1u : 0u;
             const uint64_t db = ((uint64_t)b_hi << 32) | (b_lo + 2 * kk);
             if constexpr (kPair) {
@@ -534,27 +582,27 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
             // leader's "full" barrier, which the leader arms with the bytes of all four
             const int row = row0 + prow + r * wp + sx;
             const int brow = ti.brow + (int)rank * (ti.bn / 2);
-            const uint32_t b_bytes = (uint32_t)(ti.bn / 2) * BK;
+            const uint32_t b_bytes = (uint32_t)(ti.bn / 2) * kBK;
             if (leader) {
-              mbar_arrive_expect_tx(b_full + 8 * s, 2 * (b_bytes + kStageA));
-              tma_load_2d(s_a + s * kStageA, &tmap_a, cb * BK, row, b_full + 8 * s);
-              tma_load_2d(s_b + s * stage_b_bytes, wm, q * BK, brow, b_full + 8 * s);
+              mbar_arrive_expect_tx(b_full + 8 * s, 2 * (b_bytes + kStA));
+              tma_load_2d(s_a + s * kStA, &tmap_a, cb * kBK, row, b_full + 8 * s);
+              tma_load_2d(s_b + s * stage_b_bytes, wm, q * kBK, brow, b_full + 8 * s);
             } else {
               const uint32_t fb = mapa_shared(b_full + 8 * s, 0);
-              tma_load_2d_pair(s_a + s * kStageA, &tmap_a, cb * BK, row, fb);
-              tma_load_2d_pair(s_b + s * stage_b_bytes, wm, q * BK, brow, fb);
+              tma_load_2d_pair(s_a + s * kStA, &tmap_a, cb * kBK, row, fb);
+              tma_load_2d_pair(s_b + s * stage_b_bytes, wm, q * kBK, brow, fb);
             }
             continue;
           } else if constexpr (kFlat) {
             // A: 128 consecutive rows of the padded byte image, shifted by the tap (r, s)
             const int row = row0 + prow + r * wp + sx;
-            mbar_arrive_expect_tx(b_full + 8 * s, (uint32_t)ti.bn * BK + kStageA);
-            tma_load_2d(s_a + s * kStageA, &tmap_a, cb * BK, row, b_full + 8 * s);
+            mbar_arrive_expect_tx(b_full + 8 * s, (uint32_t)ti.bn * kBK + kStA);
+            tma_load_2d(s_a + s * kStA, &tmap_a, cb * kBK, row, b_full + 8 * s);
           } else {
             (void)r; (void)sx; (void)cb;
-            mbar_arrive_expect_tx(b_full + 8 * s, (uint32_t)ti.bn * BK);
+            mbar_arrive_expect_tx(b_full + 8 * s, (uint32_t)ti.bn * kBK);
           }
-          tma_load_2d(s_b + s * stage_b_bytes, wm, q * BK, ti.brow, b_full + 8 * s);
+          tma_load_2d(s_b + s * stage_b_bytes, wm, q * kBK, ti.brow, b_full + 8 * s);
         }
       }
       if (!ok) fail(abort_flag, p.status);
@@ -641,50 +689,64 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
     bool ok = true;
     const int out_bits = p.out_bits;
     const int qmax = (1 << (out_bits & 15)) - 1;
+    // the per-column constant tables of the last tile's level and channel range: rebuilt only
+    // when a tile needs others (tiles of one job and N range keep them), so most tiles start
+    // without table loads or barriers
+    long long cur_key = -1;  // (level, first channel, width) of the tables
+    int flags = 0;           // bit 0: 32-bit requant form, 1: |bias| <= 2^30, 2: 32-bit skip form
     for (int t = first_tile; t < p.total_tiles; t += tile_stride, ++lt) {
       const TileInfo ti = tile_info(p, t);
       const ConvJobDev& jb = p.jobs[ti.job];
-      named_bar(1, kEpiThreads);
-      // Per-column constants of this tile's level. The 32-bit fast path applies when the
-      // total requant shift R = 31 + shift is >= 33 (then y = (mulhi(u, M0) + 2^(R-33)) >>
-      // (R-32) equals rhu(u * M0, R): the low product word cannot carry into the result)
-      // and |bias| <= 2^30 (acc + bias cannot leave int32 when |acc| < 2^24).
-      int fast_req = 1, small_bias = 1;
       // this tile's output channels that exist (a last N tile may reach past cout; packed
       // groups past it must not be written)
       const int TBN = ti.cn < p.cout - ti.col0 ? ti.cn : p.cout - ti.col0;
-      for (int col = et; col < 256; col += kEpiThreads) {
-        const int ch = ti.col0 + col;
-        EpiChan ec{};
-        int4 ef = make_int4((int32_t)(0u - kMagicBits), 0, 0, 1);
-        if (col < TBN && ch < p.cout) {
-          const int64_t idx = (int64_t)jb.level * p.cout + ch;
-          ec.bias = p.bias ? p.bias[idx] : 0;
-          const bool sb = ec.bias >= -(1 << 30) && ec.bias <= (1 << 30);
-          small_bias &= sb;
-          ef.x = (int32_t)((uint32_t)ec.bias - kMagicBits);
-          if (out_bits != 32) {
-            ec.m0 = p.m0[idx];
-            const int r = 31 + p.shift[idx];
-            ec.r = (int8_t)r;
-            if (r >= 33 && sb) { ef.y = ec.m0; ef.z = 1 << (r - 33); ef.w = r - 32; }
-            else fast_req = 0;
+      const long long key = ((long long)jb.level << 32) | ((long long)ti.col0 << 10) | TBN;
+      if (key != cur_key) {
+        // (the same decision in every epilogue thread: all of them see the same tiles)
+        named_bar(1, kEpiThreads);  // every epilogue warp is done with the previous tables
+        // Per-column constants of this tile's level. The 32-bit fast path applies when the
+        // total requant shift R = 31 + shift is >= 33 (then y = (mulhi(u, M0) + 2^(R-33)) >>
+        // (R-32) equals rhu(u * M0, R): the low product word cannot carry into the result)
+        // and |bias| <= 2^30 (acc + bias cannot leave int32 when |acc| < 2^24).
+        int fq = 1, sbias = 1;
+        for (int col = et; col < 256; col += kEpiThreads) {
+          const int ch = ti.col0 + col;
+          EpiChan ec{};
+          int4 ef = make_int4((int32_t)(0u - kMagicBits), 0, 0, 1);
+          if (col < TBN && ch < p.cout) {
+            const int64_t idx = (int64_t)jb.level * p.cout + ch;
+            ec.bias = p.bias ? p.bias[idx] : 0;
+            const bool sb = ec.bias >= -(1 << 30) && ec.bias <= (1 << 30);
+            sbias &= sb;
+            ef.x = (int32_t)((uint32_t)ec.bias - kMagicBits);
+            if (out_bits != 32) {
+              ec.m0 = p.m0[idx];
+              const int r = 31 + p.shift[idx];
+              ec.r = (int8_t)r;
+              if (r >= 33 && sb) { ef.y = ec.m0; ef.z = 1 << (r - 33); ef.w = r - 32; }
+              else fq = 0;
+            }
+            if (p.has_skip) { ec.c = p.skip_c[idx]; ec.d = p.skip_d[idx]; }
           }
-          if (p.has_skip) { ec.c = p.skip_c[idx]; ec.d = p.skip_d[idx]; }
+          epi[col] = ec;
+          reinterpret_cast<int4*>(epi + 256)[col] = ef;
         }
-        epi[col] = ec;
-        reinterpret_cast<int4*>(epi + 256)[col] = ef;
+        fq = named_bar_and(1, kEpiThreads, fq);
+        sbias = named_bar_and(1, kEpiThreads, sbias);
+        // 32-bit skip path (fast_skip_group): default direction, code skips, d >= 8 everywhere
+        // (int32 skips: 64-bit product, any d >= 1)
+        int fsk = 0;
+        if (kSkip && p.has_skip && p.scale_main == 0 && out_bits != 32 && fq && sbias) {
+          const int dmin = p.skip_bits <= 8 ? 8 : 1;
+          int okd = 1;
+          for (int col = et; col < TBN; col += kEpiThreads)
+            if (ti.col0 + col < p.cout && epi[col].d < dmin) okd = 0;
+          fsk = named_bar_and(1, kEpiThreads, okd);
+        }
+        flags = fq | (sbias << 1) | (fsk << 2);
+        cur_key = key;
       }
-      fast_req = named_bar_and(1, kEpiThreads, fast_req);
-      small_bias = named_bar_and(1, kEpiThreads, small_bias);
-      // 32-bit skip path (fast_skip_group): default direction, code skips, d >= 8 everywhere
-      int fast_skip = 0;
-      if (kSkip && p.has_skip && p.scale_main == 0 && p.skip_bits <= 8 && out_bits != 32 && fast_req && small_bias) {
-        int ok8 = 1;
-        for (int col = et; col < TBN; col += kEpiThreads)
-          if (ti.col0 + col < p.cout && epi[col].d < 8) ok8 = 0;
-        fast_skip = named_bar_and(1, kEpiThreads, ok8);
-      }
+      const int fast_req = flags & 1, small_bias = (flags >> 1) & 1, fast_skip = (flags >> 2) & 1;
       // 0: general int64 epilogue; 1: fast requant to codes; 2: int32 output, no skip
       const int mode = (kSplit || p.has_skip) ? 0 : (out_bits == 32 ? 2 : (fast_req ? 1 : 0));
       const bool magic = p.acc_small && (mode == 2 ? small_bias : fast_req);
@@ -793,17 +855,25 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
           } else {
             const uint8_t* srow = nullptr;
             if (kSkip && p.has_skip) {
-              const int hw = jb.ho * jb.wo;
-              const int img = m / hw;
-              const int rem = m - img * hw;
-              const int ho = rem / jb.wo, wo = rem - (rem / jb.wo) * jb.wo;
-              const int sh = ho / p.upsample, sw = wo / p.upsample;
+              int img, ho, wo;
+              if constexpr (kFlat) {
+                img = oimg; ho = oh; wo = ow;
+              } else {
+                const int hw = jb.ho * jb.wo;
+                img = m / hw;
+                const int rem = m - img * hw;
+                ho = rem / jb.wo; wo = rem - ho * jb.wo;
+              }
+              const int sh = p.upsample == 2 ? ho >> 1 : ho, sw = p.upsample == 2 ? wo >> 1 : wo;
               srow = jb.skip + (((int64_t)img * jb.skip_h + sh) * jb.skip_w + sw) * p.skip_row_bytes;
             }
             int32_t oo[32];
-            if (kSkip && fast_skip) {
+            if (kSkip && fast_skip && p.skip_bits <= 8) {
               load_skip_group(p, srow, ch0, ncols, oo);   // skip codes, replaced by the results
               fast_skip_group(v, epi + g0, oo, qmax, oo);
+            } else if (kSkip && fast_skip) {
+              load_skip_group(p, srow, ch0, ncols, oo);   // int32 skip, replaced by the results
+              fast_skip32_group(v, epi + g0, oo, qmax, oo);
             } else {
               general_group<kSkip, kSplit>(p, v, epi + g0, srow, ch0, ncols, oo);
             }
@@ -1028,10 +1098,11 @@ static EncodeTiledFn get_encode_fn(std::string* err) {
   return fn;
 }
 
-template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair = false, bool kSkip = true, bool kSplit = false>
+template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair = false, bool kSkip = true, bool kSplit = false,
+          int kBK = BK>
 static int launch_bits(const Params& prm, const CUtensorMap& map, const CUtensorMap& map_h, const CUtensorMap& map_a,
                        int grid, size_t smem, cudaStream_t stream, std::string* err) {
-  auto kern = conv_tc_kernel<kXBits, kChunkInTap, kFlat, kPair, kSkip, kSplit>;
+  auto kern = conv_tc_kernel<kXBits, kChunkInTap, kFlat, kPair, kSkip, kSplit, kBK>;
   // The opt-in limit is raised to the device maximum, never lowered to this call's size:
   // a CUDA graph node captured earlier with a larger plan must stay launchable (a graph
   // node, or a tool relaunching it, is checked against the function's current limit).
@@ -1106,8 +1177,11 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
       tiles += ((a.jobs[j].m_total + BM - 1) / BM) * prm.n_tiles;
     }
   }
-  if (flat && (kSub != 1 || a.stride != 1 || a.cin % BK != 0 || rows > a.ws_rows)) {
-    *err = "conv_tc: workspace path needs stride 1, cin % 128 == 0 and a large enough workspace";
+  // K chunk width: 128 bytes of one tap, or on the workspace path with cin % 128 != 0 the 64
+  // channels of one tap (cin % 64 == 0; 64-byte swizzled operand rows, two MMAs per chunk)
+  const int bk = (flat && a.cin % BK != 0) ? 64 : BK;
+  if (flat && (kSub != 1 || a.stride != 1 || a.cin % bk != 0 || rows > a.ws_rows || (a.split_w && bk != BK))) {
+    *err = "conv_tc: workspace path needs stride 1, cin % 64 == 0 (128 for split weights) and a large enough workspace";
     return 1;
   }
   if (tiles == 0) return 0;
@@ -1124,7 +1198,7 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   // (a half tile must start on a 32-channel packing group: BN / 2 a multiple of 32)
   if (BN % 64 == 0 && !a.split_w && rem > 0 && 2 * rem <= workers) prm.dp_tiles = tiles - rem;
   prm.total_tiles = prm.dp_tiles + 2 * (tiles - prm.dp_tiles);
-  prm.num_kchunks = a.k_pad / BK;
+  prm.num_kchunks = flat ? a.k_total / bk : a.k_pad / BK;
   prm.cin = a.cin; prm.cout = a.cout; prm.kh = a.kh; prm.kw = a.kw;
   prm.stride = a.stride; prm.pad = a.pad; prm.k_total = a.k_total;
   prm.out_bits = a.out_bits; prm.skip_bits = a.skip_bits;
@@ -1134,7 +1208,7 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   prm.upsample = a.upsample; prm.scale_main = a.scale_main; prm.has_skip = a.has_skip;
   prm.bn = BN;
   prm.acc_small = a.acc_bound < (1LL << 22) ? 1 : 0;
-  prm.cin_chunks = a.cin / BK;
+  prm.cin_chunks = a.cin / bk;
   prm.ws_out = a.ws_out;
   prm.out_pad = a.out_pad;
   prm.a_planes = flat ? (a.a_planes > 1 ? a.a_planes : 1) : 1;
@@ -1151,9 +1225,10 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
     }
   }
   prm.status = a.status;
-  // shared memory plan: stages of (BM x 128 A bytes + this CTA's B rows x 128 bytes)
+  // shared memory plan: stages of (BM x bk A bytes + this CTA's B rows x bk bytes)
   const int b_rows = pair ? BN / 2 : BN;
-  const size_t stage_bytes = (size_t)kStageA + (size_t)b_rows * BK;
+  const size_t stage_a = (size_t)kSub * 128 * bk;
+  const size_t stage_bytes = stage_a + (size_t)b_rows * bk;
   const size_t epi_bytes = 256 * sizeof(EpiChan) + 256 * sizeof(int4);
   const size_t bar_bytes = 8 * (2 * kMaxStages + 5) + 16;
   const size_t qtab_bytes = kQTab * sizeof(uint32_t);
@@ -1167,8 +1242,8 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   // most as many as the stages.
   if (stages < tma_warps(flat)) { *err = "conv_tc: fewer pipeline stages than TMA issuers"; return 2; }
   prm.stages = stages;
-  prm.off_b = (uint32_t)(stages * kStageA);
-  prm.off_epi = prm.off_b + (uint32_t)(stages * b_rows * BK);
+  prm.off_b = (uint32_t)(stages * stage_a);
+  prm.off_epi = prm.off_b + (uint32_t)(stages * b_rows * bk);
   prm.off_bar = prm.off_epi + (uint32_t)epi_bytes;
   prm.off_qtab = prm.off_bar + (uint32_t)bar_bytes;
   const size_t smem = 1024 + prm.off_qtab + qtab_bytes;
@@ -1181,18 +1256,19 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   CUtensorMap map;
   cuuint64_t gdim[2] = {(cuuint64_t)a.k_pad, (cuuint64_t)w_rows};
   cuuint64_t gstride[1] = {(cuuint64_t)a.k_pad};
-  cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)b_rows};
+  cuuint32_t box[2] = {(cuuint32_t)bk, (cuuint32_t)b_rows};
   cuuint32_t estr[2] = {1, 1};
+  const CUtensorMapSwizzle swz = bk == 64 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B;
   CUresult r = enc(&map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)a.w_e4m3, gdim, gstride, box, estr,
-                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) { *err = "cuTensorMapEncodeTiled failed: " + std::to_string((int)r); return 3; }
   // the same weights with boxes of half the rows, for the half-width tiles
   CUtensorMap map_h = map;
   if (prm.dp_tiles < prm.total_tiles) {
-    cuuint32_t box_h[2] = {(cuuint32_t)BK, (cuuint32_t)(b_rows / 2)};
+    cuuint32_t box_h[2] = {(cuuint32_t)bk, (cuuint32_t)(b_rows / 2)};
     r = enc(&map_h, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)a.w_e4m3, gdim, gstride, box_h, estr,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) { *err = "cuTensorMapEncodeTiled (half) failed: " + std::to_string((int)r); return 3; }
   }
@@ -1234,12 +1310,12 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
       if (e != cudaSuccess) { *err = std::string("expand launch: ") + cudaGetErrorString(e); return 3; }
     }
     if (a.expand_only) return 0;
-    // 2) tensor map over the workspace as a [rows][cin] byte matrix with 128 x 128 boxes
+    // 2) tensor map over the workspace as a [rows][cin] byte matrix with bk x 128 boxes
     cuuint64_t gd[2] = {(cuuint64_t)a.cin, (cuuint64_t)rows * (cuuint64_t)prm.a_planes};
     cuuint64_t gs[1] = {(cuuint64_t)a.cin};
-    cuuint32_t bx[2] = {(cuuint32_t)BK, 128};
+    cuuint32_t bx[2] = {(cuuint32_t)bk, 128};
     CUresult r2 = enc(&map_a, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)a.ws, gd, gs, bx, estr,
-                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                      CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
                       CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r2 != CUDA_SUCCESS) {
       *err = "cuTensorMapEncodeTiled (activations) failed: " + std::to_string((int)r2);
@@ -1249,21 +1325,34 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
       if (pair) return launch_bits<2, true, true, true, false, true>(prm, map, map_h, map_a, grid, smem, stream, err);
       return launch_bits<2, true, true, false, false, true>(prm, map, map_h, map_a, grid, smem, stream, err);
     }
+    if (bk == 64) {
+      if (pair)
+        return a.has_skip ? launch_bits<2, true, true, true, true, false, 64>(prm, map, map_h, map_a, grid, smem, stream, err)
+                          : launch_bits<2, true, true, true, false, false, 64>(prm, map, map_h, map_a, grid, smem, stream, err);
+      return a.has_skip ? launch_bits<2, true, true, false, true, false, 64>(prm, map, map_h, map_a, grid, smem, stream, err)
+                        : launch_bits<2, true, true, false, false, false, 64>(prm, map, map_h, map_a, grid, smem, stream, err);
+    }
     if (pair)
       return a.has_skip ? launch_bits<2, true, true, true, true>(prm, map, map_h, map_a, grid, smem, stream, err)
                         : launch_bits<2, true, true, true, false>(prm, map, map_h, map_a, grid, smem, stream, err);
     return a.has_skip ? launch_bits<2, true, true, false, true>(prm, map, map_h, map_a, grid, smem, stream, err)
                       : launch_bits<2, true, true, false, false>(prm, map, map_h, map_a, grid, smem, stream, err);
   }
+  // in-kernel unpacking; the instantiation without skip code keeps its registers for the
+  // common case
+#define AQD_INKERNEL(B)                                                                                  \
+  if (a.has_skip)                                                                                          \
+    return in_tap ? launch_bits<B, true, false, false, true>(prm, map, map_h, map_a, grid, smem, stream, err) \
+                  : launch_bits<B, false, false, false, true>(prm, map, map_h, map_a, grid, smem, stream, err); \
+  return in_tap ? launch_bits<B, true, false, false, false>(prm, map, map_h, map_a, grid, smem, stream, err)   \
+                : launch_bits<B, false, false, false, false>(prm, map, map_h, map_a, grid, smem, stream, err);
   switch (a.x_bits) {
-    case 2: return in_tap ? launch_bits<2, true, false>(prm, map, map_h, map_a, grid, smem, stream, err)
-                          : launch_bits<2, false, false>(prm, map, map_h, map_a, grid, smem, stream, err);
-    case 3: return in_tap ? launch_bits<3, true, false>(prm, map, map_h, map_a, grid, smem, stream, err)
-                          : launch_bits<3, false, false>(prm, map, map_h, map_a, grid, smem, stream, err);
-    case 4: return in_tap ? launch_bits<4, true, false>(prm, map, map_h, map_a, grid, smem, stream, err)
-                          : launch_bits<4, false, false>(prm, map, map_h, map_a, grid, smem, stream, err);
+    case 2: { AQD_INKERNEL(2) }
+    case 3: { AQD_INKERNEL(3) }
+    case 4: { AQD_INKERNEL(4) }
     default: *err = "conv_tc: activation bits must be 2, 3 or 4"; return 2;
   }
+#undef AQD_INKERNEL
 }
 
 }  // namespace aqd

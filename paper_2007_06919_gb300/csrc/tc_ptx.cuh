@@ -180,6 +180,24 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
   return d;
 }
 
+// SW64 K-major descriptor (operand rows of 64 bytes): stride byte offset 512 between
+// 8-row groups, swizzle mode 4 = 64B.
+__device__ __forceinline__ uint64_t sdesc_sw64(uint32_t saddr) {
+  uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)1 << 16;
+  d |= (uint64_t)(512 >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)4 << 61;
+  return d;
+}
+// descriptor for K chunks of kBK bytes (128: SW128, 64: SW64)
+template <int kBK>
+__device__ __forceinline__ uint64_t sdesc_k(uint32_t saddr) {
+  static_assert(kBK == 128 || kBK == 64, "K chunks of 64 or 128 bytes");
+  if constexpr (kBK == 128) return sdesc_sw128(saddr);
+  else return sdesc_sw64(saddr);
+}
+
 // Instruction descriptor, kind::f8f6f4 (A=B=E4M3) or kind::f16 (A=B=F16, the same type
 // code 0): D=F32, both K-major, N>>3, M>>4. M=256 exists only for cta_group::2.
 constexpr int kMmaM = 128;

@@ -141,12 +141,12 @@ class IntDetector:
         """Marks producer -> consumer pairs that hand over the byte image directly: the consumer
         is the next conv, reads exactly the producer's outputs (same job order), and both are
         stride-1 convs on the workspace path; the producer writes 2- to 4-bit codes in blocks of
-        128 channels. The producer still writes its packed outputs for any other reader."""
+        64 channels. The producer still writes its packed outputs for any other reader."""
         convs = [p for k, p in self.steps if k == "conv"]
         for a, b in zip(convs, convs[1:]):
             ca, cb = a.layer.conv, b.layer.conv
             if (list(b.layer.src) == list(a.layer.dst) and b.ws_bytes and a.ws_bytes
-                    and ca.stride == 1 and cb.stride == 1 and 2 <= ca.out_bits <= 4 and ca.cout % 128 == 0):
+                    and ca.stride == 1 and cb.stride == 1 and 2 <= ca.out_bits <= 4 and ca.cout % 64 == 0):
                 a.chain_to = b
                 b.reads_image = True
         # chained images are keyed by geometry (input shapes and padding): the zero border of

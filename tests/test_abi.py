@@ -105,7 +105,8 @@ def test_invalid_arguments_return_before_launch(lib):
 
 def test_workspace_bytes_host_logic(lib):
     """The expanded-activation workspace is planes * sum(n * (h+2p) * (w+2p)) * cin bytes for
-    stride-1 convolutions with cin % 128 == 0 (planes = 2 for 8-bit activation codes; 8-bit
+    stride-1 convolutions with cin % 128 == 0, or cin % 64 == 0 for codes and weights of at
+    most 4 bits (planes = 2 for 8-bit activation codes; 8-bit
     two's-complement weights take the split form), else 0; 8-bit operands also need
     K * 3825 < 2^24 (the exact FP32 partial sums)."""
     from paper_2007_06919_gb300 import aqd
@@ -129,7 +130,15 @@ def test_workspace_bytes_host_logic(lib):
     assert lib.aqd_conv_workspace_bytes(jobs8, 1, ctypes.byref(wbig), 1, 1) == 0
     w64 = aqd._Weights(256, 64, 3, 3, 64, 2, 0)
     jobs[0].x = aqd._Tensor(2, 10, 17, 64, 2, 256)
-    assert lib.aqd_conv_workspace_bytes(jobs, 1, ctypes.byref(w64), 1, 1) == 0    # cin 64
+    assert lib.aqd_conv_workspace_bytes(jobs, 1, ctypes.byref(w64), 1, 1) == 2 * 12 * 19 * 64  # 64-byte rows
+    w96 = aqd._Weights(256, 96, 3, 3, 96, 2, 0)
+    jobs[0].x = aqd._Tensor(2, 10, 17, 96, 2, 256)
+    assert lib.aqd_conv_workspace_bytes(jobs, 1, ctypes.byref(w96), 1, 1) == 0    # cin 96
+    w64s = aqd._Weights(256, 64, 3, 3, 64, 8, 0)                                   # split weights
+    jobs[0].x = aqd._Tensor(2, 10, 17, 64, 2, 256)
+    assert lib.aqd_conv_workspace_bytes(jobs, 1, ctypes.byref(w64s), 1, 1) == 0
+    jobs[0].x = aqd._Tensor(2, 10, 17, 64, 8, 256)                                # 8-bit codes, cin 64
+    assert lib.aqd_conv_workspace_bytes(jobs, 1, ctypes.byref(w64), 1, 1) == 0
 
 
 def test_set_conv_path_rejects_unknown(lib):

@@ -65,6 +65,7 @@ CASES = [
     (2, 2, 0, 1, 1, 1, 64, 64, 3, 1, 1, 2),        # 1x1 image: every tap but the centre pads
     (4, 4, 0, 1, 3, 300, 64, 32, 1, 1, 0, 8),      # 8-bit output codes
     (3, 4, 0, 1, 33, 5, 32, 96, 3, 1, 0, 3),       # no padding, cout 96
+    (4, 4, 0, 2, 9, 13, 192, 64, 3, 1, 1, 4),      # cin 192: three 64-channel chunks per tap
 ]
 
 
@@ -86,7 +87,8 @@ def test_conv_shapes_bit_exact(case, path):
     assert_same(got, want, cout, ob, f"case {case}")
 
 
-WS_CASES = [c for c in CASES if c[9] == 1 and c[6] % 128 == 0 and c[0] <= 4 and c[1] <= 4]
+# workspace path: 128-byte K chunks (cin % 128 == 0) or 64-byte ones (cin % 64 == 0)
+WS_CASES = [c for c in CASES if c[9] == 1 and c[6] % 64 == 0 and c[0] <= 4 and c[1] <= 4]
 
 
 @pytest.mark.parametrize("case", WS_CASES, ids=[str(i) for i in range(len(WS_CASES))])
@@ -124,7 +126,7 @@ def test_workspace_path_edge_shapes(shape, pairs):
 
 @pytest.mark.parametrize("path", [TC, DIRECT])
 @pytest.mark.parametrize("skip_bits,upsample,mirror", [(4, 1, 0), (4, 1, 1), (32, 1, 0), (2, 2, 0), (32, 2, 1),
-                                                        (8, 1, 0)])
+                                                        (8, 1, 0), (32, 2, 0)])
 @pytest.mark.parametrize("ws", [False, True])
 def test_conv_with_skip_bit_exact(path, skip_bits, upsample, mirror, ws):
     """Eq. 7 fused into the epilogue: identity / downsample (int32) / FPN (upsample 2) skips,

@@ -220,8 +220,8 @@ def test_expand_once_then_two_convs_bit_exact():
 
 def test_expanded_conv_needs_an_applicable_workspace():
     rng = np.random.default_rng(3)
-    W, _ = weights(synth.weight_codes(rng, (64, 3, 3, 64), 2), 2)  # cin 64: no workspace path
-    X = aqd.DTensor.empty(1, 8, 8, 64, 2)
+    W, _ = weights(synth.weight_codes(rng, (64, 3, 3, 96), 2), 2)  # cin 96: no workspace path
+    X = aqd.DTensor.empty(1, 8, 8, 96, 2)
     Y = aqd.DTensor.empty(1, 8, 8, 64, 32)
     buf = torch.zeros(1 << 20, dtype=torch.uint8, device="cuda")
     with pytest.raises(aqd.AqdError) as e:

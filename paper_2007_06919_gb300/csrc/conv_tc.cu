@@ -313,6 +313,55 @@ __device__ __forceinline__ void fast_requant_group(const uint32_t* v, const EpiC
   }
 }
 
+// Codes of 32 channels as 8 byte-words (word j holds channels 4j..4j+3, one code per byte):
+// the layout of the chained byte image, and one step from every packed layout.
+// Fastest requant (as magic_requant_group) straight into byte-words.
+__device__ __forceinline__ void magic_requant_bytes(const uint32_t* v, const int4* f, int qmax, uint32_t (&bw)[8]) {
+#pragma unroll
+  for (int j = 0; j < 8; ++j) bw[j] = 0u;
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    const int4 c = f[i];
+    const int32_t u = __float_as_int(__fmaf_rn(__uint_as_float(v[i]), 262144.0f, kMagic)) + c.x;
+    const uint32_t y = (uint32_t)min(max((__mulhi(u, c.y) + c.z) >> c.w, 0), qmax);
+    bw[i / 4] += y << (8 * (i % 4));  // codes < 256: the add is an or
+  }
+}
+// Byte-words of codes < 2^kBits -> the packed group (the layout of common.cuh: word w of the
+// 2/4/8-bit layout holds its channels 4k..4k+3 in bit field k of every byte; the 3-bit layout
+// is two 2-bit words of the low bits and one word of bit 2, channel i at bit 8 (i%4) + i/4).
+template <int kBits>
+__device__ __forceinline__ void pack_bytewords(const uint32_t (&bw)[8], uint32_t (&gw)[8]) {
+  if constexpr (kBits == 8) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) gw[j] = bw[j];
+  } else if constexpr (kBits == 4) {
+#pragma unroll
+    for (int w = 0; w < 4; ++w) gw[w] = bw[2 * w] | (bw[2 * w + 1] << 4);
+  } else if constexpr (kBits == 2) {
+#pragma unroll
+    for (int w = 0; w < 2; ++w)
+      gw[w] = bw[4 * w] | (bw[4 * w + 1] << 2) | (bw[4 * w + 2] << 4) | (bw[4 * w + 3] << 6);
+  } else {
+#pragma unroll
+    for (int w = 0; w < 2; ++w)
+      gw[w] = (bw[4 * w] & 0x03030303u) | ((bw[4 * w + 1] & 0x03030303u) << 2) |
+              ((bw[4 * w + 2] & 0x03030303u) << 4) | ((bw[4 * w + 3] & 0x03030303u) << 6);
+    uint32_t h = 0u;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) h |= ((bw[j] >> 2) & 0x01010101u) << j;
+    gw[2] = h;
+  }
+}
+// Chained output from byte-words (see chain_store).
+__device__ __forceinline__ void chain_store_bytes(const Params& p, const ConvJobDev& jb, int img, int oh, int ow,
+                                                  int ch0, const uint32_t (&bw)[8]) {
+  const int row = jb.orow_off + (img * jb.ohp + oh + p.out_pad) * jb.owp + ow + p.out_pad;
+  uint4* dst = reinterpret_cast<uint4*>(p.ws_out + (size_t)row * p.cout + ch0);
+  dst[0] = make_uint4(bw[0], bw[1], bw[2], bw[3]);
+  dst[1] = make_uint4(bw[4], bw[5], bw[6], bw[7]);
+}
+
 // Chained output: the 32 codes of one packed group, one byte each, at their place in the
 // zero-padded byte image that the next stride-1 conv (padding out_pad) reads.
 __device__ __forceinline__ void chain_store(const Params& p, const ConvJobDev& jb, int img, int oh, int ow,
@@ -813,16 +862,22 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
         if (row_ok) {
           uint8_t* yrow = jb.y + (int64_t)m * p.y_row_bytes;
           const int ch0 = ti.col0 + g0;
-          if (mode == 1) {
+          if (mode == 1 && magic) {
+            // codes as byte-words: the chained image takes them as they are, the packed
+            // output a couple of shifts per 8 codes
+            uint32_t bw[8], gw[8];
+            magic_requant_bytes(v, epf + g0, qmax, bw);
+            switch (out_bits) {
+              case 2: pack_bytewords<2>(bw, gw); break;
+              case 3: pack_bytewords<3>(bw, gw); break;
+              case 4: pack_bytewords<4>(bw, gw); break;
+              default: pack_bytewords<8>(bw, gw); break;
+            }
+            store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
+            if (kFlat && p.ws_out) chain_store_bytes(p, jb, oimg, oh, ow, ch0, bw);
+          } else if (mode == 1) {
             uint32_t gw[8];
-            if (magic) {
-              switch (out_bits) {
-                case 2: magic_requant_group<2>(v, epf + g0, qmax, gw); break;
-                case 3: magic_requant_group<3>(v, epf + g0, qmax, gw); break;
-                case 4: magic_requant_group<4>(v, epf + g0, qmax, gw); break;
-                default: magic_requant_group<8>(v, epf + g0, qmax, gw); break;
-              }
-            } else {
+            {
               switch (out_bits) {
                 case 2: fast_requant_group<2>(v, epi, g0, qmax, gw); break;
                 case 3: fast_requant_group<3>(v, epi, g0, qmax, gw); break;
@@ -883,10 +938,20 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
               for (int i = 0; i < 32; ++i)
                 if (i < ncols && ch0 + i < p.cout) yr[i] = oo[i];
             } else {
-              uint32_t gw[8];
-              pack_group_vals(oo, out_bits, gw);
+              // clipped codes (< 2^out_bits) as byte-words, then the packed group
+              uint32_t bw[8], gw[8];
+#pragma unroll
+              for (int j = 0; j < 8; ++j)
+                bw[j] = (uint32_t)oo[4 * j] | ((uint32_t)oo[4 * j + 1] << 8) | ((uint32_t)oo[4 * j + 2] << 16) |
+                        ((uint32_t)oo[4 * j + 3] << 24);
+              switch (out_bits) {
+                case 2: pack_bytewords<2>(bw, gw); break;
+                case 3: pack_bytewords<3>(bw, gw); break;
+                case 4: pack_bytewords<4>(bw, gw); break;
+                default: pack_bytewords<8>(bw, gw); break;
+              }
               store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
-              if (kFlat && p.ws_out) chain_store(p, jb, oimg, oh, ow, ch0, gw, out_bits);
+              if (kFlat && p.ws_out) chain_store_bytes(p, jb, oimg, oh, ow, ch0, bw);
             }
           }
         }

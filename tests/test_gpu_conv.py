@@ -328,3 +328,29 @@ def test_wide_operands_exact_at_the_bound():
     assert used == 4
     assert_same(got, want, 64, 32, "wide exactness")
     assert np.abs(want.view(np.int32)).max() > (1 << 26)
+
+
+@pytest.mark.parametrize("neg_m0", [False, True])
+@pytest.mark.parametrize("pairs", [True, False])
+def test_two_bit_requant_edges(neg_m0, pairs):
+    """2-bit outputs on the workspace path at the edges of Eq. 2's rescale: total shifts
+    R = 31 + shift from 1 to 62 (both the 32-bit form, R >= 33, and the int64 form in one
+    tile), biases up to +-2^29 (codes pinned at 0 or 3 for many channels), and negative
+    multipliers in some channels."""
+    rng = np.random.default_rng(11 + 2 * neg_m0 + pairs)
+    n, h, wd, cin, cout = 2, 9, 13, 256, 256
+    x = synth.act_codes(rng, (n, h, wd, cin), 2)
+    w = synth.weight_codes(rng, (cout, 3, 3, cin), 2)
+    m0 = rng.integers(1 << 30, 1 << 31, size=(1, cout), dtype=np.int64).astype(np.int32)
+    sh = rng.integers(-30, 32, size=(1, cout)).astype(np.int8)
+    sh[0, :64] = rng.integers(4, 8, size=64)         # a band where codes spread over 0..3
+    b = rng.integers(-(1 << 29), 1 << 29, size=(1, cout)).astype(np.int32)
+    b[0, :64] = rng.integers(-40, 40, size=64)
+    if neg_m0:
+        m0[0, ::7] = -m0[0, ::7]
+    got, want, used = conv_pair(x, 2, w, 2, out_bits=2, m0=m0, shift=sh, bias=b,
+                                path=TC if pairs else TC_NO_PAIR, workspace=True)
+    assert used == (4 if pairs else 3)
+    assert_same(got, want, cout, 2, "2-bit requant edges")
+    codes = oracle_unpack(want, cout, 2)
+    assert len(np.unique(codes[..., :64])) == 4

@@ -223,6 +223,9 @@ __device__ __forceinline__ void general_group(const Params& p, const uint32_t* v
   }
 }
 
+// In the 32-bit forms below, Eq. 2's clip to [0, qmax] is __vimin_s32_relu(x, qmax) =
+// max(min(x, qmax), 0), one min.relu instruction instead of a min and a max.
+
 // Skip epilogue in 32-bit arithmetic (Eq. 6, Eq. 7 with the skip rescaled, Eq. 2) when, for
 // every column of the tile, R = 31 + shift >= 33, |bias| <= 2^30 and d >= 8, and the skip
 // holds k-bit codes (s <= 255): then rhu(s * c, d) = (s * c + 2^(d-1)) >> d fits in int32,
@@ -239,7 +242,7 @@ __device__ __forceinline__ void fast_skip_group(const uint32_t* v, const EpiChan
     const int32_t st = (int32_t)((sc + (1LL << (c.d - 1))) >> c.d);
     const int32_t u = add_sat(acc + c.bias, st);
     const int r = c.r;
-    y[i] = min(max((__mulhi(u, c.m0) + (1 << (r - 33))) >> (r - 32), 0), qmax);
+    y[i] = __vimin_s32_relu((__mulhi(u, c.m0) + (1 << (r - 33))) >> (r - 32), qmax);
   }
 }
 
@@ -259,7 +262,7 @@ __device__ __forceinline__ void fast_skip32_group(const uint32_t* v, const EpiCh
     t = t > 2147483647LL ? 2147483647LL : (t < -2147483648LL ? -2147483648LL : t);
     const int32_t u = (int32_t)t;
     const int r = c.r;
-    y[i] = min(max((__mulhi(u, c.m0) + (1 << (r - 33))) >> (r - 32), 0), qmax);
+    y[i] = __vimin_s32_relu((__mulhi(u, c.m0) + (1 << (r - 33))) >> (r - 32), qmax);
   }
 }
 
@@ -278,7 +281,7 @@ __device__ __forceinline__ void magic_requant_group(const uint32_t* v, const int
   for (int i = 0; i < 32; ++i) {
     const int4 c = f[i];
     const int32_t u = __float_as_int(__fmaf_rn(__uint_as_float(v[i]), 262144.0f, kMagic)) + c.x;
-    const uint32_t y = (uint32_t)min(max((__mulhi(u, c.y) + c.z) >> c.w, 0), qmax);
+    const uint32_t y = (uint32_t)__vimin_s32_relu((__mulhi(u, c.y) + c.z) >> c.w, qmax);
     if constexpr (kOut == 3) {
       gw[i / 16] |= (y & 3u) << (8 * (i % 4) + 2 * ((i % 16) / 4));
       gw[2] |= (y >> 2) << (8 * (i % 4) + i / 4);
@@ -302,7 +305,7 @@ __device__ __forceinline__ void fast_requant_group(const uint32_t* v, const EpiC
     const int32_t acc = __float2int_rn(__uint_as_float(v[i]) * 262144.0f);  // exact integer
     const int32_t u = add_sat(acc, c.bias);
     const int r = c.r;
-    const uint32_t y = (uint32_t)min(max((__mulhi(u, c.m0) + (1 << (r - 33))) >> (r - 32), 0), qmax);
+    const uint32_t y = (uint32_t)__vimin_s32_relu((__mulhi(u, c.m0) + (1 << (r - 33))) >> (r - 32), qmax);
     if constexpr (kOut == 3) {
       gw[i / 16] |= (y & 3u) << (8 * (i % 4) + 2 * ((i % 16) / 4));
       gw[2] |= (y >> 2) << (8 * (i % 4) + i / 4);
@@ -323,7 +326,7 @@ __device__ __forceinline__ void magic_requant_bytes(const uint32_t* v, const int
   for (int i = 0; i < 32; ++i) {
     const int4 c = f[i];
     const int32_t u = __float_as_int(__fmaf_rn(__uint_as_float(v[i]), 262144.0f, kMagic)) + c.x;
-    const uint32_t y = (uint32_t)min(max((__mulhi(u, c.y) + c.z) >> c.w, 0), qmax);
+    const uint32_t y = (uint32_t)__vimin_s32_relu((__mulhi(u, c.y) + c.z) >> c.w, qmax);
     bw[i / 4] += y << (8 * (i % 4));  // codes < 256: the add is an or
   }
 }

@@ -221,7 +221,7 @@ __device__ __forceinline__ void epi_unit(const uint32_t (&v)[32], const int4* cs
       for (int i = 0; i < 32; ++i) {
         const int4 c = cst4[c0 + i];  // bias, M0, 2^(R-33), R-32
         const int32_t u = add_sat(__float2int_rn(__uint_as_float(v[i])), c.x);
-        put_code<kOut>(gw, i, (uint32_t)min(max((__mulhi(u, c.y) + c.z) >> c.w, 0), qmax));
+        put_code<kOut>(gw, i, (uint32_t)__vimin_s32_relu((__mulhi(u, c.y) + c.z) >> c.w, qmax));
       }
     } else {
 #pragma unroll

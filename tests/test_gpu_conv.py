@@ -354,3 +354,35 @@ def test_two_bit_requant_edges(neg_m0, pairs):
     assert_same(got, want, cout, 2, "2-bit requant edges")
     codes = oracle_unpack(want, cout, 2)
     assert len(np.unique(codes[..., :64])) == 4
+
+
+@pytest.mark.parametrize("out_bits", [2, 3, 4, 8])
+@pytest.mark.parametrize("pairs", [True, False])
+def test_k_bit_requant_edges(out_bits, pairs):
+    """Eq. 2's clip at both ends for every code width on the workspace path, in the 32-bit
+    requant form (every R = 31 + shift >= 40 - k here). A band of channels sits at the
+    smallest of those R with biases that spread the codes over the whole range and past
+    both ends of the clip; the others take R up to 62, biases up to +-2^29 and some
+    negative multipliers."""
+    rng = np.random.default_rng(40 + out_bits + 10 * pairs)
+    n, h, wd, cin, cout = 2, 9, 13, 256, 256
+    x = synth.act_codes(rng, (n, h, wd, cin), 2)
+    w = synth.weight_codes(rng, (cout, 3, 3, cin), 2)
+    qmax = (1 << out_bits) - 1
+    r_min = 40 - out_bits
+    m0 = rng.integers(1 << 30, 1 << 31, size=(1, cout), dtype=np.int64).astype(np.int32)
+    sh = rng.integers(r_min - 31, 32, size=(1, cout)).astype(np.int8)
+    b = rng.integers(-(1 << 29), 1 << 29, size=(1, cout)).astype(np.int32)
+    band = slice(0, 96)
+    m0[0, band] = rng.integers((1 << 31) - 4096, 1 << 31, size=96)
+    sh[0, band] = r_min - 31 + rng.integers(0, 2, size=96)
+    step = 1 << (9 - out_bits)            # accumulator units per code at R = r_min
+    b[0, band] = rng.integers(-300, (qmax + 1) * step + 300, size=96)
+    m0[0, 96::7] = -m0[0, 96::7]
+    got, want, used = conv_pair(x, 2, w, 2, out_bits=out_bits, m0=m0, shift=sh, bias=b,
+                                path=TC if pairs else TC_NO_PAIR, workspace=True)
+    assert used == (4 if pairs else 3)
+    assert_same(got, want, cout, out_bits, f"{out_bits}-bit requant edges")
+    codes = oracle_unpack(want, cout, out_bits)[..., band]
+    assert codes.min() == 0 and codes.max() == qmax
+    assert len(np.unique(codes)) == qmax + 1 if out_bits <= 4 else len(np.unique(codes)) > 100

@@ -338,6 +338,47 @@ def run_sweep(args):
                        "workspace" if p.ws_bytes else "no workspace") if kind == "conv" else "pool",
                  last_path=aqd.last_conv_path() if kind == "conv" else None)
 
+    # the standalone element-wise calls (HBM-bound), inputs larger than L2 where the call allows:
+    # requant of an int32 accumulator tensor to 2-bit codes (Eq. 6 + Eq. 2), the integer skip
+    # add of an int32 tensor and a 4-bit code tensor with requant to 2-bit (Eq. 7/8 + Eq. 2), and
+    # config 3's 3x3 stride-2 max-pool on 4-bit codes (Sec. 3.2.4)
+    if want in ("all", "eltwise"):
+        hbm = peaks["hbm_gbs"]
+        rng = np.random.default_rng(5)
+        n, h, w, c = 16, 100, 168, 256
+        A = aqd.DTensor.from_codes(torch.from_numpy(rng.integers(-20000, 20000, size=(n, h, w, c),
+                                                                 dtype=np.int32)).to(dev), 32)
+        # the same harness on a plain device copy of the int32 tensor: what this machine's HBM gives
+        # a streaming kernel here (read + write bytes)
+        cp_dst = torch.empty_like(A.data)
+        ms = timed(lambda: cp_dst.copy_(A.data))
+        nb = 2 * A.data.numel()
+        emit("eltwise_reference_torch_copy_int32_16x100x168x256", ms, 0, nb, frac_hbm=nb / (ms * 1e-3) / 1e9 / hbm,
+             hbm_peak_gbs=hbm)
+        del cp_dst
+        m0, sh, b = synth.requant_params(rng, 1, c, calib_std=8000.0, out_bits=2)
+        erq = aqd.RequantParams.from_numpy(m0, sh, b, device=dev)
+        Y2 = aqd.DTensor.empty(n, h, w, c, 2, device=dev)
+        ms = timed(lambda: aqd.requant(A, erq, Y2, stream=stream))
+        nb = n * h * w * c * 4 + n * h * w * aqd.row_bytes(c, 2)
+        emit("eltwise_requant_int32_to_2bit_16x100x168x256", ms, 0, nb, frac_hbm=nb / (ms * 1e-3) / 1e9 / hbm,
+             hbm_peak_gbs=hbm)
+        B4 = aqd.DTensor.from_codes(torch.from_numpy(synth.act_codes(rng, (n, h, w, c), 4)).to(dev), 4)
+        cc, dd = synth.skip_params(rng, 1, c, sh)
+        esp = aqd.SkipParams.from_numpy(cc, dd, device=dev)
+        ms = timed(lambda: aqd.residual_add_int(A, B4, esp, Y2, rq=erq, stream=stream))
+        nb = n * h * w * (c * 4 + aqd.row_bytes(c, 4) + aqd.row_bytes(c, 2))
+        emit("eltwise_residual_add_int32_plus_4bit_to_2bit_16x100x168x256", ms, 0, nb,
+             frac_hbm=nb / (ms * 1e-3) / 1e9 / hbm, hbm_peak_gbs=hbm)
+        del A, B4
+        n, h, w, c = 8, 400, 672, 64
+        X4 = aqd.DTensor.from_codes(torch.from_numpy(synth.act_codes(rng, (n, h, w, c), 4)).to(dev), 4)
+        P4 = aqd.DTensor.empty(n, 200, 336, c, 4, device=dev)
+        ms = timed(lambda: aqd.maxpool_codes(X4, 3, 2, 1, P4, stream=stream))
+        nb = n * (h * w + 200 * 336) * aqd.row_bytes(c, 4)
+        emit("eltwise_maxpool3x3s2_4bit_8x400x672x64", ms, 0, nb, frac_hbm=nb / (ms * 1e-3) / 1e9 / hbm,
+             hbm_peak_gbs=hbm)
+
     # config 4: first tower layer of the head at batch 16, 2/3/4/8-bit
     for bits in ((2, 3, 4, 8) if want in ("all", "config4") else ()):
         wl = synth.config4(bits)
@@ -375,7 +416,7 @@ def main():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--sweep", nargs="?", const="all", default=None, choices=["all", "config0", "config1", "config3", "config4"],
+    ap.add_argument("--sweep", nargs="?", const="all", default=None, choices=["all", "config0", "config1", "config3", "config4", "eltwise"],
                     help="measure the other workloads (several lines)")
     args = ap.parse_args()
     if args.impl == "reference":

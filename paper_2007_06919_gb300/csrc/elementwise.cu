@@ -89,6 +89,163 @@ __global__ void __launch_bounds__(kThreads) eltwise_kernel(const EltArgs a) {
   store_vals(a.y + pix * a.y_row_bytes, a.y_bits, a.c, ch0, out);
 }
 
+// The same operation for whole 32-channel groups (c % 32 == 0), with coalesced traffic and
+// broadcast table reads. A block takes spans of 256 consecutive (pixel, group) units; since
+// c % 32 == 0, unit u's input bytes sit at u * (group bytes) and its output bytes likewise,
+// so a span is one contiguous range of each. All threads copy the span's input into shared
+// memory with consecutive 16-byte loads, each thread works on one unit, and the results
+// leave the same way. When the group count G divides 256, the threads of a warp take units
+// of one channel group (pixel = lane), so the per-channel constants are read as broadcasts.
+// When there is no skip, the output is codes and every channel has R = 31 + shift >= 33,
+// Eq. 6 -> Eq. 2 runs in 32-bit form: u = sat32(a + bias) by a saturating add, and
+// rhu(u * M0, R) = (mulhi(u, M0) + 2^(R-33)) >> (R-32) (the low product word cannot carry
+// into the rounded result); the clip is one min.relu. Otherwise each element takes the
+// int64 epilogue as written.
+constexpr int kTabChannels = 512;  // channels whose constants fit the static shared table
+
+__device__ __forceinline__ int32_t sat_add32(int32_t a, int32_t b) {
+  int32_t r;
+  asm("add.sat.s32 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+
+// Bytes of one (pixel, 32-channel group) unit at `bits` (4 * bits, or 128 for int32).
+__device__ __forceinline__ int unit_bytes(int bits) { return bits == 32 ? 128 : group_bytes(bits); }
+
+// 16-byte slot q of int32 unit u in the staging buffer, rotated by the unit's key so that
+// eight lanes touching eight units, or eight slots of one unit, use eight different bank
+// groups
+__device__ __forceinline__ int stage_slot(int u, int q, int key) { return u * 8 + (q ^ key); }
+
+template <bool kHasSkip>
+__global__ void __launch_bounds__(kThreads, 3) eltwise_group_kernel(const EltArgs a) {
+  __shared__ int4 stage[kThreads * 8];   // 32 KB: one span of int32 units (or of smaller ones)
+  __shared__ EpiChan tab[kTabChannels];  // 8 KB
+  int fast = (!kHasSkip && a.y_bits != 32) ? 1 : 0;
+  for (int ch = threadIdx.x; ch < a.c; ch += kThreads) {
+    const int64_t idx = (int64_t)a.level * a.c + ch;
+    EpiChan ec{};
+    ec.bias = a.bias ? a.bias[idx] : 0;
+    if (a.y_bits != 32) {
+      ec.m0 = a.m0[idx];
+      ec.r = (int8_t)(31 + a.shift[idx]);
+      if (ec.r < 33) fast = 0;
+    }
+    if (kHasSkip) { ec.c = a.skip_c[idx]; ec.d = a.skip_d[idx]; }
+    tab[ch] = ec;
+  }
+  fast = __syncthreads_and(fast);  // also publishes the table
+  const int qmax = (1 << (a.y_bits & 15)) - 1;
+  const int G = a.c / 32;
+  const int64_t total = (int64_t)a.n * a.h * a.w * G;
+  const int tid = threadIdx.x;
+  // this thread's unit within a span, and the staging key of a unit: (unit / G) & 7 when a
+  // warp's lanes take consecutive pixels of one group, else unit & 7
+  const bool by_group = (kThreads % G) == 0;  // G is then a power of two
+  const int lg = by_group ? __ffs(G) - 1 : 0;
+  const int per_group = kThreads / G;
+  const int j = by_group ? (tid % per_group) * G + tid / per_group : tid;
+  auto key = [&](int u) { return by_group ? (u >> lg) & 7 : u & 7; };
+  const int gin = unit_bytes(a.a_bits), gout = unit_bytes(a.y_bits);
+  uint8_t* sbytes = reinterpret_cast<uint8_t*>(stage);
+  for (int64_t base = (int64_t)blockIdx.x * kThreads; base < total; base += (int64_t)gridDim.x * kThreads) {
+    const int nu = (int)(total - base < kThreads ? total - base : kThreads);
+    const bool mine = j < nu;
+    const int64_t t = base + j;
+    // pixels number below 2^31 (checked on the host), units usually too: 32-bit division then
+    const int pix = total <= 0x7FFFFFFF ? (int)t / G : (int)(t / G);
+    const int ch0 = (int)(t - (int64_t)pix * G) * 32;
+    int32_t v[32];
+    if (a.a_bits == 32) {
+      const int4* src = reinterpret_cast<const int4*>(a.a) + base * 8;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int k = tid + i * kThreads;
+        if (k < nu * 8) stage[stage_slot(k >> 3, k & 7, key(k >> 3))] = __ldg(src + k);
+      }
+      __syncthreads();
+      if (mine) {
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const int4 x = stage[stage_slot(j, q, key(j))];
+          v[4 * q] = x.x; v[4 * q + 1] = x.y; v[4 * q + 2] = x.z; v[4 * q + 3] = x.w;
+        }
+      }
+    } else {
+      // packed codes: the span's bytes as 16-byte chunks (a multiple of 4 bytes when partial)
+      const int nbytes = nu * gin;
+      const uint8_t* src = a.a + base * gin;
+      for (int k = tid; k * 16 < nbytes; k += kThreads) {
+        if (k * 16 + 16 <= nbytes) {
+          stage[k] = __ldg(reinterpret_cast<const int4*>(src) + k);
+        } else {
+          for (int b = k * 16; b < nbytes; b += 4)
+            reinterpret_cast<uint32_t*>(sbytes)[b / 4] = __ldg(reinterpret_cast<const uint32_t*>(src) + b / 4);
+        }
+      }
+      __syncthreads();
+      if (mine) unpack_group_vals(sbytes + j * gin, a.a_bits, false, v);
+    }
+    if (mine) {
+      if (!kHasSkip && fast) {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const EpiChan ec = tab[ch0 + i];
+          const int32_t u = sat_add32(v[i], ec.bias);
+          v[i] = __vimin_s32_relu((__mulhi(u, ec.m0) + (1 << (ec.r - 33))) >> (ec.r - 32), qmax);
+        }
+      } else {
+        int32_t sv[32];
+        if (kHasSkip) {
+          const int hw = a.h * a.w;
+          const int img = pix / hw;
+          const int rem = pix - img * hw;
+          const int hh = rem / a.w, ww = rem - (rem / a.w) * a.w;
+          const int64_t sp = ((int64_t)img * a.b_h + hh / a.upsample) * a.b_w + ww / a.upsample;
+          load_vals(a.b + sp * a.b_row_bytes, a.b_bits, a.c, ch0, a.b_bits == 32, sv);
+        }
+#pragma unroll 4
+        for (int i = 0; i < 32; ++i)
+          v[i] = epilogue<kHasSkip>(v[i], kHasSkip ? sv[i] : 0, tab[ch0 + i], a.scale_main, a.y_bits);
+      }
+    }
+    __syncthreads();  // every thread has read its unit from the staging buffer
+    if (a.y_bits == 32) {
+      if (mine) {
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          stage[stage_slot(j, q, key(j))] = make_int4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+      }
+      __syncthreads();
+      int4* dst = reinterpret_cast<int4*>(a.y) + base * 8;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int k = tid + i * kThreads;
+        if (k < nu * 8) dst[k] = stage[stage_slot(k >> 3, k & 7, key(k >> 3))];
+      }
+    } else {
+      if (mine) {
+        uint32_t g[8];
+        pack_group_vals(v, a.y_bits, g);
+        uint32_t* d = reinterpret_cast<uint32_t*>(sbytes + (int64_t)j * gout);
+        for (int w = 0; w < gout / 4; ++w) d[w] = g[w];
+      }
+      __syncthreads();
+      const int nbytes = nu * gout;
+      uint8_t* dst = a.y + base * gout;
+      for (int k = tid; k * 16 < nbytes; k += kThreads) {
+        if (k * 16 + 16 <= nbytes) {
+          reinterpret_cast<int4*>(dst)[k] = stage[k];
+        } else {
+          for (int b = k * 16; b < nbytes; b += 4)
+            reinterpret_cast<uint32_t*>(dst)[b / 4] = reinterpret_cast<const uint32_t*>(sbytes)[b / 4];
+        }
+      }
+    }
+    __syncthreads();  // the staging buffer is free for the next span
+  }
+}
+
 __global__ void __launch_bounds__(kThreads) maxpool_kernel(const PoolArgs a) {
   const int groups = (a.c + 31) / 32;
   const int64_t total = (int64_t)a.n * a.ho * a.wo * groups;
@@ -279,8 +436,20 @@ static int check_launch(const char* what, std::string* err) {
 int launch_elementwise(const EltArgs& a, cudaStream_t stream, std::string* err) {
   const int64_t total = (int64_t)a.n * a.h * a.w * ((a.c + 31) / 32);
   if (total == 0) return 0;
-  if (a.has_skip) elt::eltwise_kernel<true><<<elt::blocks_for(total), elt::kThreads, 0, stream>>>(a);
-  else elt::eltwise_kernel<false><<<elt::blocks_for(total), elt::kThreads, 0, stream>>>(a);
+  if (a.c <= elt::kTabChannels && a.c % 32 == 0) {
+    // enough blocks for every SM several times over; each block stages the constants once
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const unsigned cap = (unsigned)(sms > 0 ? sms : 152) * 6u;
+    const unsigned blocks = elt::blocks_for(total) < cap ? elt::blocks_for(total) : cap;
+    if (a.has_skip) elt::eltwise_group_kernel<true><<<blocks, elt::kThreads, 0, stream>>>(a);
+    else elt::eltwise_group_kernel<false><<<blocks, elt::kThreads, 0, stream>>>(a);
+  } else if (a.has_skip) {
+    elt::eltwise_kernel<true><<<elt::blocks_for(total), elt::kThreads, 0, stream>>>(a);
+  } else {
+    elt::eltwise_kernel<false><<<elt::blocks_for(total), elt::kThreads, 0, stream>>>(a);
+  }
   return check_launch("eltwise launch", err);
 }
 

@@ -41,6 +41,38 @@ def test_requant_matches_oracle(out_bits, c, levels, level):
     assert_same(Y.data.cpu().numpy().reshape(ref.packed.shape), ref.packed, c, out_bits, "requant")
 
 
+@pytest.mark.parametrize("shape,out_bits,shift_range", [
+    ((4, 100, 168, 256), 2, (8, 20)),       # many units per thread (the blocks stride), 32-bit form
+    ((2, 13, 21, 256), 4, (-31, 31)),       # R = 0 .. 62 in one table: the int64 form
+    ((1, 9, 7, 1056), 2, (8, 20)),          # more channels than the staged table holds
+    ((3, 5, 11, 512), 8, (-3, 31)),         # exactly the staged-table limit, some R < 33
+    ((2, 17, 23, 96), 3, (8, 20))])         # 3 channel groups: a warp spans several groups
+def test_requant_forms_and_sizes(shape, out_bits, shift_range):
+    """aqd_requant's forms: the 32-bit form (every R >= 33) over a tensor with several units per
+    thread, the int64 form when some R < 33, the per-element table path past the staged
+    channel limit, and int32 extremes that saturate Eq. 6's sum before the multiply. The
+    int32 input goes through the shared-memory staging of whole 256-unit spans and of a
+    partial last span."""
+    n, h, w, c = shape
+    rng = np.random.default_rng(sum(shape) + out_bits)
+    acc = rng.integers(-30000, 30000, size=shape).astype(np.int32)
+    acc[0, 0, 0, :6] = (2 ** 31 - 1, -2 ** 31, 2 ** 31 - 5, -7, 2 ** 30, -2 ** 30)
+    m0 = rng.integers(1 << 30, 1 << 31, size=(1, c), dtype=np.int64).astype(np.int32)
+    m0[0, ::5] = -m0[0, ::5]
+    sh = rng.integers(shift_range[0], shift_range[1] + 1, size=(1, c)).astype(np.int8)
+    b = rng.integers(-(1 << 30), 1 << 30, size=(1, c)).astype(np.int32)
+    b[0, : c // 2] = rng.integers(-3000, 3000, size=c // 2)
+    ref = oracle.requant(oracle.CodeTensor.from_codes(acc, 32), m0, sh, b, level=0, levels=1, out_bits=out_bits)
+    Y = aqd.DTensor.empty(n, h, w, c, out_bits)
+    Y.data.fill_(0xA5)
+    aqd.requant(to_device(oracle.CodeTensor.from_codes(acc, 32)), aqd.RequantParams.from_numpy(m0, sh, b), Y)
+    torch.cuda.synchronize()
+    assert aqd.device_status() == 0
+    assert_same(Y.data.cpu().numpy().reshape(ref.packed.shape), ref.packed, c, out_bits, f"requant {shape}")
+    codes = oracle.unpack(ref.packed, c, out_bits)
+    assert codes.min() == 0 and codes.max() == (1 << out_bits) - 1
+
+
 @pytest.mark.parametrize("a_bits,b_bits,up,mirror,out_bits,with_rq",
                          [(32, 4, 1, 0, 4, True), (4, 4, 1, 1, 4, True), (32, 32, 2, 0, 2, True),
                           (2, 8, 2, 1, 32, False), (32, 3, 1, 0, 32, True), (8, 4, 1, 0, 3, True)])
@@ -62,6 +94,56 @@ def test_residual_add_matches_oracle(a_bits, b_bits, up, mirror, out_bits, with_
     aqd.residual_add_int(to_device(at), to_device(bt), aqd.SkipParams.from_numpy(cc, dd, up, mirror), Y, rq=rq)
     torch.cuda.synchronize()
     assert_same(Y.data.cpu().numpy().reshape(ref.packed.shape), ref.packed, c, out_bits, "residual")
+
+
+@pytest.mark.parametrize("with_rq,mirror", [(False, 0), (True, 1)])
+def test_residual_add_int32_spans(with_rq, mirror):
+    """The skip add with an int32 main operand over more units than one pass of the grid
+    (blocks take several 256-unit spans, the last one partial), a 2x-upsampled 4-bit skip,
+    and an int32 result staged back through shared memory (without rq) or 4-bit codes."""
+    rng = np.random.default_rng(77 + mirror)
+    n, h, w, c = 8, 100, 167, 64
+    a = rng.integers(-(1 << 30), 1 << 30, size=(n, h, w, c)).astype(np.int32)
+    a[0, 0, 0, :4] = (2 ** 31 - 1, -2 ** 31, 2 ** 31 - 2, -2 ** 31 + 1)
+    b = synth.act_codes(rng, (n, (h + 1) // 2, (w + 1) // 2, c), 4)
+    m0, sh, bias = synth.requant_params(rng, 1, c, calib_std=2.0 ** 29, out_bits=4)
+    cc = rng.integers(1 << 30, 1 << 31, size=(1, c), dtype=np.int64).astype(np.int32)
+    dd = rng.integers(4, 12, size=(1, c)).astype(np.int8)
+    out_bits = 4 if with_rq else 32
+    kw = dict(m0=m0, shift=sh, bias=bias) if with_rq else {}
+    at, bt = oracle.CodeTensor.from_codes(a, 32), oracle.CodeTensor.from_codes(b, 4)
+    ref = oracle.residual_add(at, bt, cc, dd, upsample=2, scale_a=mirror, out_bits=out_bits, **kw)
+    Y = aqd.DTensor.empty(n, h, w, c, out_bits)
+    Y.data.fill_(0xA5)
+    rq = aqd.RequantParams.from_numpy(m0, sh, bias) if with_rq else None
+    aqd.residual_add_int(to_device(at), to_device(bt), aqd.SkipParams.from_numpy(cc, dd, 2, mirror), Y, rq=rq)
+    torch.cuda.synchronize()
+    assert aqd.device_status() == 0
+    assert_same(Y.data.cpu().numpy().reshape(ref.packed.shape), ref.packed, c, out_bits, "residual spans")
+
+
+@pytest.mark.parametrize("c,a_bits,b_bits,out_bits", [(160, 4, 32, 2), (96, 8, 2, 32), (256, 3, 4, 4)])
+def test_residual_add_packed_main_operand(c, a_bits, b_bits, out_bits):
+    """The skip add with packed codes as the main operand (their bytes staged through shared
+    memory as one range per span), channel counts whose group count divides the block
+    (256) or not, and code, int32 or code outputs."""
+    rng = np.random.default_rng(c + a_bits + b_bits)
+    n, h, w = 3, 31, 45
+    a = synth.act_codes(rng, (n, h, w, c), a_bits)
+    b = (rng.integers(-8, 8, size=(n, h, w, c)) if b_bits == 32 else
+         synth.act_codes(rng, (n, h, w, c), b_bits)).astype(np.int32)
+    m0, sh, bias = synth.requant_params(rng, 1, c, calib_std=40.0, out_bits=min(out_bits, 8))
+    cc, dd = synth.skip_params(rng, 1, c, sh)
+    kw = dict(m0=m0, shift=sh, bias=bias) if out_bits != 32 else {}
+    at, bt = oracle.CodeTensor.from_codes(a, a_bits), oracle.CodeTensor.from_codes(b, b_bits)
+    ref = oracle.residual_add(at, bt, cc, dd, upsample=1, scale_a=0, out_bits=out_bits, **kw)
+    Y = aqd.DTensor.empty(n, h, w, c, out_bits)
+    Y.data.fill_(0xA5)
+    rq = aqd.RequantParams.from_numpy(m0, sh, bias) if out_bits != 32 else None
+    aqd.residual_add_int(to_device(at), to_device(bt), aqd.SkipParams.from_numpy(cc, dd), Y, rq=rq)
+    torch.cuda.synchronize()
+    assert aqd.device_status() == 0
+    assert_same(Y.data.cpu().numpy().reshape(ref.packed.shape), ref.packed, c, out_bits, "residual packed main")
 
 
 # 16-byte units (4-bit 64 / 96 ch, 2-bit 256 ch, 8-bit 32 ch), single words (2-bit 32 ch: 8-byte

@@ -145,11 +145,9 @@ __device__ __forceinline__ TileInfo tile_info(const Params& p, int t) {
 
 // ---------------------------------------------------------------- epilogue, general case
 
-// Eq. 6 -> Eq. 7 -> Eq. 2 in int64 for 32 accumulators of one row (any shift, any skip).
-// Kept out of line: the common cases take the 32-bit fast path in the kernel body.
-// Eq. 6 -> Eq. 7 -> Eq. 2 in int64 for 32 accumulators of one row (any shift, any skip),
-// all in registers: the 32 skip values are loaded and unpacked per skip width, every index
-// is static, and nothing goes through local memory.
+// The skip values of one row's 32-channel group (Eq. 7's second operand), loaded and
+// unpacked per skip width into registers: every index is static, nothing goes through
+// local memory. Channels past cout read 0.
 __device__ __forceinline__ void load_skip_group(const Params& p, const uint8_t* srow, int ch0, int ncols,
                                                 int32_t (&sk)[32]) {
 #pragma unroll
@@ -203,6 +201,8 @@ __device__ __forceinline__ void load_skip_group(const Params& p, const uint8_t* 
   }
 }
 
+// Eq. 6 -> Eq. 7 -> Eq. 2 in int64 for 32 accumulators of one row (any shift, any skip),
+// element by element as the definition states it; the common cases take 32-bit forms.
 template <bool kSkip, bool kIntAcc = false>
 __device__ __forceinline__ void general_group(const Params& p, const uint32_t* v, const EpiChan* ep,
                                               const uint8_t* srow, int ch0, int ncols, int32_t (&out)[32]) {
@@ -270,28 +270,6 @@ __device__ __forceinline__ void fast_skip32_group(const uint32_t* v, const EpiCh
 constexpr float kMagic = 12582912.0f;
 constexpr uint32_t kMagicBits = 0x4B400000u;
 
-// Fastest requant (no skip, R >= 33, |acc| < 2^22, |bias| <= 2^30): the accumulator float
-// acc * 2^-18 becomes the int32 acc + 0x4B400000 with one FMA; c.x holds bias - 0x4B400000,
-// so one add gives acc + bias exactly (no int32 overflow under the stated bounds).
-template <int kOut>
-__device__ __forceinline__ void magic_requant_group(const uint32_t* v, const int4* f, int qmax, uint32_t gw[8]) {
-#pragma unroll
-  for (int w = 0; w < 8; ++w) gw[w] = 0u;
-#pragma unroll
-  for (int i = 0; i < 32; ++i) {
-    const int4 c = f[i];
-    const int32_t u = __float_as_int(__fmaf_rn(__uint_as_float(v[i]), 262144.0f, kMagic)) + c.x;
-    const uint32_t y = (uint32_t)__vimin_s32_relu((__mulhi(u, c.y) + c.z) >> c.w, qmax);
-    if constexpr (kOut == 3) {
-      gw[i / 16] |= (y & 3u) << (8 * (i % 4) + 2 * ((i % 16) / 4));
-      gw[2] |= (y >> 2) << (8 * (i % 4) + i / 4);
-    } else {
-      constexpr int q = 32 / kOut;
-      gw[i / q] |= y << (8 * (i % 4) + kOut * ((i % q) / 4));
-    }
-  }
-}
-
 // Fast requant of 32 accumulators of one row into one packed group (no skip, R >= 33,
 // any bias): u = sat32(acc + bias), y = clamp((mulhi(u, M0) + 2^(R-33)) >> (R-32), 0, 2^k-1).
 template <int kOut>
@@ -316,9 +294,12 @@ __device__ __forceinline__ void fast_requant_group(const uint32_t* v, const EpiC
   }
 }
 
-// Codes of 32 channels as 8 byte-words (word j holds channels 4j..4j+3, one code per byte):
-// the layout of the chained byte image, and one step from every packed layout.
-// Fastest requant (as magic_requant_group) straight into byte-words.
+// Fastest requant (no skip, R >= 33, |acc| < 2^22, |bias| <= 2^30) of 32 accumulators of one
+// row, straight into 8 byte-words (word j holds channels 4j..4j+3, one code per byte: the
+// layout of the chained byte image, and one step from every packed layout). One FMA turns
+// the accumulator float acc * 2^-18 into the int32 acc + 0x4B400000; c.x holds
+// bias - 0x4B400000, so one add gives acc + bias exactly (no int32 overflow under the stated
+// bounds); c.y, c.z, c.w are M0, 2^(R-33) and R-32.
 __device__ __forceinline__ void magic_requant_bytes(const uint32_t* v, const int4* f, int qmax, uint32_t (&bw)[8]) {
 #pragma unroll
   for (int j = 0; j < 8; ++j) bw[j] = 0u;

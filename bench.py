@@ -130,6 +130,39 @@ def oracle_tower_sample(wl, max_levels=None):
     return ops, time.perf_counter() - t0
 
 
+# The oracle on config 0 (one 3x3 64->64 conv) or config 1 (the bottleneck block, its third
+# conv adding the block input through Eq. 7), timed in a fresh interpreter so that its
+# OpenMP thread count can be set; prints "ops seconds".
+_ORACLE_CONFIG_TIMING = r"""
+import sys, time
+import oracle
+from paper_2007_06919_gb300 import synth
+which = sys.argv[1]
+wl = synth.config0() if which == "config0" else synth.config1()
+x = oracle.CodeTensor.from_codes(wl.inputs[0], wl.bits)
+inp, ops, t0 = x, 0, time.perf_counter()
+for i, cv in enumerate(wl.convs):
+    wp = oracle.pack(cv.w.reshape(-1, cv.cin), cv.w_bits)
+    skip = dict(skip=inp, skip_c=cv.skip_c, skip_d=cv.skip_d) if cv.skip_c is not None else {}
+    y = oracle.conv_int(x, wp, cv.w_bits, 0, cv.kh, cv.kw, cv.stride, cv.pad, cv.cout, m0=cv.m0, shift=cv.shift,
+                        bias=cv.bias, levels=1, out_bits=cv.out_bits, **skip)
+    ops += 2 * y.n * y.h * y.w * cv.cout * cv.kh * cv.kw * cv.cin
+    x = y
+print(ops, time.perf_counter() - t0)
+"""
+
+
+def oracle_config_timing(which: str, threads: int) -> tuple[float, float]:
+    """(ops, seconds) of the CPU oracle on `which` ("config0" or "config1") with `threads`
+    OpenMP threads, run in a child interpreter that never touches the GPU."""
+    env = dict(os.environ, OMP_NUM_THREADS=str(threads))
+    here = os.path.dirname(os.path.abspath(__file__))
+    r = subprocess.run([sys.executable, "-c", _ORACLE_CONFIG_TIMING, which], env=env, cwd=here,
+                       capture_output=True, text=True, check=True)
+    ops, secs = r.stdout.split()[-2:]
+    return float(ops), float(secs)
+
+
 def max_over_ranks(x: float, device) -> float:
     """The largest x over all ranks (the job's time is its slowest replica's)."""
     import torch
@@ -255,9 +288,18 @@ def run_sweep(args):
     y = aqd.DTensor.empty(1, 32, 32, 64, 2, device=dev)
     W = aqd.ConvWeights(torch.from_numpy(cv.w).to(dev), 2)
     rq = aqd.RequantParams.from_numpy(cv.m0, cv.shift, cv.bias, device=dev)
+    def cpu_oracle(which):
+        """The oracle on the same config, all host cores and one core (TOPS)."""
+        out = {}
+        for nm, th in (("all_cores", omp_threads()), ("one_core", 1)):
+            o, t = oracle_config_timing(which, th)
+            out[nm] = {"threads": th, "TOPS": o / t / 1e12, "seconds": t}
+        return out
+
     if want in ("all", "config0"):
         ms = timed(lambda: aqd.conv_int(x, W, 1, 1, y, rq=rq, stream=stream))
-        emit("config0_conv3x3_64_32x32_b1_2bit", ms, 2 * 1024 * 64 * 576, 8192 + 8192 + 64 * 576 // 4)
+        emit("config0_conv3x3_64_32x32_b1_2bit", ms, 2 * 1024 * 64 * 576, 8192 + 8192 + 64 * 576 // 4,
+             cpu_oracle=cpu_oracle("config0"))
 
     # config 1: ResNet-50 C3 bottleneck (1x1 512->128, 3x3 128->128, 1x1 128->512 + identity)
     wl = synth.config1()
@@ -294,7 +336,7 @@ def run_sweep(args):
     if parts_wanted:
         ms = timed(block)
         emit("config1_r50_c3_bottleneck_b2_100x152_4bit", ms, ops, nbytes, images_per_s=n / (ms * 1e-3),
-             launches=4)
+             launches=4, cpu_oracle=cpu_oracle("config1"))
     parts = [("expand_x", lambda: aqd.conv_expand_input([(x, None, None, 0)], Ws[0], 1, 0, wsx, stream=stream), 0),
              ("conv1x1_512_128", lambda: aqd.conv_int_grouped_chain([(x, t1, None, 0)], Ws[0], 1, 0, rq=rqs[0],
                                                                     workspace=wsx, next_pad=1, next_workspace=ws1,

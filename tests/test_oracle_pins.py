@@ -438,3 +438,128 @@ def test_maxpool_commutes_with_dequant(oracle_mod):
     alpha = 0.37
     want = fq.maxpool_real(x * alpha, 3, 2, 1)
     np.testing.assert_allclose(y * alpha, want, rtol=0, atol=1e-12)
+
+
+# ------------------------------------------------------------------ Eq. 7 with Sec. 3.2.4's 2x up-read
+
+
+def _dyadic_upsample_case(rng, b, cin, cout, n, h, w):
+    """Codes and dyadic scales for an exact float64 restatement of Eq. 4 -> Eq. 7 -> Eq. 2 in
+    which the skip is the coarser map of the FPN top-down path, read through nearest 2x
+    upsampling. h and w are odd and differ, so a swapped or ceil-rounded up-index fails."""
+    x = synth.act_codes(rng, (n, h, w, cin), b)
+    wt = synth.weight_codes(rng, (cout, 3, 3, cin), b)
+    skip = synth.act_codes(rng, (n, (h + 1) // 2, (w + 1) // 2, cout), b)
+    s_int = rng.integers(-40, 40, cout)
+    k_mult = rng.integers(1, 16, cout) * 2.0 ** -6     # M0 / 2^R, four significant bits
+    j = rng.integers(1, 4, cout)                        # integer ratio of the two scales
+    return x, wt, skip, s_int, k_mult, j
+
+
+def _multipliers(oracle_mod, k_mult):
+    cout = k_mult.size
+    m0 = np.zeros((1, cout), np.int64)
+    shift = np.zeros((1, cout), np.int64)
+    for i in range(cout):
+        m0[0, i], shift[0, i] = oracle_mod.quantize_multiplier(k_mult[i])
+        assert Fraction(int(m0[0, i]), 2 ** (31 + int(shift[0, i]))) == Fraction(k_mult[i])
+    return m0, shift
+
+
+def _eq7_real(acc_real, s_int, skip_up, j, k_mult, mirror, b):
+    """Eq. 7's real sum quantized by Eq. 2 (nu_next = 2^b - 1, so Eq. 2's scale is 1).
+    Default direction: the skip is in units j * alpha_z of the main branch's scale alpha_z.
+    Mirror: the main branch is in units j * alpha_s of the skip's scale alpha_s. The
+    output multiplier is k_mult per unit of the finer scale in both cases."""
+    if mirror:
+        y_real = ((acc_real + s_int) * j + skip_up) * k_mult
+    else:
+        y_real = (acc_real + s_int + skip_up * j) * k_mult
+    return fq.quantize_act_exact(y_real, float((1 << b) - 1), b)
+
+
+@pytest.mark.parametrize("mirror", [0, 1])
+def test_conv_upsample2_skip_exact_fake_quant(oracle_mod, mirror):
+    """Sec. 3.2.4's FPN top-down add as Eq. 7 inside the conv epilogue: the skip tensor is
+    the coarser map, read at (ho // 2, wo // 2) by nearest upsampling. The float64
+    restatement upsamples with numpy (repeat along H and W), crops to the output and adds
+    in real arithmetic; with dyadic scales each float step is exact, so the oracle's codes
+    must match exactly on an odd, non-square output (9 x 13)."""
+    rng = np.random.default_rng(40 + mirror)
+    b, cin, cout, n, h, w = 4, 32, 32, 2, 9, 13
+    x, wt, skip, s_int, k_mult, j = _dyadic_upsample_case(rng, b, cin, cout, n, h, w)
+    alpha_x, alpha_w = 2.0 ** -3, 2.0 ** -5
+    acc_real = fq.conv2d_real(x * alpha_x, wt * alpha_w, 1, 1) / (alpha_x * alpha_w)
+    skip_up = fq.upsample_nearest2(skip)[:, :h, :w, :]
+    want = _eq7_real(acc_real, s_int, skip_up, j, k_mult, mirror, b)
+    m0, shift = _multipliers(oracle_mod, k_mult)
+    got = oracle_mod.conv_int(oracle_mod.CodeTensor.from_codes(x, b), _pack_w(oracle_mod, wt, b), b, 0, 3, 3, 1, 1,
+                              cout, m0=m0, shift=shift, bias=s_int[None],
+                              skip=oracle_mod.CodeTensor.from_codes(skip, b), skip_c=j[None] * 4,
+                              skip_d=np.full((1, cout), 2), upsample=2, scale_main=mirror, out_bits=b).codes()
+    assert (got == want).all()
+    assert len(np.unique(got)) > 4
+    # the up-read matters here: the same call without it (skip at full resolution, rows
+    # and columns repeated by hand) gives the same codes, and a skip that is not repeated
+    # does not
+    full = np.ascontiguousarray(skip_up)
+    again = oracle_mod.conv_int(oracle_mod.CodeTensor.from_codes(x, b), _pack_w(oracle_mod, wt, b), b, 0, 3, 3, 1, 1,
+                                cout, m0=m0, shift=shift, bias=s_int[None],
+                                skip=oracle_mod.CodeTensor.from_codes(full, b), skip_c=j[None] * 4,
+                                skip_d=np.full((1, cout), 2), upsample=1, scale_main=mirror, out_bits=b).codes()
+    assert (again == want).all()
+
+
+@pytest.mark.parametrize("mirror", [0, 1])
+def test_residual_add_upsample2_exact_fake_quant(oracle_mod, mirror):
+    """The standalone integer skip add (Eq. 7, then Eq. 2) with the coarser operand read by
+    nearest 2x upsampling, against the float64 restatement (numpy repeat, crop, real add)."""
+    rng = np.random.default_rng(42 + mirror)
+    b, c, n, h, w = 3, 64, 2, 7, 11
+    acc = rng.integers(-3000, 3000, size=(n, h, w, c)).astype(np.int32)
+    skip = synth.act_codes(rng, (n, (h + 1) // 2, (w + 1) // 2, c), b)
+    s_int = rng.integers(-40, 40, c)
+    k_mult = rng.integers(1, 16, c) * 2.0 ** -9
+    j = rng.integers(1, 4, c)
+    want = _eq7_real(acc.astype(np.float64), s_int, fq.upsample_nearest2(skip)[:, :h, :w, :], j, k_mult, mirror, b)
+    m0, shift = _multipliers(oracle_mod, k_mult)
+    got = oracle_mod.residual_add(oracle_mod.CodeTensor.from_codes(acc, 32), oracle_mod.CodeTensor.from_codes(skip, b),
+                                  j[None] * 8, np.full((1, c), 3), upsample=2, scale_a=mirror, m0=m0, shift=shift,
+                                  bias=s_int[None], out_bits=b).codes()
+    assert (got == want).all()
+    assert len(np.unique(got)) > 3
+
+
+# ------------------------------------------------------------------ the sampled-pixel entry
+
+
+@pytest.mark.parametrize("stride,upsample", [(1, 2), (2, 1)])
+def test_conv_int_pixels_matches_definition(oracle_mod, stride, upsample):
+    """conv_int_pixels (the oracle's entry for sampled output pixels, flattened as
+    (image, ho, wo) in row-major order) gives, at any list of pixels (unsorted, repeated,
+    from every image, at the ragged borders), the codes of the float64 restatement at those
+    pixels, and the same rows as the full convolution."""
+    rng = np.random.default_rng(44 + stride)
+    b, cin, cout, n, h, w = 4, 32, 64, 3, 9, 13
+    x, wt, _, s_int, k_mult, j = _dyadic_upsample_case(rng, b, cin, cout, n, h, w)
+    ho, wo = (h + 2 - 3) // stride + 1, (w + 2 - 3) // stride + 1
+    skip = synth.act_codes(rng, (n, (ho + upsample - 1) // upsample, (wo + upsample - 1) // upsample, cout), b)
+    alpha_x, alpha_w = 2.0 ** -3, 2.0 ** -5
+    acc_real = fq.conv2d_real(x * alpha_x, wt * alpha_w, stride, 1) / (alpha_x * alpha_w)
+    skip_up = (fq.upsample_nearest2(skip) if upsample == 2 else skip)[:, :ho, :wo, :]
+    want = _eq7_real(acc_real, s_int, skip_up, j, k_mult, 0, b).reshape(n * ho * wo, cout)
+    m0, shift = _multipliers(oracle_mod, k_mult)
+    total = n * ho * wo
+    corners = [0, wo - 1, (ho - 1) * wo, total - 1, ho * wo, ho * wo + wo - 1, 2 * ho * wo + 3]
+    pix = np.concatenate([rng.permutation(total)[:40], corners, corners[:3]])
+    rng.shuffle(pix)
+    kw = dict(m0=m0, shift=shift, bias=s_int[None], skip=oracle_mod.CodeTensor.from_codes(skip, b),
+              skip_c=j[None] * 4, skip_d=np.full((1, cout), 2), upsample=upsample, out_bits=b)
+    xt = oracle_mod.CodeTensor.from_codes(x, b)
+    wp = _pack_w(oracle_mod, wt, b)
+    got = oracle_mod.conv_int_pixels(xt, wp, b, 0, 3, 3, stride, 1, cout, pix, **kw)
+    assert got.shape == (pix.size, cout)
+    assert (got == want[pix]).all()
+    full = oracle_mod.conv_int(xt, wp, b, 0, 3, 3, stride, 1, cout, **kw).codes().reshape(total, cout)
+    assert (got == full[pix]).all()
+    assert len(np.unique(got)) > 4

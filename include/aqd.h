@@ -143,6 +143,18 @@ aqd_status aqd_device_status(aqd_stream_t stream, int32_t* code);
 int32_t aqd_set_conv_path(int32_t path);
 int32_t aqd_last_conv_path(void);
 
+/* Diagnostics (the paper has no counterpart): exercises the device-side failure path that
+ * every tensor-core kernel uses, without faulting anything. One thread waits, with the
+ * kernels' bounded mbarrier wait shortened to 2 ms, on a barrier that nobody arrives at; the
+ * wait expires and latches AQD_ERR_TIMEOUT in the device status word; a second thread,
+ * waiting the kernels' full 1 s limit on another such barrier, leaves through the kernel's
+ * shared abort flag. out: 5 int64 in device memory, written by the kernel:
+ * [0] 1 if the short wait expired, [1] its duration in ns, [2] 1 if the second wait
+ * returned without its phase, [3] its duration in ns, [4] 1 if a control barrier whose
+ * phase completed was seen as complete. The next aqd_device_status() returns
+ * AQD_ERR_TIMEOUT once and clears it. */
+aqd_status aqd_selftest_wait_timeout(int64_t* out, aqd_stream_t stream);
+
 /* ---- codes <-> int32 ----------------------------------------------------------- */
 
 /* Packs rows x c int32 codes (device) into the k-bit layout (low k bits of each value;
@@ -242,8 +254,13 @@ aqd_status aqd_conv_int_grouped_chain(const aqd_conv_job* jobs, int32_t njobs,
  * stream capture. Every call on a device shares the one array: calls that overlap in time
  * (other streams, other host threads) race on it and must be ordered by the caller;
  * nothing in it needs to start at zero (each call writes every byte it reads).
- * Returns AQD_ERR_UNSUPPORTED, launching nothing, when the workspace path does not apply
- * (aqd_conv_workspace_bytes would be 0) or needs more than AQD_STATIC_WORKSPACE_BYTES. */
+ * The array's address is looked up once per (device, context): a context created later on
+ * the same device (after cudaDeviceReset) gets its own lookup on its first call.
+ * Argument errors return AQD_ERR_INVALID as aqd_conv_int does. Returns AQD_ERR_UNSUPPORTED,
+ * launching nothing, whenever the call would not run on the workspace path: the path does
+ * not apply (aqd_conv_workspace_bytes would be 0), the kernel choice would take a kernel
+ * that reads no workspace (8-bit codes with a skip, or a forced CUDA-core path), or the
+ * problem needs more than AQD_STATIC_WORKSPACE_BYTES. */
 aqd_status aqd_conv_int_static_workspace(const aqd_tensor* x, const aqd_conv_weights* w, int32_t stride,
                                          int32_t pad, int32_t level, const aqd_requant_params* rq,
                                          const aqd_tensor* skip, const aqd_skip_params* sp, aqd_tensor* y,

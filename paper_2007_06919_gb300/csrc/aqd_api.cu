@@ -26,26 +26,65 @@ static aqd_status fail(aqd_status s, const std::string& msg) {
   return s;
 }
 
-// Device address of the status word, looked up once per device.
-static uint32_t* status_ptr(std::string* err) {
-  static std::mutex mu;
-  static uint32_t* ptrs[64] = {nullptr};
+// Current CUDA context (driver handle, fetched through the runtime's entry-point query so
+// the library needs no link against libcuda); NULL if none is current or the query fails.
+typedef int (*CtxGetCurrentFn)(void**);
+static void* current_context() {
+  static CtxGetCurrentFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<CtxGetCurrentFn>(p);
+  });
+  void* ctx = nullptr;
+  if (fn && fn(&ctx) != 0) ctx = nullptr;
+  return ctx;
+}
+
+// Device address of a __device__ symbol, looked up with that device current and cached per
+// (device, context): a context created later on the same device (after cudaDeviceReset,
+// say) loads the module again at another address, so it gets its own lookup.
+struct SymbolCache {
+  std::mutex mu;
+  struct Entry { int dev; void* ctx; void* ptr; } e[64];
+  int n = 0;
+};
+static void* symbol_ptr(SymbolCache& c, const void* symbol, const char* what, std::string* err) {
   int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+  if (cudaGetDevice(&dev) != cudaSuccess) {
     *err = "cudaGetDevice failed";
     return nullptr;
   }
-  std::lock_guard<std::mutex> lk(mu);
-  if (!ptrs[dev]) {
-    void* p = nullptr;
-    cudaError_t e = cudaGetSymbolAddress(&p, g_status_word);
-    if (e != cudaSuccess) {
-      *err = std::string("cudaGetSymbolAddress(status): ") + cudaGetErrorString(e);
+  void* ctx = current_context();
+  if (!ctx) {
+    // no context yet on this thread (first CUDA use): make the device's primary context
+    // current, so the context read here is the one the lookup and the later launches use
+    if (cudaFree(nullptr) != cudaSuccess) {
+      *err = "no usable CUDA context";
       return nullptr;
     }
-    ptrs[dev] = static_cast<uint32_t*>(p);
+    ctx = current_context();
   }
-  return ptrs[dev];
+  std::lock_guard<std::mutex> lk(c.mu);
+  for (int i = 0; i < c.n; ++i)
+    if (c.e[i].dev == dev && c.e[i].ctx == ctx) return c.e[i].ptr;
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, symbol);
+  if (e != cudaSuccess) {
+    *err = std::string("cudaGetSymbolAddress(") + what + "): " + cudaGetErrorString(e);
+    return nullptr;
+  }
+  const int slot = c.n < 64 ? c.n++ : (int)(((uintptr_t)ctx >> 4) % 64);  // more than 64: overwrite one
+  c.e[slot] = {dev, ctx, p};
+  return p;
+}
+
+static uint32_t* status_ptr(std::string* err) {
+  static SymbolCache cache;
+  return static_cast<uint32_t*>(symbol_ptr(cache, (const void*)&g_status_word, "status", err));
 }
 
 WeightGeom weight_geom(int32_t cout, int32_t kh, int32_t kw, int32_t cin) {
@@ -149,6 +188,15 @@ int32_t aqd_set_conv_path(int32_t path) {
 }
 
 int32_t aqd_last_conv_path(void) { return g_last_path; }
+
+aqd_status aqd_selftest_wait_timeout(int64_t* out, aqd_stream_t stream) {
+  if (!out || (reinterpret_cast<uintptr_t>(out) & 7) != 0) return fail(AQD_ERR_INVALID, "out must be an 8-byte aligned device pointer");
+  std::string err;
+  uint32_t* sp = status_ptr(&err);
+  if (!sp) return fail(AQD_ERR_CUDA, err);
+  const int st = launch_wait_selftest(sp, out, static_cast<cudaStream_t>(stream), &err);
+  return st ? fail((aqd_status)st, err) : AQD_OK;
+}
 
 aqd_status aqd_pack_codes(const int32_t* codes, int64_t rows, int32_t c, int32_t bits, void* out,
                           aqd_stream_t stream) {
@@ -266,7 +314,8 @@ struct ChainOut {
 static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
                                int32_t stride, int32_t pad, const aqd_requant_params* rq,
                                const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
-                               aqd_stream_t stream, ConvStage stage, const ChainOut* chain = nullptr);
+                               aqd_stream_t stream, ConvStage stage, const ChainOut* chain = nullptr,
+                               bool require_ws = false);
 
 aqd_status aqd_conv_int_grouped(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
                                 int32_t stride, int32_t pad, const aqd_requant_params* rq,
@@ -319,7 +368,8 @@ aqd_status aqd_conv_int_grouped_chain(const aqd_conv_job* jobs, int32_t njobs, c
 static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
                                int32_t stride, int32_t pad, const aqd_requant_params* rq,
                                const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
-                               aqd_stream_t stream, ConvStage stage, const ChainOut* chain) {
+                               aqd_stream_t stream, ConvStage stage, const ChainOut* chain,
+                               bool require_ws) {
   std::string err;
   if (!jobs || njobs <= 0 || njobs > kMaxJobs) return fail(AQD_ERR_INVALID, "njobs must be 1..8");
   if (!check_weights(w, &err)) return fail(AQD_ERR_INVALID, err);
@@ -430,6 +480,9 @@ static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aq
   }
   if (path == 1 && !tc_ok && !a.ws) path = 2;  // the split form exists only on the workspace path
   if (path == 2 && !direct_ok) return fail(AQD_ERR_UNSUPPORTED, "accumulator bound exceeds int32");
+  // a caller that gave the library's own workspace wants the workspace path or nothing
+  if (require_ws && (path != 1 || !a.ws))
+    return fail(AQD_ERR_UNSUPPORTED, "this convolution does not run on the expanded-activation workspace path");
   if (stage != kStageBoth) {
     if (path != 1) return fail(AQD_ERR_UNSUPPORTED, "the tensor-core kernel does not take this convolution");
     if (!workspace) return fail(AQD_ERR_INVALID, "the workspace must not be NULL");
@@ -555,24 +608,8 @@ aqd_status aqd_maxpool_codes(const aqd_tensor* x, int32_t k, int32_t stride, int
 static __device__ __align__(256) uint8_t g_static_ws[AQD_STATIC_WORKSPACE_BYTES];
 
 static uint8_t* static_ws_ptr(std::string* err) {
-  static std::mutex mu;
-  static uint8_t* ptrs[64] = {nullptr};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
-    *err = "cudaGetDevice failed";
-    return nullptr;
-  }
-  std::lock_guard<std::mutex> lk(mu);
-  if (!ptrs[dev]) {
-    void* p = nullptr;
-    const cudaError_t e = cudaGetSymbolAddress(&p, g_static_ws);
-    if (e != cudaSuccess) {
-      *err = std::string("cudaGetSymbolAddress(static workspace): ") + cudaGetErrorString(e);
-      return nullptr;
-    }
-    ptrs[dev] = static_cast<uint8_t*>(p);
-  }
-  return ptrs[dev];
+  static SymbolCache cache;
+  return static_cast<uint8_t*>(symbol_ptr(cache, (const void*)g_static_ws, "static workspace", err));
 }
 
 extern "C" {
@@ -581,19 +618,30 @@ aqd_status aqd_conv_int_static_workspace(const aqd_tensor* x, const aqd_conv_wei
                                          int32_t pad, int32_t level, const aqd_requant_params* rq,
                                          const aqd_tensor* skip, const aqd_skip_params* sp, aqd_tensor* y,
                                          aqd_stream_t stream) {
+  // argument errors first, as aqd_conv_int reports them: AQD_ERR_INVALID with the cause
+  std::string err;
   if (!x || !y) return fail(AQD_ERR_INVALID, "x and y must not be NULL");
+  if (!check_weights(w, &err)) return fail(AQD_ERR_INVALID, err);
+  if (!check_tensor(x, false, "x", &err) || !check_tensor(y, true, "y", &err)) return fail(AQD_ERR_INVALID, err);
+  if (x->c != w->cin) return fail(AQD_ERR_INVALID, "x.c != weights cin");
+  if (stride <= 0 || pad < 0) return fail(AQD_ERR_INVALID, "stride must be > 0 and pad >= 0");
+  if (skip && !skip->data) return fail(AQD_ERR_INVALID, "skip->data is NULL");
   aqd_conv_job job{};
   job.x = *x;
   job.y = *y;
+  if (skip) job.skip = *skip;
+  job.level = level;
   const size_t need = aqd_conv_workspace_bytes(&job, 1, w, stride, pad);
   if (need == 0) return fail(AQD_ERR_UNSUPPORTED, "the expanded-activation workspace path does not apply");
   if (need > (size_t)AQD_STATIC_WORKSPACE_BYTES)
     return fail(AQD_ERR_UNSUPPORTED, "needs " + std::to_string(need) + " workspace bytes, more than the " +
                                          std::to_string((size_t)AQD_STATIC_WORKSPACE_BYTES) + " of the static one");
-  std::string err;
   uint8_t* ws = static_ws_ptr(&err);
   if (!ws) return fail(AQD_ERR_CUDA, err);
-  return aqd_conv_int(x, w, stride, pad, level, rq, skip, sp, y, ws, (size_t)AQD_STATIC_WORKSPACE_BYTES, stream);
+  // the call runs on the workspace path or is refused before any launch (the shared kernel
+  // choice could otherwise pick a kernel that ignores the workspace, e.g. 8-bit codes with a skip)
+  return conv_grouped(&job, 1, w, stride, pad, rq, sp, ws, (size_t)AQD_STATIC_WORKSPACE_BYTES, stream, kStageBoth,
+                      nullptr, true);
 }
 
 }  // extern "C"

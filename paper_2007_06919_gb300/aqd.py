@@ -57,7 +57,7 @@ EXPORTS = ["aqd_row_bytes", "aqd_quantize_multiplier", "aqd_status_string", "aqd
            "aqd_unpack_codes", "aqd_conv_weights_bytes", "aqd_conv_prepare_weights", "aqd_conv_int",
            "aqd_conv_int_grouped", "aqd_conv_workspace_bytes", "aqd_conv_expand_input",
            "aqd_conv_int_grouped_expanded", "aqd_conv_int_grouped_chain", "aqd_requant", "aqd_residual_add_int",
-           "aqd_maxpool_codes", "aqd_conv_int_static_workspace"]
+           "aqd_maxpool_codes", "aqd_conv_int_static_workspace", "aqd_selftest_wait_timeout"]
 
 _lib = None
 
@@ -108,6 +108,8 @@ def load(build_if_missing: bool = True):
                                                 ctypes.POINTER(_Requant), ctypes.POINTER(_Tensor),
                                                 ctypes.POINTER(_Skip), ctypes.POINTER(_Tensor), vp]
     L.aqd_conv_int_static_workspace.restype = c_int
+    L.aqd_selftest_wait_timeout.argtypes = [vp, vp]
+    L.aqd_selftest_wait_timeout.restype = c_int
     L.aqd_conv_workspace_bytes.restype = ctypes.c_size_t
     L.aqd_conv_workspace_bytes.argtypes = [ctypes.POINTER(_Job), i32, ctypes.POINTER(_Weights), i32, i32]
     L.aqd_requant.argtypes = [ctypes.POINTER(_Tensor), ctypes.POINTER(_Requant), i32, ctypes.POINTER(_Tensor), vp]
@@ -439,6 +441,13 @@ def device_status(stream=None) -> int:
     code = ctypes.c_int32()
     _check(load().aqd_device_status(_stream(stream), ctypes.byref(code)), "aqd_device_status")
     return int(code.value)
+
+
+def selftest_wait_timeout(out: torch.Tensor, stream=None) -> None:
+    """Launches the bounded-wait self-test into ``out`` (5 int64 on the device); see
+    aqd_selftest_wait_timeout."""
+    assert out.dtype == torch.int64 and out.is_cuda and out.numel() >= 5
+    _check(load().aqd_selftest_wait_timeout(_ptr(out), _stream(stream)), "aqd_selftest_wait_timeout")
 
 
 def set_conv_path(path: int) -> int:

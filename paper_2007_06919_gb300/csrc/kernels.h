@@ -116,4 +116,7 @@ struct PoolArgs {
 };
 int launch_maxpool(const PoolArgs& a, cudaStream_t stream, std::string* err);
 
+// the bounded-wait self-test (selftest.cu): out receives 5 int64 values
+int launch_wait_selftest(uint32_t* status, int64_t* out, cudaStream_t stream, std::string* err);
+
 }  // namespace aqd

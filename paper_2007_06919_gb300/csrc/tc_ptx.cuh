@@ -92,9 +92,11 @@ __device__ __forceinline__ bool mbar_poll(uint32_t bar, uint32_t parity, volatil
   return mbar_test(bar, parity) || mbar_poll_slow(bar, parity, abort_flag);
 }
 
-// Bounded wait: false if the deadline passed or another role aborted.
+// Bounded wait: false if the deadline (kLimitNs after the call) passed or another role
+// aborted. The kernels use the 1 s limit; the wait self-test instantiates a short one.
+template <uint64_t kLimitNs = kTimeoutNs>
 static __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
-  const uint64_t deadline = globaltimer() + kTimeoutNs;
+  const uint64_t deadline = globaltimer() + kLimitNs;
   for (uint32_t spin = 1;; ++spin) {
     if (AQD_WAIT_HINT_NS > 0 ? mbar_try_sleep(bar, parity, AQD_WAIT_HINT_NS) : mbar_try(bar, parity)) return true;
     if ((spin & 63) == 0) {
@@ -104,8 +106,9 @@ static __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity
   }
 }
 
+template <uint64_t kLimitNs = kTimeoutNs>
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
-  return mbar_try(bar, parity) || mbar_wait_slow(bar, parity, abort_flag);
+  return mbar_try(bar, parity) || mbar_wait_slow<kLimitNs>(bar, parity, abort_flag);
 }
 
 __device__ __forceinline__ void fail(volatile int* abort_flag, uint32_t* status) {

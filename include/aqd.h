@@ -240,6 +240,41 @@ aqd_status aqd_conv_int_grouped_chain(const aqd_conv_job* jobs, int32_t njobs,
                                       void* workspace, size_t ws_bytes, int32_t next_pad,
                                       void* next_workspace, size_t next_ws_bytes, aqd_stream_t stream);
 
+/* ---- a chained tower, layers overlapped tile by tile -------------------------------- */
+
+/* Bytes of per-tile counters that aqd_conv_int_grouped_tower needs to overlap its layers:
+ * 4 x (layers - 1) x the tiles of one layer (256 output positions of the padded-width grid
+ * per tile). 0 for invalid arguments or a single layer. */
+size_t aqd_conv_tower_sync_bytes(const aqd_conv_job* jobs, int32_t njobs, int32_t layers, int32_t pad);
+
+/* Runs `layers` grouped stride-1 convolutions in a chain, as the shared detector head applies
+ * its tower to every FPN level (Sec. 3.2.2, Fig. 3: one weight set per layer, one parameter
+ * row per level): layer i is Eq. 4 -> Eq. 6 -> Eq. 2 (no skip) of w[i] and rq[i] on layer
+ * i-1's output codes.
+ *   jobs: layers x njobs, row-major: jobs[i * njobs + j] is job j of layer i; its x must be
+ *     jobs[(i-1) * njobs + j].y (same data pointer and shape) for i > 0; skip must be empty.
+ *     Every layer keeps the spatial size: w[i].kh = w[i].kw = 2 pad + 1.
+ *   Layers 0 .. layers-2 write 2/3/4-bit codes (their packed y, and, in the same epilogue,
+ *     the next layer's zero-padded byte image); the last layer any output (int32 heads).
+ *   ws_a, ws_b: two expanded-activation workspaces of ws_bytes each (256-byte aligned, each
+ *     at least aqd_conv_workspace_bytes of every layer); layer i reads ws_a for even i, ws_b
+ *     for odd i. input_expanded == 0: the call expands layer 0's input into ws_a first
+ *     (aqd_conv_expand_input); nonzero: ws_a already holds it (written by that call, or by a
+ *     chained previous layer). The call never writes ws_b's zero border: zero ws_b once
+ *     before its first use.
+ *   sync: device counters of aqd_conv_tower_sync_bytes() bytes (4-byte aligned), cleared on
+ *     `stream` by the call's first kernel. When every layer runs on CTA pairs with
+ *     one output-channel tile (cout <= 256), layer i+1 starts as soon as SMs free up and each
+ *     of its tiles waits (a bounded wait, AQD_ERR_TIMEOUT on expiry) only for the tiles of
+ *     layer i whose rows it reads. With sync NULL, or when that condition fails, each layer
+ *     waits for the whole previous one. Calls that share sync or the workspaces must not
+ *     overlap in time.
+ * Every layer is validated before anything is launched; an error names the layer. */
+aqd_status aqd_conv_int_grouped_tower(const aqd_conv_job* jobs, int32_t njobs, int32_t layers,
+                                      const aqd_conv_weights* w, const aqd_requant_params* rq, int32_t pad,
+                                      void* ws_a, void* ws_b, size_t ws_bytes, void* sync, size_t sync_bytes,
+                                      int32_t input_expanded, aqd_stream_t stream);
+
 /* ---- convolution without a caller workspace ---------------------------------------- */
 
 /* Size of the library's own expanded-activation workspace (16 MiB per device context). */

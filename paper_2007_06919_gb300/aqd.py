@@ -57,7 +57,8 @@ EXPORTS = ["aqd_row_bytes", "aqd_quantize_multiplier", "aqd_status_string", "aqd
            "aqd_unpack_codes", "aqd_conv_weights_bytes", "aqd_conv_prepare_weights", "aqd_conv_int",
            "aqd_conv_int_grouped", "aqd_conv_workspace_bytes", "aqd_conv_expand_input",
            "aqd_conv_int_grouped_expanded", "aqd_conv_int_grouped_chain", "aqd_requant", "aqd_residual_add_int",
-           "aqd_maxpool_codes", "aqd_conv_int_static_workspace", "aqd_selftest_wait_timeout"]
+           "aqd_maxpool_codes", "aqd_conv_int_static_workspace", "aqd_selftest_wait_timeout",
+           "aqd_conv_tower_sync_bytes", "aqd_conv_int_grouped_tower"]
 
 _lib = None
 
@@ -108,6 +109,12 @@ def load(build_if_missing: bool = True):
                                                 ctypes.POINTER(_Requant), ctypes.POINTER(_Tensor),
                                                 ctypes.POINTER(_Skip), ctypes.POINTER(_Tensor), vp]
     L.aqd_conv_int_static_workspace.restype = c_int
+    L.aqd_conv_tower_sync_bytes.restype = ctypes.c_size_t
+    L.aqd_conv_tower_sync_bytes.argtypes = [ctypes.POINTER(_Job), i32, i32, i32]
+    L.aqd_conv_int_grouped_tower.argtypes = [ctypes.POINTER(_Job), i32, i32, ctypes.POINTER(_Weights),
+                                             ctypes.POINTER(_Requant), i32, vp, vp, ctypes.c_size_t, vp,
+                                             ctypes.c_size_t, i32, vp]
+    L.aqd_conv_int_grouped_tower.restype = c_int
     L.aqd_selftest_wait_timeout.argtypes = [vp, vp]
     L.aqd_selftest_wait_timeout.restype = c_int
     L.aqd_conv_workspace_bytes.restype = ctypes.c_size_t
@@ -411,6 +418,29 @@ def conv_int_grouped_chain(jobs, w: ConvWeights, stride: int, pad: int, *, rq: R
                                              ctypes.byref(spc) if spc is not None else None, wsp, wsb,
                                              next_pad, nwp, nwb, _stream(stream)),
            "aqd_conv_int_grouped_chain")
+
+
+def tower_sync_bytes(jobs, layers: int, pad: int) -> int:
+    """Bytes of per-tile counters for conv_int_grouped_tower (jobs: layer 0's jobs)."""
+    return int(load().aqd_conv_tower_sync_bytes(_jobs(jobs), len(jobs), layers, pad))
+
+
+def conv_int_grouped_tower(layer_jobs, ws: list, rqs: list, pad: int, *, ws_a: torch.Tensor,
+                           ws_b: torch.Tensor, sync: torch.Tensor | None, input_expanded: bool = False,
+                           stream=None):
+    """layer_jobs: one list of (x, y, None, level) per layer, layer i's x being layer i-1's y;
+    ws: ConvWeights per layer; rqs: RequantParams per layer. See aqd_conv_int_grouped_tower."""
+    nl, nj = len(layer_jobs), len(layer_jobs[0])
+    arr = _jobs([jb for jobs in layer_jobs for jb in jobs])
+    wd = (_Weights * nl)(*[w.desc for w in ws])
+    rqa = (_Requant * nl)(*[r.c() for r in rqs])
+    wap, wab = _ws(ws_a)
+    wbp, wbb = _ws(ws_b)
+    assert wab == wbb, "ws_a and ws_b must have the same size"
+    sp_, sb = _ws(sync) if sync is not None else (None, 0)
+    _check(load().aqd_conv_int_grouped_tower(arr, nj, nl, wd, rqa, pad, wap, wbp, wab, sp_, sb, int(input_expanded),
+                                             _stream(stream)),
+           "aqd_conv_int_grouped_tower")
 
 
 def requant(acc: DTensor, rq: RequantParams, y: DTensor, *, level: int = 0, stream=None) -> DTensor:

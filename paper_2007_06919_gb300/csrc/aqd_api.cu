@@ -302,8 +302,9 @@ size_t aqd_conv_workspace_bytes(const aqd_conv_job* jobs, int32_t njobs, const a
 // What one grouped call runs on the workspace path: expansion + convolution (the public
 // grouped call), the expansion alone, or the convolution from an already expanded workspace.
 // kStageChain is kStageConvOnly that also writes the output codes, one byte each, as the
-// zero-padded byte image the next stride-1 conv reads.
-enum ConvStage { kStageBoth = 0, kStageExpandOnly = 1, kStageConvOnly = 2, kStageChain = 3 };
+// zero-padded byte image the next stride-1 conv reads; kStageBothChain is kStageBoth that
+// does the same.
+enum ConvStage { kStageBoth = 0, kStageExpandOnly = 1, kStageConvOnly = 2, kStageChain = 3, kStageBothChain = 4 };
 
 struct ChainOut {
   int32_t pad;
@@ -311,65 +312,19 @@ struct ChainOut {
   size_t bytes;
 };
 
-static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
+// A validated grouped convolution, ready to launch.
+struct ConvPlan {
+  ConvArgs a;
+  int path;     // 1 tensor core, 2 CUDA core, 5 stem
+  ConvStage stage;
+};
+
+// Validates one grouped call and decides its kernel; launches nothing. require_ws: the call
+// must run on the expanded-activation workspace path (else AQD_ERR_UNSUPPORTED).
+static aqd_status plan_grouped(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
                                int32_t stride, int32_t pad, const aqd_requant_params* rq,
                                const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
-                               aqd_stream_t stream, ConvStage stage, const ChainOut* chain = nullptr,
-                               bool require_ws = false);
-
-aqd_status aqd_conv_int_grouped(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
-                                int32_t stride, int32_t pad, const aqd_requant_params* rq,
-                                const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
-                                aqd_stream_t stream) {
-  return conv_grouped(jobs, njobs, w, stride, pad, rq, sp, workspace, ws_bytes, stream, kStageBoth);
-}
-
-aqd_status aqd_conv_int_grouped_expanded(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
-                                         int32_t stride, int32_t pad, const aqd_requant_params* rq,
-                                         const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
-                                         aqd_stream_t stream) {
-  return conv_grouped(jobs, njobs, w, stride, pad, rq, sp, workspace, ws_bytes, stream, kStageConvOnly);
-}
-
-aqd_status aqd_conv_expand_input(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
-                                 int32_t stride, int32_t pad, void* workspace, size_t ws_bytes,
-                                 aqd_stream_t stream) {
-  if (!jobs || njobs <= 0 || njobs > kMaxJobs) return fail(AQD_ERR_INVALID, "njobs must be 1..8");
-  if (!workspace) return fail(AQD_ERR_INVALID, "the workspace must not be NULL");
-  // only the inputs matter here: give every job an int32 output of the right shape so the
-  // shared validation accepts it (nothing is written to it)
-  aqd_conv_job tmp[kMaxJobs];
-  for (int j = 0; j < njobs; ++j) {
-    tmp[j] = jobs[j];
-    tmp[j].skip = aqd_tensor{};
-    tmp[j].level = 0;
-    if (w && stride > 0 && pad >= 0) {
-      tmp[j].y.n = jobs[j].x.n;
-      tmp[j].y.h = (jobs[j].x.h + 2 * pad - w->kh) / stride + 1;
-      tmp[j].y.w = (jobs[j].x.w + 2 * pad - w->kw) / stride + 1;
-      tmp[j].y.c = w->cout;
-    }
-    tmp[j].y.bits = 32;
-    tmp[j].y.data = workspace;  // any non-null aligned pointer; never dereferenced
-  }
-  return conv_grouped(tmp, njobs, w, stride, pad, nullptr, nullptr, workspace, ws_bytes, stream,
-                      kStageExpandOnly);
-}
-
-aqd_status aqd_conv_int_grouped_chain(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
-                                      int32_t stride, int32_t pad, const aqd_requant_params* rq,
-                                      const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
-                                      int32_t next_pad, void* next_workspace, size_t next_ws_bytes,
-                                      aqd_stream_t stream) {
-  const ChainOut c{next_pad, next_workspace, next_ws_bytes};
-  return conv_grouped(jobs, njobs, w, stride, pad, rq, sp, workspace, ws_bytes, stream, kStageChain, &c);
-}
-
-static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
-                               int32_t stride, int32_t pad, const aqd_requant_params* rq,
-                               const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
-                               aqd_stream_t stream, ConvStage stage, const ChainOut* chain,
-                               bool require_ws) {
+                               ConvStage stage, const ChainOut* chain, bool require_ws, ConvPlan* plan) {
   std::string err;
   if (!jobs || njobs <= 0 || njobs > kMaxJobs) return fail(AQD_ERR_INVALID, "njobs must be 1..8");
   if (!check_weights(w, &err)) return fail(AQD_ERR_INVALID, err);
@@ -387,7 +342,9 @@ static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aq
     if (sp->scale_main != 0 && sp->scale_main != 1) return fail(AQD_ERR_INVALID, "sp->scale_main must be 0 or 1");
     if (!rq) return fail(AQD_ERR_INVALID, "a skip needs rq (its level count indexes sp's tables)");
   }
-  ConvArgs a{};
+  ConvArgs& a = plan->a;
+  a = ConvArgs{};
+  plan->stage = stage;
   a.njobs = njobs;
   a.cin = w->cin; a.cout = w->cout; a.kh = w->kh; a.kw = w->kw; a.stride = stride; a.pad = pad;
   a.x_bits = jobs[0].x.bits;
@@ -489,7 +446,7 @@ static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aq
     if (!a.ws) return fail(AQD_ERR_INVALID, "the workspace path does not apply, or the workspace is too small");
   }
   a.skip_expand = (stage == kStageConvOnly || stage == kStageChain) ? 1 : 0;
-  if (stage == kStageChain) {
+  if (stage == kStageChain || stage == kStageBothChain) {
     if (!chain || !chain->ws) return fail(AQD_ERR_INVALID, "next_workspace must not be NULL");
     if ((reinterpret_cast<uintptr_t>(chain->ws) & 255) != 0) return fail(AQD_ERR_INVALID, "next_workspace must be 256-byte aligned");
     if (chain->pad < 0) return fail(AQD_ERR_INVALID, "next_pad must be >= 0");
@@ -508,11 +465,175 @@ static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aq
     a.out_pad = chain->pad;
   }
   a.expand_only = stage == kStageExpandOnly ? 1 : 0;
+  plan->path = path;
+  return AQD_OK;
+}
+
+static aqd_status launch_plan(const ConvPlan& plan, aqd_stream_t stream) {
+  std::string err;
+  const ConvArgs& a = plan.a;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int path = plan.path;
   int rc = path == 1 ? launch_conv_tc(a, st, &err) : path == 5 ? launch_stem(a, st, &err) : launch_conv_direct(a, st, &err);
   if (rc) return fail((aqd_status)rc, err);
-  if (stage != kStageExpandOnly)
+  if (plan.stage != kStageExpandOnly)
     g_last_path = (path == 1 && a.ws) ? (conv_tc_uses_pair(a) ? 4 : 3) : path;
+  return AQD_OK;
+}
+
+static aqd_status conv_grouped(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
+                               int32_t stride, int32_t pad, const aqd_requant_params* rq,
+                               const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
+                               aqd_stream_t stream, ConvStage stage, const ChainOut* chain = nullptr,
+                               bool require_ws = false) {
+  ConvPlan plan;
+  const aqd_status s = plan_grouped(jobs, njobs, w, stride, pad, rq, sp, workspace, ws_bytes, stage, chain,
+                                    require_ws, &plan);
+  if (s != AQD_OK) return s;
+  return launch_plan(plan, stream);
+}
+
+aqd_status aqd_conv_int_grouped(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
+                                int32_t stride, int32_t pad, const aqd_requant_params* rq,
+                                const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
+                                aqd_stream_t stream) {
+  return conv_grouped(jobs, njobs, w, stride, pad, rq, sp, workspace, ws_bytes, stream, kStageBoth);
+}
+
+aqd_status aqd_conv_int_grouped_expanded(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
+                                         int32_t stride, int32_t pad, const aqd_requant_params* rq,
+                                         const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
+                                         aqd_stream_t stream) {
+  return conv_grouped(jobs, njobs, w, stride, pad, rq, sp, workspace, ws_bytes, stream, kStageConvOnly);
+}
+
+aqd_status aqd_conv_expand_input(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
+                                 int32_t stride, int32_t pad, void* workspace, size_t ws_bytes,
+                                 aqd_stream_t stream) {
+  if (!jobs || njobs <= 0 || njobs > kMaxJobs) return fail(AQD_ERR_INVALID, "njobs must be 1..8");
+  if (!workspace) return fail(AQD_ERR_INVALID, "the workspace must not be NULL");
+  // only the inputs matter here: give every job an int32 output of the right shape so the
+  // shared validation accepts it (nothing is written to it)
+  aqd_conv_job tmp[kMaxJobs];
+  for (int j = 0; j < njobs; ++j) {
+    tmp[j] = jobs[j];
+    tmp[j].skip = aqd_tensor{};
+    tmp[j].level = 0;
+    if (w && stride > 0 && pad >= 0) {
+      tmp[j].y.n = jobs[j].x.n;
+      tmp[j].y.h = (jobs[j].x.h + 2 * pad - w->kh) / stride + 1;
+      tmp[j].y.w = (jobs[j].x.w + 2 * pad - w->kw) / stride + 1;
+      tmp[j].y.c = w->cout;
+    }
+    tmp[j].y.bits = 32;
+    tmp[j].y.data = workspace;  // any non-null aligned pointer; never dereferenced
+  }
+  return conv_grouped(tmp, njobs, w, stride, pad, nullptr, nullptr, workspace, ws_bytes, stream,
+                      kStageExpandOnly);
+}
+
+aqd_status aqd_conv_int_grouped_chain(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
+                                      int32_t stride, int32_t pad, const aqd_requant_params* rq,
+                                      const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
+                                      int32_t next_pad, void* next_workspace, size_t next_ws_bytes,
+                                      aqd_stream_t stream) {
+  const ChainOut c{next_pad, next_workspace, next_ws_bytes};
+  return conv_grouped(jobs, njobs, w, stride, pad, rq, sp, workspace, ws_bytes, stream, kStageChain, &c);
+}
+
+// ---------------------------------------------------------------- chained tower
+
+static bool same_tensor(const aqd_tensor& a, const aqd_tensor& b) {
+  return a.data == b.data && a.n == b.n && a.h == b.h && a.w == b.w && a.c == b.c && a.bits == b.bits;
+}
+
+// Validates a tower: layers x njobs jobs, layer i's inputs are layer i-1's outputs, every
+// layer a stride-1 conv that keeps the spatial size (kh = kw = 2 pad + 1), no skips.
+static aqd_status check_tower(const aqd_conv_job* jobs, int32_t njobs, int32_t layers,
+                              const aqd_conv_weights* w, int32_t pad) {
+  if (!jobs || !w) return fail(AQD_ERR_INVALID, "jobs and w must not be NULL");
+  if (njobs <= 0 || njobs > kMaxJobs) return fail(AQD_ERR_INVALID, "njobs must be 1..8");
+  if (layers <= 0 || layers > 64) return fail(AQD_ERR_INVALID, "layers must be 1..64");
+  if (pad < 0) return fail(AQD_ERR_INVALID, "pad must be >= 0");
+  for (int i = 0; i < layers; ++i) {
+    if (w[i].kh != 2 * pad + 1 || w[i].kw != 2 * pad + 1)
+      return fail(AQD_ERR_INVALID, "every tower layer needs kh = kw = 2 pad + 1");
+    for (int j = 0; j < njobs; ++j) {
+      const aqd_conv_job& jb = jobs[(size_t)i * njobs + j];
+      if (jb.skip.data) return fail(AQD_ERR_INVALID, "tower layers take no skip");
+      if (i > 0 && !same_tensor(jb.x, jobs[(size_t)(i - 1) * njobs + j].y))
+        return fail(AQD_ERR_INVALID, "layer " + std::to_string(i) + " job " + std::to_string(j) +
+                                         ": x must be the previous layer's y");
+    }
+  }
+  return AQD_OK;
+}
+
+size_t aqd_conv_tower_sync_bytes(const aqd_conv_job* jobs, int32_t njobs, int32_t layers, int32_t pad) {
+  if (!jobs || njobs <= 0 || njobs > kMaxJobs || layers < 2 || pad < 0) return 0;
+  int64_t tiles = 0;
+  for (int j = 0; j < njobs; ++j) {
+    const aqd_tensor& x = jobs[j].x;
+    if (x.n <= 0 || x.h <= 0 || x.w <= 0) return 0;
+    tiles += (int64_t)x.n * (((int64_t)x.h * (x.w + 2 * pad) + 255) / 256);
+  }
+  return (size_t)(layers - 1) * (size_t)tiles * sizeof(uint32_t);
+}
+
+aqd_status aqd_conv_int_grouped_tower(const aqd_conv_job* jobs, int32_t njobs, int32_t layers,
+                                      const aqd_conv_weights* w, const aqd_requant_params* rq, int32_t pad,
+                                      void* ws_a, void* ws_b, size_t ws_bytes, void* sync, size_t sync_bytes,
+                                      int32_t input_expanded, aqd_stream_t stream) {
+  aqd_status s = check_tower(jobs, njobs, layers, w, pad);
+  if (s != AQD_OK) return s;
+  if (!rq) return fail(AQD_ERR_INVALID, "rq must not be NULL");
+  if (!ws_a || (layers > 1 && !ws_b)) return fail(AQD_ERR_INVALID, "ws_a and ws_b must not be NULL");
+  // every layer planned (validated, kernel chosen) before anything is launched
+  ConvPlan plans[64];
+  for (int i = 0; i < layers; ++i) {
+    void* ws = (i % 2 == 0) ? ws_a : ws_b;
+    void* nxt = (i % 2 == 0) ? ws_b : ws_a;
+    const ChainOut c{pad, nxt, ws_bytes};
+    const bool expand = i == 0 && !input_expanded;
+    const ConvStage st = i < layers - 1 ? (expand ? kStageBothChain : kStageChain)
+                                        : (expand ? kStageBoth : kStageConvOnly);
+    s = plan_grouped(jobs + (size_t)i * njobs, njobs, &w[i], 1, pad, &rq[i], nullptr, ws, ws_bytes, st,
+                     i < layers - 1 ? &c : nullptr, true, &plans[i]);
+    if (s != AQD_OK) {
+      g_last_error = "layer " + std::to_string(i) + ": " + g_last_error;
+      return s;
+    }
+  }
+  // tile-by-tile overlap when every layer runs on CTA pairs with one N tile (the same tiles
+  // in every layer) and the caller gave counters; otherwise each layer waits for the last
+  const size_t need = aqd_conv_tower_sync_bytes(jobs, njobs, layers, pad);
+  bool overlap = layers > 1 && sync != nullptr;
+  for (int i = 0; i < layers && overlap; ++i) {
+    const ConvArgs& a = plans[i].a;
+    overlap = conv_tc_uses_pair(a) && !a.split_w && a.bn == a.cout_pad &&
+              conv_tc_pair_tiles(a) * (int64_t)(layers - 1) * (int64_t)sizeof(uint32_t) == (int64_t)need;
+  }
+  if (overlap) {
+    if ((reinterpret_cast<uintptr_t>(sync) & 3) != 0) return fail(AQD_ERR_INVALID, "sync must be 4-byte aligned");
+    if (sync_bytes < need) return fail(AQD_ERR_INVALID, "sync is smaller than aqd_conv_tower_sync_bytes()");
+    uint32_t* cnt = static_cast<uint32_t*>(sync);
+    const int64_t tiles = conv_tc_pair_tiles(plans[0].a);
+    // the counters are cleared by the expansion pass that precedes layer 0 (an expansion of no
+    // rows when the input is already expanded): layer 0 waits for that grid before raising
+    // any, and the previous user of the counters, the last layer of an earlier call on this
+    // stream, has seen every counter raised before it completed
+    plans[0].a.zero = cnt;
+    plans[0].a.zero_words = (int32_t)(need / sizeof(uint32_t));
+    for (int i = 0; i < layers; ++i) {
+      plans[i].a.dep_split = i > 0 ? (int32_t)conv_tc_pair_split(plans[i - 1].a) : 0;
+      plans[i].a.dep_wait = i > 0 ? cnt + (size_t)(i - 1) * tiles : nullptr;
+      plans[i].a.dep_signal = i < layers - 1 ? cnt + (size_t)i * tiles : nullptr;
+    }
+  }
+  for (int i = 0; i < layers; ++i) {
+    s = launch_plan(plans[i], stream);
+    if (s != AQD_OK) return s;
+  }
   return AQD_OK;
 }
 

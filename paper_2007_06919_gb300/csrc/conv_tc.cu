@@ -93,6 +93,20 @@ struct Params {
   int32_t plane_rows; // workspace rows per plane
   int32_t split_w;    // weights in the split layout: a tile's bn B rows give bn/2 channels
   uint32_t* status;
+  // Tile-by-tile overlap of chained layers (workspace path on CTA pairs, one N tile): this
+  // layer's tile t reads the previous layer's output rows written by its tiles t - K .. t + K
+  // of the same image (K = 1 + wp / 256), which are also the only tiles of that layer that
+  // read the rows tile t writes. Each epilogue warp adds 1 to dep_signal[t] (release) after
+  // its stores; the TMA issuers wait (acquire, bounded) for dep_wait[t'] >= dep_target on
+  // those tiles before loading A. With dep_wait NULL the kernel waits for the whole previous
+  // grid instead (griddepcontrol.wait).
+  // Tiles split into two half-width tiles (the last, partial wave) raise the counter of their
+  // M tile: 2 x dep_target arrivals complete an M tile at or past dep_split (the layer's
+  // dp_tiles, the same for every layer of a tower: same tiles, same SMs).
+  const uint32_t* dep_wait;
+  uint32_t* dep_signal;
+  uint32_t dep_target;
+  int32_t dep_split;
 };
 
 static_assert(kSubA == kMmaM * BK, "one sub-tile is one M=128 MMA operand");
@@ -117,6 +131,31 @@ __device__ __forceinline__ FlatTile flat_tile(const ConvJobDev& jb, int mt, int 
   f.v0 = (mt - f.img * jb.tpi) * rows;
   return f;
 }
+// Waits until every tile of the previous layer that writes the rows M tile mt of job j reads
+// has been stored (see Params::dep_wait), then orders those stores before this thread's TMA
+// loads. kTileRows: rows of a tile (the previous layer's tiles have the same geometry).
+template <int kTileRows>
+__device__ __forceinline__ bool wait_dep_tiles(const Params& p, int j, int mt, volatile int* abort_flag) {
+  const ConvJobDev& jb = p.jobs[j];
+  const int img = mt / jb.tpi, m_in = mt - img * jb.tpi;
+  const int K = 1 + jb.wp / kTileRows;
+  const int lo = m_in - K < 0 ? 0 : m_in - K;
+  const int hi = m_in + K > jb.tpi - 1 ? jb.tpi - 1 : m_in + K;
+  // M tiles before dep_split (global index) complete with dep_target arrivals, later ones
+  // (split into two half-width tiles) with twice that
+  const int g0 = jb.tile_begin + img * jb.tpi;
+  const uint32_t* c = p.dep_wait + g0;
+  const int nfull = p.dep_split - (g0 + lo);  // how many of [lo, hi] come before dep_split
+  if (nfull > 0 && !counters_wait(c + lo, nfull < hi - lo + 1 ? nfull : hi - lo + 1, p.dep_target, abort_flag))
+    return false;
+  if (nfull < hi - lo + 1) {
+    const int first = nfull > 0 ? lo + nfull : lo;
+    if (!counters_wait(c + first, hi - first + 1, 2 * p.dep_target, abort_flag)) return false;
+  }
+  fence_proxy_async_global();
+  return true;
+}
+
 // Global tile t -> (job, M tile, channel range). Tiles past dp_tiles split the remaining
 // full tiles into two halves of N, so the last, partial wave covers more SMs.
 __device__ __forceinline__ TileInfo tile_info(const Params& p, int t) {
@@ -507,7 +546,8 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   // everything above overlaps the previous kernel; global memory is touched only after this
-  grid_dep_wait();
+  // (or, chained tile by tile, only after the per-tile waits of the TMA issuers)
+  if (!p.dep_wait) grid_dep_wait();
   if (threadIdx.x == 0) grid_dep_launch();
 
   const int nk = p.num_kchunks * p.a_planes;  // K chunks, over every plane of the image
@@ -594,8 +634,14 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
           wp = jb.wp;
         }
         const CUtensorMap* wm = ti.bn == BN ? &tmap_w : &tmap_wh;
+        bool deps_ready = !kFlat || p.dep_wait == nullptr;
         for (int q2 = 0; q2 < nk; ++q2, ++it, s = (s + 1 == (uint32_t)S) ? 0 : s + 1, ph ^= (s == 0)) {
           if ((int)(it % kTma) != tw) continue;
+          if (!deps_ready) {
+            // the previous layer's tiles that this tile reads (and that read what it writes)
+            if (!wait_dep_tiles<kTileRows>(p, ti.job, ti.mt, abort_flag)) { ok = false; break; }
+            deps_ready = true;
+          }
           if (!mbar_wait(b_empty + 8 * s, ph ^ 1, abort_flag)) { ok = false; break; }
           // plane of the byte image (8-bit activations: x_lo, then 16 x_hi) and K chunk in it
           const int plane = q2 >= p.num_kchunks ? 1 : 0;
@@ -954,6 +1000,16 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
         if (kPair && !leader) mbar_arrive_cluster(mapa_shared(b_tempty + 8 * buf, 0));
         else mbar_arrive(b_tempty + 8 * buf);
       }
+      if (kFlat && p.dep_signal) {
+        // this warp's stores of tile t are done: order them for the next layer's TMA (async
+        // proxy) loads, gather the warp (__syncwarp orders its lanes' stores before lane 0's
+        // next operations), and count the warp in with one release (cumulative over them)
+        fence_proxy_async_global();
+        __syncwarp();
+        // (a half-width tile counts toward its M tile)
+        const int mtile = t < p.dp_tiles ? t : p.dp_tiles + ((t - p.dp_tiles) >> 1);
+        if (lane == 0) red_release_gpu_add(p.dep_signal + mtile, 1u);
+      }
     }
     if (!ok) fail(abort_flag, p.status);
   }
@@ -985,6 +1041,10 @@ struct ExpandArgs {
   int64_t x_row_bytes;
   int64_t total_rows;     // rows of one plane
   uint8_t* ws;
+  // per-tile counters of a chained tower, cleared here (before the first layer, which waits
+  // for this grid, can raise them)
+  uint32_t* zero;
+  int32_t zero_words;
 };
 
 // E4M3 byte of the value 16 n * 2^-9 = n * 2^-5, n in [0, 15] (the raw byte n is n * 2^-9):
@@ -1042,6 +1102,8 @@ __global__ void __launch_bounds__(256) expand_kernel(const __grid_constant__ Exp
   // the previous kernel in the stream may still be reading the workspace or writing x
   grid_dep_wait();
   if (threadIdx.x == 0) grid_dep_launch();
+  if (blockIdx.x == 0)
+    for (int i = threadIdx.x; i < a.zero_words; i += blockDim.x) a.zero[i] = 0u;
   const int chunks = a.cin >> 4;
   const int total = (int)a.total_rows * chunks;
   const int lane = threadIdx.x & 31;
@@ -1193,6 +1255,33 @@ bool conv_tc_uses_pair(const ConvArgs& a) {
   return a.ws != nullptr && a.bn >= 16 && a.bn % 16 == 0 && tc::kSub == 1 && !a.no_pair;
 }
 
+// Last-wave balancing: with `workers` persistent CTAs (or CTA pairs), the full tiles past the
+// last complete wave run as two half-width (N/2) tiles each, when those halves still fit in
+// one wave; half as long per tile, they end the kernel sooner. A half tile must start on a
+// 32-channel packing group (bn / 2 a multiple of 32). Returns the first split tile.
+static int split_start(int tiles, int workers, int bn, bool split_w) {
+  const int rem = tiles % workers;
+  return (bn % 64 == 0 && !split_w && rem > 0 && 2 * rem <= workers) ? tiles - rem : tiles;
+}
+
+int64_t conv_tc_pair_split(const ConvArgs& a) {
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (sms < 2) sms = 2;
+  return split_start((int)conv_tc_pair_tiles(a), sms / 2, a.split_w ? 256 : a.bn, a.split_w != 0);
+}
+
+int64_t conv_tc_pair_tiles(const ConvArgs& a) {
+  int64_t tiles = 0;
+  for (int j = 0; j < a.njobs; ++j) {
+    const ConvJobDev& jb = a.jobs[j];
+    const int64_t wp = jb.w + 2 * a.pad;
+    tiles += (int64_t)jb.n * ((jb.ho * wp + 255) / 256);
+  }
+  return tiles;
+}
+
 int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   using namespace tc;
   Params prm{};
@@ -1241,11 +1330,12 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   // Last-wave balancing: with `workers` persistent CTAs (or CTA pairs), the full tiles past
   // the last complete wave run as two half-width (N/2) tiles each, when those halves still
   // fit in one wave; half as long per tile, they end the kernel sooner.
-  const int workers = pair ? sms / 2 : sms;
-  const int rem = tiles % workers;
-  prm.dp_tiles = tiles;
-  // (a half tile must start on a 32-channel packing group: BN / 2 a multiple of 32)
-  if (BN % 64 == 0 && !a.split_w && rem > 0 && 2 * rem <= workers) prm.dp_tiles = tiles - rem;
+  prm.dp_tiles = split_start(tiles, pair ? sms / 2 : sms, BN, a.split_w != 0);
+  const bool overlap = a.dep_wait != nullptr || a.dep_signal != nullptr;
+  if (overlap && !(flat && pair && prm.n_tiles == 1 && !a.split_w)) {
+    *err = "conv_tc: tile-by-tile chaining needs the workspace path on CTA pairs with one N tile";
+    return 1;
+  }
   prm.total_tiles = prm.dp_tiles + 2 * (tiles - prm.dp_tiles);
   prm.num_kchunks = flat ? a.k_total / bk : a.k_pad / BK;
   prm.cin = a.cin; prm.cout = a.cout; prm.kh = a.kh; prm.kw = a.kw;
@@ -1274,6 +1364,10 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
     }
   }
   prm.status = a.status;
+  prm.dep_wait = a.dep_wait;
+  prm.dep_signal = a.dep_signal;
+  prm.dep_target = (uint32_t)(2 * kEpiWarps);  // epilogue warps of both CTAs of a pair
+  prm.dep_split = a.dep_split;
   // shared memory plan: stages of (BM x bk A bytes + this CTA's B rows x bk bytes)
   const int b_rows = pair ? BN / 2 : BN;
   const size_t stage_a = (size_t)kSub * 128 * bk;
@@ -1330,14 +1424,17 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   if (flat) {
     // 1) expand the packed codes of every job into the zero-padded byte workspace (unless
     //    the caller expanded them already)
-    if (!a.skip_expand) {
+    if (!a.skip_expand || a.zero_words > 0) {
+      // (with skip_expand, only the counters are cleared: an expansion of no rows)
       ExpandArgs ea{};
       for (int j = 0; j < a.njobs; ++j) ea.jobs[j] = prm.jobs[j];
       ea.njobs = a.njobs; ea.cin = a.cin; ea.pad = a.pad; ea.x_row_bytes = a.x_row_bytes;
-      ea.total_rows = rows; ea.ws = a.ws;
+      ea.total_rows = a.skip_expand ? 0 : rows; ea.ws = a.ws;
+      ea.zero = a.zero_words > 0 ? a.zero : nullptr;
+      ea.zero_words = a.zero_words;
       // one warp per run of 32 * 8 (row, 16-byte chunk) pairs, 8 warps per block
-      const int64_t pairs = rows * (a.cin / 16);
-      const unsigned blocks = (unsigned)((pairs + 2047) / 2048);
+      const int64_t pairs = ea.total_rows * (a.cin / 16);
+      const unsigned blocks = pairs > 0 ? (unsigned)((pairs + 2047) / 2048) : 1u;
       cudaLaunchConfig_t cfg = {};
       cfg.gridDim = dim3(blocks);
       cfg.blockDim = dim3(256);

@@ -60,7 +60,21 @@ struct ConvArgs {
   uint8_t* ws_out;        // chained output: also write the output codes as the next conv's byte image
   int32_t out_pad;        // padding of that next conv
   uint32_t* status;       // device status word
+  // tile-by-tile chaining of stride-1 layers (workspace path, CTA pairs, one N tile): per-tile
+  // counters of the previous layer to wait on (NULL: wait for the whole previous grid), and
+  // this layer's counters to raise (NULL: none)
+  const uint32_t* dep_wait;
+  uint32_t* dep_signal;
+  int32_t dep_split;      // the previous layer's first M tile run as two half-width tiles
+  uint32_t* zero;         // words cleared by the expansion pass before the conv (NULL: none)
+  int32_t zero_words;
 };
+// Tiles of one grouped workspace-path launch on CTA pairs with one N tile (the length of its
+// per-tile counter array).
+int64_t conv_tc_pair_tiles(const ConvArgs& a);
+// The first tile that such a launch splits into two half-width tiles (its last, partial wave;
+// the tile count when it splits none).
+int64_t conv_tc_pair_split(const ConvArgs& a);
 
 // Prepared-weight geometry shared by the API and the weight-prep kernel.
 struct WeightGeom {

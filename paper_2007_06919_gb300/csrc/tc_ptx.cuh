@@ -119,6 +119,42 @@ __device__ __forceinline__ void fail(volatile int* abort_flag, uint32_t* status)
 __device__ __forceinline__ void fence_proxy_async() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
+// orders this thread's generic-proxy view of global memory with its async-proxy (TMA)
+// accesses: after a store that TMA reads elsewhere, and after the acquire that makes other
+// threads' stores visible, before this thread's TMA loads of them
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t ld_relaxed_gpu(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+// with a preceding relaxed load that observed a release, forms the acquire side of the pattern
+__device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
+__device__ __forceinline__ void red_release_gpu_add(uint32_t* p, uint32_t v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+// Bounded wait until c[i] >= target for every i in [0, n): the counters are read together
+// (relaxed loads, no ordering among them) until all are reached, then one fence.acq_rel
+// makes the writes released before them visible to this thread. False if the deadline passed
+// or another role aborted.
+static __device__ __noinline__ bool counters_wait(const uint32_t* c, int n, uint32_t target, volatile int* abort_flag) {
+  uint64_t deadline = 0;
+  for (uint32_t spin = 0;; ++spin) {
+    bool all = true;
+    for (int i = 0; i < n; ++i) all &= ld_relaxed_gpu(c + i) >= target;
+    if (all) break;
+    if (spin == 0) deadline = globaltimer() + kTimeoutNs;
+    __nanosleep(64);
+    if ((spin & 15) == 15) {
+      if (*abort_flag) return false;
+      if (globaltimer() > deadline) return false;
+    }
+  }
+  fence_acq_rel_gpu();
+  return true;
+}
 __device__ __forceinline__ void fence_barrier_init() {
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }

@@ -263,12 +263,13 @@ size_t aqd_conv_tower_sync_bytes(const aqd_conv_job* jobs, int32_t njobs, int32_
  *     chained previous layer). The call never writes ws_b's zero border: zero ws_b once
  *     before its first use.
  *   sync: device counters of aqd_conv_tower_sync_bytes() bytes (4-byte aligned), cleared on
- *     `stream` by the call's first kernel. When every layer runs on CTA pairs with
- *     one output-channel tile (cout <= 256), layer i+1 starts as soon as SMs free up and each
- *     of its tiles waits (a bounded wait, AQD_ERR_TIMEOUT on expiry) only for the tiles of
- *     layer i whose rows it reads. With sync NULL, or when that condition fails, each layer
- *     waits for the whole previous one. Calls that share sync or the workspaces must not
- *     overlap in time.
+ *     `stream` by the call's first kernel. With sync given, the longest leading run of
+ *     layers of one shape (same weight geometry and code widths, at most 4, each running on
+ *     CTA pairs with one output-channel tile, cout <= 256) runs as ONE persistent launch in
+ *     layer-major tile order: each tile waits (a bounded wait, AQD_ERR_TIMEOUT on expiry)
+ *     only for the tiles of the previous layer whose rows it reads. The remaining layers,
+ *     and every layer when sync is NULL, run one launch each, each waiting for the whole
+ *     previous launch. Calls that share sync or the workspaces must not overlap in time.
  * Every layer is validated before anything is launched; an error names the layer. */
 aqd_status aqd_conv_int_grouped_tower(const aqd_conv_job* jobs, int32_t njobs, int32_t layers,
                                       const aqd_conv_weights* w, const aqd_requant_params* rq, int32_t pad,

@@ -604,33 +604,49 @@ aqd_status aqd_conv_int_grouped_tower(const aqd_conv_job* jobs, int32_t njobs, i
       return s;
     }
   }
-  // tile-by-tile overlap when every layer runs on CTA pairs with one N tile (the same tiles
-  // in every layer) and the caller gave counters; otherwise each layer waits for the last
-  const size_t need = aqd_conv_tower_sync_bytes(jobs, njobs, layers, pad);
-  bool overlap = layers > 1 && sync != nullptr;
-  for (int i = 0; i < layers && overlap; ++i) {
-    const ConvArgs& a = plans[i].a;
-    overlap = conv_tc_uses_pair(a) && !a.split_w && a.bn == a.cout_pad &&
-              conv_tc_pair_tiles(a) * (int64_t)(layers - 1) * (int64_t)sizeof(uint32_t) == (int64_t)need;
+  // The longest prefix of layers of one shape (same weights geometry and code widths, chained
+  // 2/3/4-bit outputs, CTA pairs with one N tile) runs as one launch when the caller gave
+  // counters: layer l + 1's tiles start as soon as the tiles of layer l they read are stored.
+  // The other layers run one launch each, each waiting for the previous launch.
+  int fused = 1;
+  if (sync != nullptr) {
+    auto same_shape = [&](const ConvArgs& a, const ConvArgs& b) {
+      return a.cin == b.cin && a.cout == b.cout && a.kh == b.kh && a.kw == b.kw && a.x_bits == b.x_bits &&
+             a.out_bits == b.out_bits && a.bn == b.bn && a.cout_pad == b.cout_pad && a.k_pad == b.k_pad &&
+             a.acc_bound == b.acc_bound;
+    };
+    auto fusable = [&](const ConvArgs& a) {
+      return conv_tc_uses_pair(a) && !a.split_w && a.a_planes <= 1 && a.bn == a.cout_pad && a.ws_out != nullptr;
+    };
+    while (fused < layers && fused < kMaxLayers && fusable(plans[fused - 1].a) && plans[fused].path == 1 &&
+           same_shape(plans[0].a, plans[fused].a) && conv_tc_uses_pair(plans[fused].a))
+      ++fused;
   }
-  if (overlap) {
+  if (fused > 1) {
+    const int64_t tiles = conv_tc_pair_tiles(plans[0].a);
+    const size_t need = (size_t)(fused - 1) * (size_t)tiles * sizeof(uint32_t);
     if ((reinterpret_cast<uintptr_t>(sync) & 3) != 0) return fail(AQD_ERR_INVALID, "sync must be 4-byte aligned");
     if (sync_bytes < need) return fail(AQD_ERR_INVALID, "sync is smaller than aqd_conv_tower_sync_bytes()");
-    uint32_t* cnt = static_cast<uint32_t*>(sync);
-    const int64_t tiles = conv_tc_pair_tiles(plans[0].a);
-    // the counters are cleared by the expansion pass that precedes layer 0 (an expansion of no
-    // rows when the input is already expanded): layer 0 waits for that grid before raising
-    // any, and the previous user of the counters, the last layer of an earlier call on this
-    // stream, has seen every counter raised before it completed
-    plans[0].a.zero = cnt;
-    plans[0].a.zero_words = (int32_t)(need / sizeof(uint32_t));
-    for (int i = 0; i < layers; ++i) {
-      plans[i].a.dep_split = i > 0 ? (int32_t)conv_tc_pair_split(plans[i - 1].a) : 0;
-      plans[i].a.dep_wait = i > 0 ? cnt + (size_t)(i - 1) * tiles : nullptr;
-      plans[i].a.dep_signal = i < layers - 1 ? cnt + (size_t)i * tiles : nullptr;
+    ConvPlan f = plans[0];
+    ConvArgs& a = f.a;
+    a.nlayers = fused;
+    for (int l = 0; l < fused; ++l) {
+      const ConvArgs& b = plans[l].a;
+      a.layer[l].w_e4m3 = b.w_e4m3;
+      a.layer[l].m0 = b.m0; a.layer[l].shift = b.shift; a.layer[l].bias = b.bias;
+      for (int j = 0; j < njobs; ++j) a.layer[l].y[j] = b.jobs[j].y;
+      a.layer[l].ws_out = b.ws_out;
     }
+    a.ws2 = static_cast<uint8_t*>(ws_b);
+    a.dep = static_cast<uint32_t*>(sync);
+    // the counters are cleared by the expansion pass that precedes the launch (an expansion of
+    // no rows when the input is already expanded); the launch waits for that grid first
+    a.zero = a.dep;
+    a.zero_words = (int32_t)(need / sizeof(uint32_t));
+    s = launch_plan(f, stream);
+    if (s != AQD_OK) return s;
   }
-  for (int i = 0; i < layers; ++i) {
+  for (int i = fused > 1 ? fused : 0; i < layers; ++i) {
     s = launch_plan(plans[i], stream);
     if (s != AQD_OK) return s;
   }

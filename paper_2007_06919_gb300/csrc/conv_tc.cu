@@ -69,15 +69,30 @@ __host__ __device__ constexpr int threads_for(bool flat) { return flat ? (kWarpT
 constexpr int kMaxStages = 16;
 constexpr int kQTab = 256;  // K-chunk table entries (larger K falls back to division)
 
+// One layer of a launch: its per-channel tables, the packed output of each job and the
+// zero-padded byte image its epilogue writes for the next layer (NULL: none).
+struct LayerDev {
+  const int32_t* m0;
+  const int8_t* shift;
+  const int32_t* bias;
+  uint8_t* y[kMaxJobs];
+  uint8_t* ws_out;
+};
+
+// The tensor maps of a launch: the weights of each layer, the weights with half-height
+// boxes (half-width tiles), and the two byte images that chained layers read in turn.
+struct Maps {
+  CUtensorMap w[kMaxLayers];
+  CUtensorMap wh;
+  CUtensorMap a[2];
+};
+
 struct Params {
   ConvJobDev jobs[kMaxJobs];
   int32_t njobs, total_tiles, n_tiles, num_kchunks;
   int32_t cin, cout, kh, kw, stride, pad, k_total;
   int32_t out_bits, skip_bits;
   int64_t x_row_bytes, y_row_bytes, skip_row_bytes;
-  const int32_t* m0;
-  const int8_t* shift;
-  const int32_t* bias;
   const int32_t* skip_c;
   const int8_t* skip_d;
   int32_t upsample, scale_main, has_skip;
@@ -87,26 +102,24 @@ struct Params {
   int32_t dp_tiles;   // tiles [0, dp_tiles) are bn wide; later ones are the two bn/2 halves
                       // of the remaining full tiles (the last, partial wave)
   uint32_t off_b, off_epi, off_bar, off_qtab;
-  uint8_t* ws_out;    // chained output image (NULL: none)
   int32_t out_pad;
   int32_t a_planes;   // K runs over this many planes of the byte image (2: 8-bit activations)
   int32_t plane_rows; // workspace rows per plane
   int32_t split_w;    // weights in the split layout: a tile's bn B rows give bn/2 channels
   uint32_t* status;
-  // Tile-by-tile overlap of chained layers (workspace path on CTA pairs, one N tile): this
-  // layer's tile t reads the previous layer's output rows written by its tiles t - K .. t + K
-  // of the same image (K = 1 + wp / 256), which are also the only tiles of that layer that
-  // read the rows tile t writes. Each epilogue warp adds 1 to dep_signal[t] (release) after
-  // its stores; the TMA issuers wait (acquire, bounded) for dep_wait[t'] >= dep_target on
-  // those tiles before loading A. With dep_wait NULL the kernel waits for the whole previous
-  // grid instead (griddepcontrol.wait).
-  // Tiles split into two half-width tiles (the last, partial wave) raise the counter of their
-  // M tile: 2 x dep_target arrivals complete an M tile at or past dep_split (the layer's
-  // dp_tiles, the same for every layer of a tower: same tiles, same SMs).
-  const uint32_t* dep_wait;
-  uint32_t* dep_signal;
+  // Several chained stride-1 layers of one shape in one launch (workspace path, CTA pairs,
+  // one N tile, no half-width tiles): layer l covers the tiles [l * layer_tiles, (l + 1) *
+  // layer_tiles), in that order over the persistent CTAs. Tile t of layer l reads the
+  // previous layer's output rows written by its tiles t - K .. t + K of the same image
+  // (K = 1 + wp / 256), which are also the only tiles of that layer that read the rows tile
+  // t writes. Each epilogue warp of a tile of layer l < nlayers - 1 adds 1 to
+  // dep[l * layer_tiles + t] (release) after its stores; the TMA issuers of a tile of layer
+  // l > 0 wait (acquire, bounded) for dep[(l - 1) * layer_tiles + t'] >= dep_target on those
+  // tiles before loading A.
+  int32_t nlayers, layer_tiles;
+  LayerDev layers[kMaxLayers];
+  uint32_t* dep;
   uint32_t dep_target;
-  int32_t dep_split;
 };
 
 static_assert(kSubA == kMmaM * BK, "one sub-tile is one M=128 MMA operand");
@@ -114,6 +127,7 @@ static_assert(kSubA == kMmaM * BK, "one sub-tile is one M=128 MMA operand");
 // ---------------------------------------------------------------- tile bookkeeping
 
 struct TileInfo {
+  int layer;
   int job, mt;
   int bn;    // MMA N of this tile (weight rows): p.bn, or p.bn / 2 for a half tile
   int col0;  // first output channel
@@ -131,27 +145,18 @@ __device__ __forceinline__ FlatTile flat_tile(const ConvJobDev& jb, int mt, int 
   f.v0 = (mt - f.img * jb.tpi) * rows;
   return f;
 }
-// Waits until every tile of the previous layer that writes the rows M tile mt of job j reads
-// has been stored (see Params::dep_wait), then orders those stores before this thread's TMA
-// loads. kTileRows: rows of a tile (the previous layer's tiles have the same geometry).
+// Waits until every tile of layer l - 1 that writes the rows M tile mt of job j (of layer l)
+// reads has been stored (see Params::dep), then orders those stores before this thread's TMA
+// loads. kTileRows: rows of a tile (every layer of a launch has the same tiles).
 template <int kTileRows>
-__device__ __forceinline__ bool wait_dep_tiles(const Params& p, int j, int mt, volatile int* abort_flag) {
+__device__ __forceinline__ bool wait_dep_tiles(const Params& p, int l, int j, int mt, volatile int* abort_flag) {
   const ConvJobDev& jb = p.jobs[j];
   const int img = mt / jb.tpi, m_in = mt - img * jb.tpi;
   const int K = 1 + jb.wp / kTileRows;
   const int lo = m_in - K < 0 ? 0 : m_in - K;
   const int hi = m_in + K > jb.tpi - 1 ? jb.tpi - 1 : m_in + K;
-  // M tiles before dep_split (global index) complete with dep_target arrivals, later ones
-  // (split into two half-width tiles) with twice that
-  const int g0 = jb.tile_begin + img * jb.tpi;
-  const uint32_t* c = p.dep_wait + g0;
-  const int nfull = p.dep_split - (g0 + lo);  // how many of [lo, hi] come before dep_split
-  if (nfull > 0 && !counters_wait(c + lo, nfull < hi - lo + 1 ? nfull : hi - lo + 1, p.dep_target, abort_flag))
-    return false;
-  if (nfull < hi - lo + 1) {
-    const int first = nfull > 0 ? lo + nfull : lo;
-    if (!counters_wait(c + first, hi - first + 1, 2 * p.dep_target, abort_flag)) return false;
-  }
+  const uint32_t* c = p.dep + (size_t)(l - 1) * p.layer_tiles + jb.tile_begin + img * jb.tpi;
+  if (!counters_wait(c + lo, hi - lo + 1, p.dep_target, abort_flag)) return false;
   fence_proxy_async_global();
   return true;
 }
@@ -159,6 +164,8 @@ __device__ __forceinline__ bool wait_dep_tiles(const Params& p, int j, int mt, v
 // Global tile t -> (job, M tile, channel range). Tiles past dp_tiles split the remaining
 // full tiles into two halves of N, so the last, partial wave covers more SMs.
 __device__ __forceinline__ TileInfo tile_info(const Params& p, int t) {
+  const int layer = p.nlayers > 1 ? t / p.layer_tiles : 0;
+  t -= layer * p.layer_tiles;
   int half = -1;
   if (t >= p.dp_tiles) {
     const int h = t - p.dp_tiles;
@@ -170,6 +177,7 @@ __device__ __forceinline__ TileInfo tile_info(const Params& p, int t) {
   while (j + 1 < p.njobs && t >= p.jobs[j + 1].tile_begin) ++j;
   int local = t - p.jobs[j].tile_begin;
   TileInfo ti;
+  ti.layer = layer;
   ti.job = j;
   ti.mt = local / p.n_tiles;
   const int nt = local - ti.mt * p.n_tiles;
@@ -377,18 +385,18 @@ __device__ __forceinline__ void pack_bytewords(const uint32_t (&bw)[8], uint32_t
   }
 }
 // Chained output from byte-words (see chain_store).
-__device__ __forceinline__ void chain_store_bytes(const Params& p, const ConvJobDev& jb, int img, int oh, int ow,
-                                                  int ch0, const uint32_t (&bw)[8]) {
+__device__ __forceinline__ void chain_store_bytes(const Params& p, uint8_t* ws_out, const ConvJobDev& jb, int img,
+                                                  int oh, int ow, int ch0, const uint32_t (&bw)[8]) {
   const int row = jb.orow_off + (img * jb.ohp + oh + p.out_pad) * jb.owp + ow + p.out_pad;
-  uint4* dst = reinterpret_cast<uint4*>(p.ws_out + (size_t)row * p.cout + ch0);
+  uint4* dst = reinterpret_cast<uint4*>(ws_out + (size_t)row * p.cout + ch0);
   dst[0] = make_uint4(bw[0], bw[1], bw[2], bw[3]);
   dst[1] = make_uint4(bw[4], bw[5], bw[6], bw[7]);
 }
 
 // Chained output: the 32 codes of one packed group, one byte each, at their place in the
 // zero-padded byte image that the next stride-1 conv (padding out_pad) reads.
-__device__ __forceinline__ void chain_store(const Params& p, const ConvJobDev& jb, int img, int oh, int ow,
-                                            int ch0, const uint32_t gw[8], int out_bits) {
+__device__ __forceinline__ void chain_store(const Params& p, uint8_t* ws_out, const ConvJobDev& jb, int img, int oh,
+                                            int ow, int ch0, const uint32_t gw[8], int out_bits) {
   uint32_t o[8];
   switch (out_bits) {
     case 2: unpack_group_bytes<2>(gw, o); break;
@@ -396,7 +404,7 @@ __device__ __forceinline__ void chain_store(const Params& p, const ConvJobDev& j
     default: unpack_group_bytes<4>(gw, o); break;
   }
   const int row = jb.orow_off + (img * jb.ohp + oh + p.out_pad) * jb.owp + ow + p.out_pad;
-  uint4* dst = reinterpret_cast<uint4*>(p.ws_out + (size_t)row * p.cout + ch0);
+  uint4* dst = reinterpret_cast<uint4*>(ws_out + (size_t)row * p.cout + ch0);
   dst[0] = make_uint4(o[0], o[1], o[2], o[3]);
   dst[1] = make_uint4(o[4], o[5], o[6], o[7]);
 }
@@ -465,8 +473,7 @@ __device__ __forceinline__ void load_chunk(const Params& p, RowCursor<kXBits>& r
 // kSplit: the 8-bit split form (split weights combined as D1 + 16 D2 in the epilogue).
 template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair, bool kSkip, bool kSplit, int kBK>
 __global__ void __launch_bounds__(threads_for(kFlat), 1)
-conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_wh,
-               const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ Params p) {
+conv_tc_kernel(const __grid_constant__ Maps maps, const __grid_constant__ Params p) {
   static_assert(!kPair || kFlat, "the CTA-pair form exists for the workspace path only");
   static_assert(kBK == BK || kFlat, "64-byte K chunks exist for the workspace path only");
   // bytes of one stage's A operand: kSub sub-tiles of 128 rows x kBK bytes
@@ -533,11 +540,13 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
     }
   }
   if (warp >= kWarpTma && warp < kWarpTma + kTma && lane == 0) {
-    asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmap_w) : "memory");
-    if (p.dp_tiles < p.total_tiles) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmap_wh) : "memory");
+    for (int l = 0; l < p.nlayers; ++l) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&maps.w[l]) : "memory");
+    if (p.dp_tiles < p.layer_tiles) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&maps.wh) : "memory");
+    if (kFlat) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&maps.a[0]) : "memory");
+      if (p.nlayers > 1) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&maps.a[1]) : "memory");
+    }
   }
-  if (kFlat && warp >= kWarpTma && warp < kWarpTma + kTma && lane == 0)
-    asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmap_a) : "memory");
   tc_fence_before();
   __syncthreads();
   // the peer signals this CTA's barriers (and the leader's MMAs read the peer's shared
@@ -546,8 +555,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   // everything above overlaps the previous kernel; global memory is touched only after this
-  // (or, chained tile by tile, only after the per-tile waits of the TMA issuers)
-  if (!p.dep_wait) grid_dep_wait();
+  grid_dep_wait();
   if (threadIdx.x == 0) grid_dep_launch();
 
   const int nk = p.num_kchunks * p.a_planes;  // K chunks, over every plane of the image
@@ -571,7 +579,9 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       bool next_ready = false;  // the stage after the current one is known to be full
       for (int t = first_tile; t < p.total_tiles && ok; t += tile_stride, ++lt) {
         const uint32_t buf = lt & 1;
-        const uint32_t idesc = t < p.dp_tiles ? idesc_full : idesc_half;
+        // (half-width tiles are counted within a layer; a launch of several layers has none)
+        const int t_in_layer = p.nlayers > 1 ? t - (t / p.layer_tiles) * p.layer_tiles : t;
+        const uint32_t idesc = t_in_layer < p.dp_tiles ? idesc_full : idesc_half;
         if (!mbar_poll(b_tempty + 8 * buf, ((lt >> 1) & 1) ^ 1, abort_flag)) { ok = false; break; }
         tc_fence_after();
         const uint32_t d0 = tmem_base + buf * (uint32_t)(kSub * BN);  // sub-tile j at +j*BN
@@ -633,13 +643,14 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
           row0 = jb.row_off + ft.img * jb.hp * jb.wp + ft.v0 + (int)rank * 128;
           wp = jb.wp;
         }
-        const CUtensorMap* wm = ti.bn == BN ? &tmap_w : &tmap_wh;
-        bool deps_ready = !kFlat || p.dep_wait == nullptr;
+        const CUtensorMap* wm = ti.bn == BN ? &maps.w[ti.layer] : &maps.wh;
+        const CUtensorMap* am = &maps.a[ti.layer & 1];  // layers read the two images in turn
+        bool deps_ready = !kFlat || ti.layer == 0;
         for (int q2 = 0; q2 < nk; ++q2, ++it, s = (s + 1 == (uint32_t)S) ? 0 : s + 1, ph ^= (s == 0)) {
           if ((int)(it % kTma) != tw) continue;
           if (!deps_ready) {
             // the previous layer's tiles that this tile reads (and that read what it writes)
-            if (!wait_dep_tiles<kTileRows>(p, ti.job, ti.mt, abort_flag)) { ok = false; break; }
+            if (!wait_dep_tiles<kTileRows>(p, ti.layer, ti.job, ti.mt, abort_flag)) { ok = false; break; }
             deps_ready = true;
           }
           if (!mbar_wait(b_empty + 8 * s, ph ^ 1, abort_flag)) { ok = false; break; }
@@ -664,11 +675,11 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
             const uint32_t b_bytes = (uint32_t)(ti.bn / 2) * kBK;
             if (leader) {
               mbar_arrive_expect_tx(b_full + 8 * s, 2 * (b_bytes + kStA));
-              tma_load_2d(s_a + s * kStA, &tmap_a, cb * kBK, row, b_full + 8 * s);
+              tma_load_2d(s_a + s * kStA, am, cb * kBK, row, b_full + 8 * s);
               tma_load_2d(s_b + s * stage_b_bytes, wm, q * kBK, brow, b_full + 8 * s);
             } else {
               const uint32_t fb = mapa_shared(b_full + 8 * s, 0);
-              tma_load_2d_pair(s_a + s * kStA, &tmap_a, cb * kBK, row, fb);
+              tma_load_2d_pair(s_a + s * kStA, am, cb * kBK, row, fb);
               tma_load_2d_pair(s_b + s * stage_b_bytes, wm, q * kBK, brow, fb);
             }
             continue;
@@ -676,7 +687,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
             // A: 128 consecutive rows of the padded byte image, shifted by the tap (r, s)
             const int row = row0 + prow + r * wp + sx;
             mbar_arrive_expect_tx(b_full + 8 * s, (uint32_t)ti.bn * kBK + kStA);
-            tma_load_2d(s_a + s * kStA, &tmap_a, cb * kBK, row, b_full + 8 * s);
+            tma_load_2d(s_a + s * kStA, am, cb * kBK, row, b_full + 8 * s);
           } else {
             (void)r; (void)sx; (void)cb;
             mbar_arrive_expect_tx(b_full + 8 * s, (uint32_t)ti.bn * kBK);
@@ -779,7 +790,9 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       // this tile's output channels that exist (a last N tile may reach past cout; packed
       // groups past it must not be written)
       const int TBN = ti.cn < p.cout - ti.col0 ? ti.cn : p.cout - ti.col0;
-      const long long key = ((long long)jb.level << 32) | ((long long)ti.col0 << 10) | TBN;
+      const LayerDev& ly = p.layers[ti.layer];
+      const long long key =
+          ((long long)ti.layer << 48) | ((long long)jb.level << 32) | ((long long)ti.col0 << 10) | TBN;
       if (key != cur_key) {
         // (the same decision in every epilogue thread: all of them see the same tiles)
         named_bar(1, kEpiThreads);  // every epilogue warp is done with the previous tables
@@ -794,13 +807,13 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
           int4 ef = make_int4((int32_t)(0u - kMagicBits), 0, 0, 1);
           if (col < TBN && ch < p.cout) {
             const int64_t idx = (int64_t)jb.level * p.cout + ch;
-            ec.bias = p.bias ? p.bias[idx] : 0;
+            ec.bias = ly.bias ? ly.bias[idx] : 0;
             const bool sb = ec.bias >= -(1 << 30) && ec.bias <= (1 << 30);
             sbias &= sb;
             ef.x = (int32_t)((uint32_t)ec.bias - kMagicBits);
             if (out_bits != 32) {
-              ec.m0 = p.m0[idx];
-              const int r = 31 + p.shift[idx];
+              ec.m0 = ly.m0[idx];
+              const int r = 31 + ly.shift[idx];
               ec.r = (int8_t)r;
               if (r >= 33 && sb) { ef.y = ec.m0; ef.z = 1 << (r - 33); ef.w = r - 32; }
               else fq = 0;
@@ -890,7 +903,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
           row_ok = m < jb.m_total;
         }
         if (row_ok) {
-          uint8_t* yrow = jb.y + (int64_t)m * p.y_row_bytes;
+          uint8_t* yrow = ly.y[ti.job] + (int64_t)m * p.y_row_bytes;
           const int ch0 = ti.col0 + g0;
           if (mode == 1 && magic) {
             // codes as byte-words: the chained image takes them as they are, the packed
@@ -904,7 +917,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
               default: pack_bytewords<8>(bw, gw); break;
             }
             store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
-            if (kFlat && p.ws_out) chain_store_bytes(p, jb, oimg, oh, ow, ch0, bw);
+            if (kFlat && ly.ws_out) chain_store_bytes(p, ly.ws_out, jb, oimg, oh, ow, ch0, bw);
           } else if (mode == 1) {
             uint32_t gw[8];
             {
@@ -916,7 +929,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
               }
             }
             store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
-            if (kFlat && p.ws_out) chain_store(p, jb, oimg, oh, ow, ch0, gw, out_bits);
+            if (kFlat && ly.ws_out) chain_store(p, ly.ws_out, jb, oimg, oh, ow, ch0, gw, out_bits);
           } else if (mode == 2) {
             int32_t* yr = reinterpret_cast<int32_t*>(yrow) + ch0;
             const bool whole = ncols == 32 && ch0 + 32 <= p.cout;
@@ -981,7 +994,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
                 default: pack_bytewords<8>(bw, gw); break;
               }
               store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
-              if (kFlat && p.ws_out) chain_store_bytes(p, jb, oimg, oh, ow, ch0, bw);
+              if (kFlat && ly.ws_out) chain_store_bytes(p, ly.ws_out, jb, oimg, oh, ow, ch0, bw);
             }
           }
         }
@@ -1000,15 +1013,14 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
         if (kPair && !leader) mbar_arrive_cluster(mapa_shared(b_tempty + 8 * buf, 0));
         else mbar_arrive(b_tempty + 8 * buf);
       }
-      if (kFlat && p.dep_signal) {
+      if (kFlat && p.dep && ti.layer < p.nlayers - 1) {
         // this warp's stores of tile t are done: order them for the next layer's TMA (async
         // proxy) loads, gather the warp (__syncwarp orders its lanes' stores before lane 0's
         // next operations), and count the warp in with one release (cumulative over them)
         fence_proxy_async_global();
         __syncwarp();
-        // (a half-width tile counts toward its M tile)
-        const int mtile = t < p.dp_tiles ? t : p.dp_tiles + ((t - p.dp_tiles) >> 1);
-        if (lane == 0) red_release_gpu_add(p.dep_signal + mtile, 1u);
+        // (a tower launch has no half-width tiles: t is layer * layer_tiles + the tile)
+        if (lane == 0) red_release_gpu_add(p.dep + t, 1u);
       }
     }
     if (!ok) fail(abort_flag, p.status);
@@ -1211,8 +1223,8 @@ static EncodeTiledFn get_encode_fn(std::string* err) {
 
 template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair = false, bool kSkip = true, bool kSplit = false,
           int kBK = BK>
-static int launch_bits(const Params& prm, const CUtensorMap& map, const CUtensorMap& map_h, const CUtensorMap& map_a,
-                       int grid, size_t smem, cudaStream_t stream, std::string* err) {
+static int launch_bits(const Params& prm, const Maps& maps, int grid, size_t smem, cudaStream_t stream,
+                       std::string* err) {
   auto kern = conv_tc_kernel<kXBits, kChunkInTap, kFlat, kPair, kSkip, kSplit, kBK>;
   // The opt-in limit is raised to the device maximum, never lowered to this call's size:
   // a CUDA graph node captured earlier with a larger plan must stay launchable (a graph
@@ -1240,7 +1252,7 @@ static int launch_bits(const Params& prm, const CUtensorMap& map, const CUtensor
   attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = kPair ? 2 : 1;
-  e = cudaLaunchKernelEx(&cfg, kern, map, map_h, map_a, prm);
+  e = cudaLaunchKernelEx(&cfg, kern, maps, prm);
   if (e != cudaSuccess) { *err = std::string("conv_tc launch: ") + cudaGetErrorString(e); return 3; }
   e = cudaGetLastError();
   if (e != cudaSuccess) { *err = std::string("conv_tc launch: ") + cudaGetErrorString(e); return 3; }
@@ -1262,14 +1274,6 @@ bool conv_tc_uses_pair(const ConvArgs& a) {
 static int split_start(int tiles, int workers, int bn, bool split_w) {
   const int rem = tiles % workers;
   return (bn % 64 == 0 && !split_w && rem > 0 && 2 * rem <= workers) ? tiles - rem : tiles;
-}
-
-int64_t conv_tc_pair_split(const ConvArgs& a) {
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  if (sms < 2) sms = 2;
-  return split_start((int)conv_tc_pair_tiles(a), sms / 2, a.split_w ? 256 : a.bn, a.split_w != 0);
 }
 
 int64_t conv_tc_pair_tiles(const ConvArgs& a) {
@@ -1330,30 +1334,47 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   // Last-wave balancing: with `workers` persistent CTAs (or CTA pairs), the full tiles past
   // the last complete wave run as two half-width (N/2) tiles each, when those halves still
   // fit in one wave; half as long per tile, they end the kernel sooner.
-  prm.dp_tiles = split_start(tiles, pair ? sms / 2 : sms, BN, a.split_w != 0);
-  const bool overlap = a.dep_wait != nullptr || a.dep_signal != nullptr;
-  if (overlap && !(flat && pair && prm.n_tiles == 1 && !a.split_w)) {
-    *err = "conv_tc: tile-by-tile chaining needs the workspace path on CTA pairs with one N tile";
+  const int nlayers = a.nlayers > 1 ? a.nlayers : 1;
+  if (nlayers > 1 && !(flat && pair && prm.n_tiles == 1 && !a.split_w && a.a_planes <= 1 && a.ws2 && a.dep &&
+                       nlayers <= kMaxLayers)) {
+    *err = "conv_tc: chained layers in one launch need the workspace path on CTA pairs with one N tile";
     return 1;
   }
-  prm.total_tiles = prm.dp_tiles + 2 * (tiles - prm.dp_tiles);
+  // (a launch of several layers has no half-width tiles: every layer keeps the same tiles)
+  prm.dp_tiles = nlayers > 1 ? tiles : split_start(tiles, pair ? sms / 2 : sms, BN, a.split_w != 0);
+  prm.total_tiles = nlayers * (prm.dp_tiles + 2 * (tiles - prm.dp_tiles));
+  prm.nlayers = nlayers;
+  prm.layer_tiles = prm.total_tiles / nlayers;
   prm.num_kchunks = flat ? a.k_total / bk : a.k_pad / BK;
   prm.cin = a.cin; prm.cout = a.cout; prm.kh = a.kh; prm.kw = a.kw;
   prm.stride = a.stride; prm.pad = a.pad; prm.k_total = a.k_total;
   prm.out_bits = a.out_bits; prm.skip_bits = a.skip_bits;
   prm.x_row_bytes = a.x_row_bytes; prm.y_row_bytes = a.y_row_bytes; prm.skip_row_bytes = a.skip_row_bytes;
-  prm.m0 = a.m0; prm.shift = a.shift; prm.bias = a.bias;
+  if (nlayers > 1) {
+    for (int l = 0; l < nlayers; ++l) {
+      LayerDev& ly = prm.layers[l];
+      ly.m0 = a.layer[l].m0; ly.shift = a.layer[l].shift; ly.bias = a.layer[l].bias;
+      for (int j = 0; j < a.njobs; ++j) ly.y[j] = a.layer[l].y[j];
+      ly.ws_out = a.layer[l].ws_out;
+    }
+  } else {
+    LayerDev& ly = prm.layers[0];
+    ly.m0 = a.m0; ly.shift = a.shift; ly.bias = a.bias;
+    for (int j = 0; j < a.njobs; ++j) ly.y[j] = a.jobs[j].y;
+    ly.ws_out = a.ws_out;
+  }
   prm.skip_c = a.skip_c; prm.skip_d = a.skip_d;
   prm.upsample = a.upsample; prm.scale_main = a.scale_main; prm.has_skip = a.has_skip;
   prm.bn = BN;
   prm.acc_small = a.acc_bound < (1LL << 22) ? 1 : 0;
   prm.cin_chunks = a.cin / bk;
-  prm.ws_out = a.ws_out;
   prm.out_pad = a.out_pad;
   prm.a_planes = flat ? (a.a_planes > 1 ? a.a_planes : 1) : 1;
   prm.plane_rows = (int32_t)rows;
   prm.split_w = a.split_w;
-  if (a.ws_out) {
+  bool chained = a.ws_out != nullptr;
+  for (int l = 0; l < nlayers && nlayers > 1; ++l) chained |= a.layer[l].ws_out != nullptr;
+  if (chained) {
     int64_t orows = 0;
     for (int j = 0; j < a.njobs; ++j) {
       ConvJobDev& jb = prm.jobs[j];
@@ -1364,10 +1385,8 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
     }
   }
   prm.status = a.status;
-  prm.dep_wait = a.dep_wait;
-  prm.dep_signal = a.dep_signal;
+  prm.dep = nlayers > 1 ? a.dep : nullptr;
   prm.dep_target = (uint32_t)(2 * kEpiWarps);  // epilogue warps of both CTAs of a pair
-  prm.dep_split = a.dep_split;
   // shared memory plan: stages of (BM x bk A bytes + this CTA's B rows x bk bytes)
   const int b_rows = pair ? BN / 2 : BN;
   const size_t stage_a = (size_t)kSub * 128 * bk;
@@ -1396,23 +1415,26 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
 
   EncodeTiledFn enc = get_encode_fn(err);
   if (!enc) return 3;
-  CUtensorMap map;
+  Maps maps{};
   cuuint64_t gdim[2] = {(cuuint64_t)a.k_pad, (cuuint64_t)w_rows};
   cuuint64_t gstride[1] = {(cuuint64_t)a.k_pad};
   cuuint32_t box[2] = {(cuuint32_t)bk, (cuuint32_t)b_rows};
   cuuint32_t estr[2] = {1, 1};
   const CUtensorMapSwizzle swz = bk == 64 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B;
-  CUresult r = enc(&map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)a.w_e4m3, gdim, gstride, box, estr,
-                   CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
-                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  if (r != CUDA_SUCCESS) { *err = "cuTensorMapEncodeTiled failed: " + std::to_string((int)r); return 3; }
+  for (int l = 0; l < nlayers; ++l) {
+    const uint8_t* wl = nlayers > 1 ? a.layer[l].w_e4m3 : a.w_e4m3;
+    const CUresult r = enc(&maps.w[l], CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)wl, gdim, gstride, box, estr,
+                           CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) { *err = "cuTensorMapEncodeTiled failed: " + std::to_string((int)r); return 3; }
+  }
   // the same weights with boxes of half the rows, for the half-width tiles
-  CUtensorMap map_h = map;
-  if (prm.dp_tiles < prm.total_tiles) {
+  maps.wh = maps.w[0];
+  if (prm.dp_tiles < prm.layer_tiles) {
     cuuint32_t box_h[2] = {(cuuint32_t)bk, (cuuint32_t)(b_rows / 2)};
-    r = enc(&map_h, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)a.w_e4m3, gdim, gstride, box_h, estr,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
-            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    const CUresult r = enc(&maps.wh, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)a.w_e4m3, gdim, gstride, box_h, estr,
+                           CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) { *err = "cuTensorMapEncodeTiled (half) failed: " + std::to_string((int)r); return 3; }
   }
 
@@ -1420,7 +1442,6 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   int grid = units < sms ? units : sms;
   if (pair) grid = 2 * (units < sms / 2 ? units : sms / 2);
   const bool in_tap = (a.cin % BK) == 0;
-  CUtensorMap map_a = map;  // unused unless flat
   if (flat) {
     // 1) expand the packed codes of every job into the zero-padded byte workspace (unless
     //    the caller expanded them already)
@@ -1456,42 +1477,45 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
       if (e != cudaSuccess) { *err = std::string("expand launch: ") + cudaGetErrorString(e); return 3; }
     }
     if (a.expand_only) return 0;
-    // 2) tensor map over the workspace as a [rows][cin] byte matrix with bk x 128 boxes
+    // 2) tensor maps over the workspace (and, for chained layers in one launch, the second
+    //    image) as [rows][cin] byte matrices with bk x 128 boxes
     cuuint64_t gd[2] = {(cuuint64_t)a.cin, (cuuint64_t)rows * (cuuint64_t)prm.a_planes};
     cuuint64_t gs[1] = {(cuuint64_t)a.cin};
     cuuint32_t bx[2] = {(cuuint32_t)bk, 128};
-    CUresult r2 = enc(&map_a, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)a.ws, gd, gs, bx, estr,
-                      CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
-                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    if (r2 != CUDA_SUCCESS) {
-      *err = "cuTensorMapEncodeTiled (activations) failed: " + std::to_string((int)r2);
-      return 3;
+    for (int i = 0; i < (nlayers > 1 ? 2 : 1); ++i) {
+      const CUresult r2 = enc(&maps.a[i], CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)(i == 0 ? a.ws : a.ws2), gd, gs, bx,
+                              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+                              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+      if (r2 != CUDA_SUCCESS) {
+        *err = "cuTensorMapEncodeTiled (activations) failed: " + std::to_string((int)r2);
+        return 3;
+      }
     }
     if (a.split_w) {  // (no skip: the API keeps skips off the split form)
-      if (pair) return launch_bits<2, true, true, true, false, true>(prm, map, map_h, map_a, grid, smem, stream, err);
-      return launch_bits<2, true, true, false, false, true>(prm, map, map_h, map_a, grid, smem, stream, err);
+      if (pair) return launch_bits<2, true, true, true, false, true>(prm, maps, grid, smem, stream, err);
+      return launch_bits<2, true, true, false, false, true>(prm, maps, grid, smem, stream, err);
     }
     if (bk == 64) {
       if (pair)
-        return a.has_skip ? launch_bits<2, true, true, true, true, false, 64>(prm, map, map_h, map_a, grid, smem, stream, err)
-                          : launch_bits<2, true, true, true, false, false, 64>(prm, map, map_h, map_a, grid, smem, stream, err);
-      return a.has_skip ? launch_bits<2, true, true, false, true, false, 64>(prm, map, map_h, map_a, grid, smem, stream, err)
-                        : launch_bits<2, true, true, false, false, false, 64>(prm, map, map_h, map_a, grid, smem, stream, err);
+        return a.has_skip ? launch_bits<2, true, true, true, true, false, 64>(prm, maps, grid, smem, stream, err)
+                          : launch_bits<2, true, true, true, false, false, 64>(prm, maps, grid, smem, stream, err);
+      return a.has_skip ? launch_bits<2, true, true, false, true, false, 64>(prm, maps, grid, smem, stream, err)
+                        : launch_bits<2, true, true, false, false, false, 64>(prm, maps, grid, smem, stream, err);
     }
     if (pair)
-      return a.has_skip ? launch_bits<2, true, true, true, true>(prm, map, map_h, map_a, grid, smem, stream, err)
-                        : launch_bits<2, true, true, true, false>(prm, map, map_h, map_a, grid, smem, stream, err);
-    return a.has_skip ? launch_bits<2, true, true, false, true>(prm, map, map_h, map_a, grid, smem, stream, err)
-                      : launch_bits<2, true, true, false, false>(prm, map, map_h, map_a, grid, smem, stream, err);
+      return a.has_skip ? launch_bits<2, true, true, true, true>(prm, maps, grid, smem, stream, err)
+                        : launch_bits<2, true, true, true, false>(prm, maps, grid, smem, stream, err);
+    return a.has_skip ? launch_bits<2, true, true, false, true>(prm, maps, grid, smem, stream, err)
+                      : launch_bits<2, true, true, false, false>(prm, maps, grid, smem, stream, err);
   }
   // in-kernel unpacking; the instantiation without skip code keeps its registers for the
   // common case
 #define AQD_INKERNEL(B)                                                                                  \
   if (a.has_skip)                                                                                          \
-    return in_tap ? launch_bits<B, true, false, false, true>(prm, map, map_h, map_a, grid, smem, stream, err) \
-                  : launch_bits<B, false, false, false, true>(prm, map, map_h, map_a, grid, smem, stream, err); \
-  return in_tap ? launch_bits<B, true, false, false, false>(prm, map, map_h, map_a, grid, smem, stream, err)   \
-                : launch_bits<B, false, false, false, false>(prm, map, map_h, map_a, grid, smem, stream, err);
+    return in_tap ? launch_bits<B, true, false, false, true>(prm, maps, grid, smem, stream, err) \
+                  : launch_bits<B, false, false, false, true>(prm, maps, grid, smem, stream, err); \
+  return in_tap ? launch_bits<B, true, false, false, false>(prm, maps, grid, smem, stream, err)   \
+                : launch_bits<B, false, false, false, false>(prm, maps, grid, smem, stream, err);
   switch (a.x_bits) {
     case 2: { AQD_INKERNEL(2) }
     case 3: { AQD_INKERNEL(3) }

@@ -8,6 +8,7 @@
 namespace aqd {
 
 constexpr int kMaxJobs = 8;
+constexpr int kMaxLayers = 4;  // chained layers of one shape in one tensor-core launch
 
 struct ConvJobDev {
   const uint8_t* x;
@@ -60,21 +61,27 @@ struct ConvArgs {
   uint8_t* ws_out;        // chained output: also write the output codes as the next conv's byte image
   int32_t out_pad;        // padding of that next conv
   uint32_t* status;       // device status word
-  // tile-by-tile chaining of stride-1 layers (workspace path, CTA pairs, one N tile): per-tile
-  // counters of the previous layer to wait on (NULL: wait for the whole previous grid), and
-  // this layer's counters to raise (NULL: none)
-  const uint32_t* dep_wait;
-  uint32_t* dep_signal;
-  int32_t dep_split;      // the previous layer's first M tile run as two half-width tiles
   uint32_t* zero;         // words cleared by the expansion pass before the conv (NULL: none)
   int32_t zero_words;
+  // Several chained layers of this shape in one launch (workspace path, CTA pairs, one N
+  // tile): layer l reads ws for even l and ws2 for odd l, and writes layer[l].ws_out (the
+  // other image); its tiles wait on the per-tile counters dep of layer l - 1 (see conv_tc.cu).
+  // nlayers <= 1: one layer, described by the fields above.
+  int32_t nlayers;
+  struct Layer {
+    const uint8_t* w_e4m3;
+    const int32_t* m0;
+    const int8_t* shift;
+    const int32_t* bias;
+    uint8_t* y[kMaxJobs];
+    uint8_t* ws_out;
+  } layer[kMaxLayers];
+  uint8_t* ws2;
+  uint32_t* dep;
 };
-// Tiles of one grouped workspace-path launch on CTA pairs with one N tile (the length of its
-// per-tile counter array).
+// Tiles of one layer of a grouped workspace-path launch on CTA pairs with one N tile (the
+// per-layer length of a chained launch's counter array).
 int64_t conv_tc_pair_tiles(const ConvArgs& a);
-// The first tile that such a launch splits into two half-width tiles (its last, partial wave;
-// the tile count when it splits none).
-int64_t conv_tc_pair_split(const ConvArgs& a);
 
 // Prepared-weight geometry shared by the API and the weight-prep kernel.
 struct WeightGeom {

@@ -145,7 +145,7 @@ def test_graph_replays_and_back_to_back_calls():
 
 
 def test_tower_argument_errors():
-    levels = [(6, 9)]
+    levels = [(20, 34)]  # three tiles per layer: the two fused tower layers need 12 bytes of counters
     wl = synth.head_tower(72, 1, 2, levels=levels, calibrated=True)
     t = Tower(wl, 2, ntower=2)
     # layer 1's input is not layer 0's output
@@ -155,7 +155,8 @@ def test_tower_argument_errors():
         aqd.conv_int_grouped_tower(bad, [w for w, _ in t.W] + [t.Wh[0]], t.rqs + [t.rqh], 1, ws_a=t.ws_a,
                                    ws_b=t.ws_b, sync=t.sync)
     assert e.value.status == 1
-    # counters too small
+    # counters too small (4 of the 12 bytes)
+    assert aqd.tower_sync_bytes(t.layer_jobs[0], 2, 1) == 12
     with pytest.raises(aqd.AqdError) as e:
         aqd.conv_int_grouped_tower(t.layer_jobs, [w for w, _ in t.W] + [t.Wh[0]], t.rqs + [t.rqh], 1,
                                    ws_a=t.ws_a, ws_b=t.ws_b, sync=t.sync[:4])

@@ -134,12 +134,21 @@ aqd_status aqd_device_status(aqd_stream_t stream, int32_t* code);
 
 /* Diagnostics: force the convolution kernel (0 = automatic choice, 1 = tensor-core
  * kernel when the shape allows it, 2 = CUDA-core kernel, 3 = as 1 but never on CTA
- * pairs); returns the previous setting, or -1 for an unknown value. aqd_last_conv_path()
- * reports the kernel the calling thread's last successful conv call used (1 tensor core
- * unpacking in-kernel, 2 CUDA core, 3 tensor core fed from the expanded workspace, 4 the
- * same on CTA pairs sharing each weight tile, 5 the F16 tensor-core kernel of a network's
- * first conv on a 3-channel 8-bit image with a 7x7 kernel, 0 none yet). Forcing 2 also
- * turns path 5 off. */
+ * pairs, 4 = as 1 but never on the FP4 pipe, 5 = as 1 but on neither); returns the previous
+ * setting, or -1 for an unknown value. aqd_last_conv_path() reports the kernel the calling thread's last
+ * successful conv call used (1 tensor core unpacking in-kernel, 2 CUDA core, 3 tensor core
+ * fed from the expanded workspace, 4 the same on CTA pairs sharing each weight tile, 5 the
+ * F16 tensor-core kernel of a network's first conv on a 3-channel 8-bit image with a 7x7
+ * kernel, 6 the FP4 tensor-core pipe for 2-bit codes, 0 none yet). Forcing 2 also turns
+ * paths 5 and 6 off.
+ *
+ * The FP4 pipe (path 6, kind::mxf4nvf4 with unit block scales) takes 2-bit activation codes
+ * with weights |w| <= 4 (2-bit two's complement or Eq. 3's odd grid, 3-bit two's complement),
+ * cin % 256 == 0 and at most 240 output channels per tile, on the workspace path, in
+ * aqd_conv_int / aqd_conv_int_grouped (which expand their own input) and for the last layer
+ * of aqd_conv_int_grouped_tower; each code and weight is the E2M1 value n / 2, w / 2, so
+ * every product is exact and the FP32 sum is 1/4 of the integer sum, as exact as the E4M3
+ * embedding. The split calls (expand / expanded / chain) always use byte images. */
 int32_t aqd_set_conv_path(int32_t path);
 int32_t aqd_last_conv_path(void);
 

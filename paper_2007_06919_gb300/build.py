@@ -41,6 +41,9 @@ def _compile(src):
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"nvcc failed for {src}:\n{r.stdout}\n{r.stderr}")
+    # ptxas's warnings (register spills, by function) beside the object, for the build checks
+    with open(obj[:-2] + ".log", "w") as f:
+        f.write(r.stderr)
     return obj
 
 

@@ -17,7 +17,9 @@ namespace aqd {
 
 static thread_local std::string g_last_error;
 static thread_local int32_t g_last_path = 0;
-static int32_t g_forced_path = 0;  // 0 auto, 1 tensor core, 2 direct, 3 tensor core without CTA pairs
+// 0 auto, 1 tensor core, 2 direct, 3 tensor core without CTA pairs, 4 tensor core without the
+// FP4 pipe, 5 tensor core without either
+static int32_t g_forced_path = 0;
 
 __device__ uint32_t g_status_word;
 
@@ -100,7 +102,9 @@ WeightGeom weight_geom(int32_t cout, int32_t kh, int32_t kw, int32_t cin) {
   // 128 rows of w_hi = w >> 4 (floor), so it is sized for the larger of the two
   g.e4m3_bytes = (size_t)(g.cout_pad > g.split_rows ? g.cout_pad : g.split_rows) * g.k_pad;
   g.i16_offset = (g.e4m3_bytes + 255) / 256 * 256;
-  g.total_bytes = g.i16_offset + 2 * (size_t)cout * g.k_total;
+  g.fp4_offset = (g.i16_offset + 2 * (size_t)cout * g.k_total + 255) / 256 * 256;
+  g.fp4_bytes = (size_t)g.cout_pad * (size_t)(g.k_pad / 2);
+  g.total_bytes = g.fp4_offset + g.fp4_bytes;
   return g;
 }
 
@@ -181,7 +185,7 @@ aqd_status aqd_device_status(aqd_stream_t stream, int32_t* code) {
 }
 
 int32_t aqd_set_conv_path(int32_t path) {
-  if (path < 0 || path > 3) return -1;
+  if (path < 0 || path > 5) return -1;
   const int32_t old = g_forced_path;
   g_forced_path = path;
   return old;
@@ -321,10 +325,15 @@ struct ConvPlan {
 
 // Validates one grouped call and decides its kernel; launches nothing. require_ws: the call
 // must run on the expanded-activation workspace path (else AQD_ERR_UNSUPPORTED).
+// in_nib: the workspace image the convolution reads is a nibble image (two 2-bit codes per
+// byte, written by a previous layer for this one); then the convolution must run on the FP4
+// pipe (else AQD_ERR_UNSUPPORTED). A convolution that expands its own input (kStageBoth) takes
+// the FP4 pipe whenever it applies; the other stages read byte images.
 static aqd_status plan_grouped(const aqd_conv_job* jobs, int32_t njobs, const aqd_conv_weights* w,
                                int32_t stride, int32_t pad, const aqd_requant_params* rq,
                                const aqd_skip_params* sp, void* workspace, size_t ws_bytes,
-                               ConvStage stage, const ChainOut* chain, bool require_ws, ConvPlan* plan) {
+                               ConvStage stage, const ChainOut* chain, bool require_ws, ConvPlan* plan,
+                               bool in_nib = false) {
   std::string err;
   if (!jobs || njobs <= 0 || njobs > kMaxJobs) return fail(AQD_ERR_INVALID, "njobs must be 1..8");
   if (!check_weights(w, &err)) return fail(AQD_ERR_INVALID, err);
@@ -417,8 +426,8 @@ static aqd_status plan_grouped(const aqd_conv_job* jobs, int32_t njobs, const aq
   // the network's first conv (3-channel 8-bit image, 7x7): its own F16 tensor-core kernel
   const bool stem_ok = !tc_ok && !wide_ok && stage == kStageBoth && stem_applicable(a);
   int path = (tc_ok || wide_ok) ? 1 : (stem_ok ? 5 : 2);
-  if ((g_forced_path == 1 || g_forced_path == 3) && (tc_ok || wide_ok)) path = 1;
-  a.no_pair = g_forced_path == 3 ? 1 : 0;
+  if (g_forced_path != 0 && g_forced_path != 2 && (tc_ok || wide_ok)) path = 1;
+  a.no_pair = (g_forced_path == 3 || g_forced_path == 5) ? 1 : 0;
   if (g_forced_path == 2) path = 2;
   // expanded-activation path when a large enough, aligned workspace is supplied
   a.ws = nullptr;
@@ -465,6 +474,18 @@ static aqd_status plan_grouped(const aqd_conv_job* jobs, int32_t njobs, const aq
     a.out_pad = chain->pad;
   }
   a.expand_only = stage == kStageExpandOnly ? 1 : 0;
+  // The FP4 pipe (kind::mxf4nvf4): 2-bit codes and weights exact as E2M1 values w / 2
+  // (|w| <= 4), read from a nibble image in 128-byte chunks (cin % 256 == 0), tiles of at most
+  // 240 channels (TMEM holds two accumulators and the scales), one launch of one layer that
+  // chains nothing; the accumulator bound keeps the FP32 sum exact (|sum| / 4 < 2^24).
+  const bool fp4_ok = path == 1 && a.ws && !a.split_w && a.a_planes == 1 && a.x_bits == 2 && a.cin % 256 == 0 &&
+                      fp4_weights(w->w_bits, w->w_format) && 2 * g.bn + 32 <= 512 && !a.ws_out &&
+                      stage != kStageExpandOnly && g_forced_path != 4 && g_forced_path != 5 && bound < (1LL << 24);
+  if (in_nib && !fp4_ok) return fail(AQD_ERR_UNSUPPORTED, "the FP4 pipe does not take this convolution");
+  if (fp4_ok && (in_nib || stage == kStageBoth)) {
+    a.fp4 = 1;
+    a.w_fp4 = static_cast<const uint8_t*>(w->data) + g.fp4_offset;
+  }
   plan->path = path;
   return AQD_OK;
 }
@@ -477,7 +498,7 @@ static aqd_status launch_plan(const ConvPlan& plan, aqd_stream_t stream) {
   int rc = path == 1 ? launch_conv_tc(a, st, &err) : path == 5 ? launch_stem(a, st, &err) : launch_conv_direct(a, st, &err);
   if (rc) return fail((aqd_status)rc, err);
   if (plan.stage != kStageExpandOnly)
-    g_last_path = (path == 1 && a.ws) ? (conv_tc_uses_pair(a) ? 4 : 3) : path;
+    g_last_path = (path == 1 && a.ws) ? (a.fp4 ? 6 : conv_tc_uses_pair(a) ? 4 : 3) : path;
   return AQD_OK;
 }
 
@@ -604,6 +625,18 @@ aqd_status aqd_conv_int_grouped_tower(const aqd_conv_job* jobs, int32_t njobs, i
       return s;
     }
   }
+  // The last layer runs on the FP4 pipe when it applies: the layer before it then writes its
+  // chained output as a nibble image.
+  if (layers > 1 && plans[layers - 2].a.out_bits == 2) {
+    ConvPlan last;
+    const aqd_status st4 = plan_grouped(jobs + (size_t)(layers - 1) * njobs, njobs, &w[layers - 1], 1, pad,
+                                        &rq[layers - 1], nullptr, (layers - 1) % 2 == 0 ? ws_a : ws_b, ws_bytes,
+                                        kStageConvOnly, nullptr, true, &last, true);
+    if (st4 == AQD_OK) {
+      plans[layers - 1] = last;
+      plans[layers - 2].a.ws_out_nib = 1;
+    }
+  }
   // The longest prefix of layers of one shape (same weights geometry and code widths, chained
   // 2/3/4-bit outputs, CTA pairs with one N tile) runs as one launch when the caller gave
   // counters: layer l + 1's tiles start as soon as the tiles of layer l they read are stored.
@@ -636,6 +669,7 @@ aqd_status aqd_conv_int_grouped_tower(const aqd_conv_job* jobs, int32_t njobs, i
       a.layer[l].m0 = b.m0; a.layer[l].shift = b.shift; a.layer[l].bias = b.bias;
       for (int j = 0; j < njobs; ++j) a.layer[l].y[j] = b.jobs[j].y;
       a.layer[l].ws_out = b.ws_out;
+      a.layer[l].ws_nib = b.ws_out_nib;
     }
     a.ws2 = static_cast<uint8_t*>(ws_b);
     a.dep = static_cast<uint32_t*>(sync);

@@ -9,6 +9,14 @@
 // times 2^-18, and the FP32 accumulator holds the exact integer sum times 2^-18 as long as
 // K * max|x| * max|w| < 2^24, which the host checks before choosing this kernel.
 //
+// 2-bit codes on the FP4 pipe (kFp4): E2M1 holds n / 2 exactly for n <= 4, so a code n and a
+// weight |w| <= 4 become the E2M1 values n / 2 and w / 2 (raw nibbles n and sign | |w|), every
+// product is an integer / 4, and kind::mxf4nvf4 (K = 64 per instruction, one UE8M0 scale
+// per 32 K elements, all set to 2^0 in TMEM) accumulates the exact integer sum / 4 in FP32.
+// Operands are nibble images (two codes per byte), so a 128-byte K chunk holds 256 codes. A
+// nibble image keeps the byte image's row stride (cin bytes) and fills the first cin / 2
+// bytes of each row, so its zero border lies where a byte image's does in the same workspace.
+//
 // Per CTA (one per SM, persistent over tiles of 128 output pixels x BN channels):
 //   warps 0..E-1  epilogue (E = 4 or 8): tcgen05.ld of the accumulator, integer epilogue,
 //              bit-pack, store (warp w reads TMEM lanes 32*(w%4)..; with 8 warps each takes
@@ -67,6 +75,7 @@ constexpr int kTmaWarpsFlat = 3;
 __host__ __device__ constexpr int tma_warps(bool flat) { return flat ? kTmaWarpsFlat : kTmaWarps; }
 __host__ __device__ constexpr int threads_for(bool flat) { return flat ? (kWarpTma + kTmaWarpsFlat) * 32 : kThreads; }
 constexpr int kMaxStages = 16;
+constexpr int kStageRow = 36;  // words per row of an int32 staging block (16-byte aligned, conflict-free)
 constexpr int kQTab = 256;  // K-chunk table entries (larger K falls back to division)
 
 // One layer of a launch: its per-channel tables, the packed output of each job and the
@@ -77,6 +86,7 @@ struct LayerDev {
   const int32_t* bias;
   uint8_t* y[kMaxJobs];
   uint8_t* ws_out;
+  int32_t ws_nib;  // ws_out holds two 2-bit codes per byte (the next layer runs on the FP4 pipe)
 };
 
 // The tensor maps of a launch: the weights of each layer, the weights with half-height
@@ -102,6 +112,7 @@ struct Params {
   int32_t dp_tiles;   // tiles [0, dp_tiles) are bn wide; later ones are the two bn/2 halves
                       // of the remaining full tiles (the last, partial wave)
   uint32_t off_b, off_epi, off_bar, off_qtab;
+  uint32_t off_ostage;  // int32 outputs: per-warp staging blocks for row-contiguous stores (0: none)
   int32_t out_pad;
   int32_t a_planes;   // K runs over this many planes of the byte image (2: 8-bit activations)
   int32_t plane_rows; // workspace rows per plane
@@ -118,6 +129,7 @@ struct Params {
   // tiles before loading A.
   int32_t nlayers, layer_tiles;
   LayerDev layers[kMaxLayers];
+  int32_t sf_col;     // FP4: first of the 32 TMEM columns that hold the unit block scales
   uint32_t* dep;
   uint32_t dep_target;
 };
@@ -250,9 +262,10 @@ __device__ __forceinline__ void load_skip_group(const Params& p, const uint8_t* 
 
 // Eq. 6 -> Eq. 7 -> Eq. 2 in int64 for 32 accumulators of one row (any shift, any skip),
 // element by element as the definition states it; the common cases take 32-bit forms.
+// (sc: the FP32 accumulator holds the integer sum / sc: 2^18 on the E4M3 pipe, 4 on the FP4 one)
 template <bool kSkip, bool kIntAcc = false>
 __device__ __forceinline__ void general_group(const Params& p, const uint32_t* v, const EpiChan* ep,
-                                              const uint8_t* srow, int ch0, int ncols, int32_t (&out)[32]) {
+                                              const uint8_t* srow, int ch0, int ncols, float sc, int32_t (&out)[32]) {
   int32_t sk[32];
   if (kSkip && p.has_skip) load_skip_group(p, srow, ch0, ncols, sk);
   else {
@@ -263,7 +276,7 @@ __device__ __forceinline__ void general_group(const Params& p, const uint32_t* v
   for (int i = 0; i < 32; ++i) {
     // v: FP32 accumulators of exact integers x 2^-18, or (kIntAcc) int32 sums already
     const int64_t acc = kIntAcc ? (int64_t)(int32_t)v[i]
-                                : (int64_t)__float2int_rn(__uint_as_float(v[i]) * 262144.0f);
+                                : (int64_t)__float2int_rn(__uint_as_float(v[i]) * sc);
     const EpiChan ec = ep[i];
     out[i] = (kSkip && p.has_skip) ? epilogue<true>(acc, sk[i], ec, p.scale_main, p.out_bits)
                         : epilogue<false>(acc, 0, ec, p.scale_main, p.out_bits);
@@ -280,11 +293,11 @@ __device__ __forceinline__ void general_group(const Params& p, const uint32_t* v
 // exact sum; the requant is the same 32-bit form as fast_requant_group.
 // (y may be sk itself: element i is read before it is written)
 __device__ __forceinline__ void fast_skip_group(const uint32_t* v, const EpiChan* ep, const int32_t (&sk)[32],
-                                                int qmax, int32_t (&y)[32]) {
+                                                int qmax, float sc, int32_t (&y)[32]) {
 #pragma unroll
   for (int i = 0; i < 32; ++i) {
     const EpiChan c = ep[i];
-    const int32_t acc = __float2int_rn(__uint_as_float(v[i]) * 262144.0f);  // exact integer
+    const int32_t acc = __float2int_rn(__uint_as_float(v[i]) * sc);  // exact integer
     const int64_t sc = (int64_t)sk[i] * (int64_t)c.c;
     const int32_t st = (int32_t)((sc + (1LL << (c.d - 1))) >> c.d);
     const int32_t u = add_sat(acc + c.bias, st);
@@ -299,11 +312,11 @@ __device__ __forceinline__ void fast_skip_group(const uint32_t* v, const EpiChan
 // int32 (|acc| < 2^24); the sum is saturated to int32 as in Eq. 7's int64 form, and the requant
 // is the 32-bit form of fast_requant_group.
 __device__ __forceinline__ void fast_skip32_group(const uint32_t* v, const EpiChan* ep, const int32_t (&sk)[32],
-                                                  int qmax, int32_t (&y)[32]) {
+                                                  int qmax, float sc, int32_t (&y)[32]) {
 #pragma unroll
   for (int i = 0; i < 32; ++i) {
     const EpiChan c = ep[i];
-    const int32_t acc = __float2int_rn(__uint_as_float(v[i]) * 262144.0f);  // exact integer
+    const int32_t acc = __float2int_rn(__uint_as_float(v[i]) * sc);  // exact integer
     const int64_t st = ((int64_t)sk[i] * (int64_t)c.c + (1LL << (c.d - 1))) >> c.d;
     int64_t t = (int64_t)(acc + c.bias) + st;
     t = t > 2147483647LL ? 2147483647LL : (t < -2147483648LL ? -2147483648LL : t);
@@ -320,14 +333,14 @@ constexpr uint32_t kMagicBits = 0x4B400000u;
 // Fast requant of 32 accumulators of one row into one packed group (no skip, R >= 33,
 // any bias): u = sat32(acc + bias), y = clamp((mulhi(u, M0) + 2^(R-33)) >> (R-32), 0, 2^k-1).
 template <int kOut>
-__device__ __forceinline__ void fast_requant_group(const uint32_t* v, const EpiChan* ep, int g0, int qmax,
+__device__ __forceinline__ void fast_requant_group(const uint32_t* v, const EpiChan* ep, int g0, int qmax, float sc,
                                                    uint32_t gw[8]) {
 #pragma unroll
   for (int w = 0; w < 8; ++w) gw[w] = 0u;
 #pragma unroll
   for (int i = 0; i < 32; ++i) {
     const EpiChan c = ep[g0 + i];
-    const int32_t acc = __float2int_rn(__uint_as_float(v[i]) * 262144.0f);  // exact integer
+    const int32_t acc = __float2int_rn(__uint_as_float(v[i]) * sc);  // exact integer
     const int32_t u = add_sat(acc, c.bias);
     const int r = c.r;
     const uint32_t y = (uint32_t)__vimin_s32_relu((__mulhi(u, c.m0) + (1 << (r - 33))) >> (r - 32), qmax);
@@ -344,16 +357,17 @@ __device__ __forceinline__ void fast_requant_group(const uint32_t* v, const EpiC
 // Fastest requant (no skip, R >= 33, |acc| < 2^22, |bias| <= 2^30) of 32 accumulators of one
 // row, straight into 8 byte-words (word j holds channels 4j..4j+3, one code per byte: the
 // layout of the chained byte image, and one step from every packed layout). One FMA turns
-// the accumulator float acc * 2^-18 into the int32 acc + 0x4B400000; c.x holds
+// the accumulator float acc / sc into the int32 acc + 0x4B400000; c.x holds
 // bias - 0x4B400000, so one add gives acc + bias exactly (no int32 overflow under the stated
 // bounds); c.y, c.z, c.w are M0, 2^(R-33) and R-32.
-__device__ __forceinline__ void magic_requant_bytes(const uint32_t* v, const int4* f, int qmax, uint32_t (&bw)[8]) {
+__device__ __forceinline__ void magic_requant_bytes(const uint32_t* v, const int4* f, int qmax, float sc,
+                                                    uint32_t (&bw)[8]) {
 #pragma unroll
   for (int j = 0; j < 8; ++j) bw[j] = 0u;
 #pragma unroll
   for (int i = 0; i < 32; ++i) {
     const int4 c = f[i];
-    const int32_t u = __float_as_int(__fmaf_rn(__uint_as_float(v[i]), 262144.0f, kMagic)) + c.x;
+    const int32_t u = __float_as_int(__fmaf_rn(__uint_as_float(v[i]), sc, kMagic)) + c.x;
     const uint32_t y = (uint32_t)__vimin_s32_relu((__mulhi(u, c.y) + c.z) >> c.w, qmax);
     bw[i / 4] += y << (8 * (i % 4));  // codes < 256: the add is an or
   }
@@ -384,29 +398,39 @@ __device__ __forceinline__ void pack_bytewords(const uint32_t (&bw)[8], uint32_t
     gw[2] = h;
   }
 }
-// Chained output from byte-words (see chain_store).
-__device__ __forceinline__ void chain_store_bytes(const Params& p, uint8_t* ws_out, const ConvJobDev& jb, int img,
-                                                  int oh, int ow, int ch0, const uint32_t (&bw)[8]) {
+// Chained output: the 32 codes of one packed group (byte-words bw: channels 4j..4j+3 in word
+// j) at their place in the zero-padded image that the next stride-1 conv (padding out_pad)
+// reads: one byte per code, or, when that conv runs on the FP4 pipe (nib), two codes per byte
+// (channel 2k in the low nibble of byte k) in the first half of the same row.
+__device__ __forceinline__ void chain_store_bw(const Params& p, uint8_t* ws_out, int nib, const ConvJobDev& jb,
+                                               int img, int oh, int ow, int ch0, const uint32_t (&bw)[8]) {
   const int row = jb.orow_off + (img * jb.ohp + oh + p.out_pad) * jb.owp + ow + p.out_pad;
-  uint4* dst = reinterpret_cast<uint4*>(ws_out + (size_t)row * p.cout + ch0);
-  dst[0] = make_uint4(bw[0], bw[1], bw[2], bw[3]);
-  dst[1] = make_uint4(bw[4], bw[5], bw[6], bw[7]);
+  if (nib) {
+    uint32_t o[4];
+#pragma unroll
+    for (int m = 0; m < 4; ++m) {
+      // bytes 0 and 2 of t hold the nibble pairs (c0, c1) and (c2, c3) of a byte-word
+      const uint32_t t0 = bw[2 * m] | (bw[2 * m] >> 4), t1 = bw[2 * m + 1] | (bw[2 * m + 1] >> 4);
+      o[m] = __byte_perm(t0, t1, 0x6420);
+    }
+    *reinterpret_cast<uint4*>(ws_out + (size_t)row * p.cout + (ch0 >> 1)) = make_uint4(o[0], o[1], o[2], o[3]);
+  } else {
+    uint4* dst = reinterpret_cast<uint4*>(ws_out + (size_t)row * p.cout + ch0);
+    dst[0] = make_uint4(bw[0], bw[1], bw[2], bw[3]);
+    dst[1] = make_uint4(bw[4], bw[5], bw[6], bw[7]);
+  }
 }
 
-// Chained output: the 32 codes of one packed group, one byte each, at their place in the
-// zero-padded byte image that the next stride-1 conv (padding out_pad) reads.
-__device__ __forceinline__ void chain_store(const Params& p, uint8_t* ws_out, const ConvJobDev& jb, int img, int oh,
-                                            int ow, int ch0, const uint32_t gw[8], int out_bits) {
+// The same from a packed group gw of out_bits codes.
+__device__ __forceinline__ void chain_store(const Params& p, uint8_t* ws_out, int nib, const ConvJobDev& jb, int img,
+                                            int oh, int ow, int ch0, const uint32_t gw[8], int out_bits) {
   uint32_t o[8];
   switch (out_bits) {
     case 2: unpack_group_bytes<2>(gw, o); break;
     case 3: unpack_group_bytes<3>(gw, o); break;
     default: unpack_group_bytes<4>(gw, o); break;
   }
-  const int row = jb.orow_off + (img * jb.ohp + oh + p.out_pad) * jb.owp + ow + p.out_pad;
-  uint4* dst = reinterpret_cast<uint4*>(ws_out + (size_t)row * p.cout + ch0);
-  dst[0] = make_uint4(o[0], o[1], o[2], o[3]);
-  dst[1] = make_uint4(o[4], o[5], o[6], o[7]);
+  chain_store_bw(p, ws_out, nib, jb, img, oh, ow, ch0, o);
 }
 
 // ---------------------------------------------------------------- the kernel
@@ -471,11 +495,17 @@ __device__ __forceinline__ void load_chunk(const Params& p, RowCursor<kXBits>& r
 // kSkip: the instantiation that handles a skip tensor (Eq. 7); the others carry no skip code,
 // which keeps the common path's registers free.
 // kSplit: the 8-bit split form (split weights combined as D1 + 16 D2 in the epilogue).
-template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair, bool kSkip, bool kSplit, int kBK>
+// kOStage: int32 outputs go through per-warp shared-memory staging blocks (an instantiation of
+// its own, so that the other forms keep their registers)
+template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair, bool kSkip, bool kSplit, int kBK, bool kFp4,
+          bool kOStage>
 __global__ void __launch_bounds__(threads_for(kFlat), 1)
 conv_tc_kernel(const __grid_constant__ Maps maps, const __grid_constant__ Params p) {
   static_assert(!kPair || kFlat, "the CTA-pair form exists for the workspace path only");
   static_assert(kBK == BK || kFlat, "64-byte K chunks exist for the workspace path only");
+  static_assert(!kFp4 || (kFlat && kBK == BK && !kSplit), "the FP4 pipe reads nibble images in 128-byte chunks");
+  // the FP32 accumulator holds the integer sum / kAccSc
+  constexpr float kAccSc = kFp4 ? 4.0f : 262144.0f;
   // bytes of one stage's A operand: kSub sub-tiles of 128 rows x kBK bytes
   constexpr int kStA = kSub * 128 * kBK;
   constexpr int kTma = tma_warps(kFlat);
@@ -554,6 +584,21 @@ conv_tc_kernel(const __grid_constant__ Maps maps, const __grid_constant__ Params
   if constexpr (kPair) cluster_sync();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  if constexpr (kFp4) {
+    // unit block scales (UE8M0 127 = 2^0) in the 32 TMEM columns from sf_col, every lane of
+    // both CTAs of a pair: the MMAs read the A scales from the first 16, the B scales from
+    // the next 16, whatever the scale vectors' layout inside them
+    if (warp < 4) {
+      const uint32_t ta = tmem_base + ((uint32_t)(32 * warp) << 16) + (uint32_t)p.sf_col;
+      tmem_st16_fill(ta, 0x7F7F7F7Fu);
+      tmem_st16_fill(ta + 16, 0x7F7F7F7Fu);
+      tmem_wait_st();
+    }
+    tc_fence_before();
+    __syncthreads();
+    if constexpr (kPair) cluster_sync();
+    tc_fence_after();
+  }
   // everything above overlaps the previous kernel; global memory is touched only after this
   grid_dep_wait();
   if (threadIdx.x == 0) grid_dep_launch();
@@ -565,8 +610,10 @@ conv_tc_kernel(const __grid_constant__ Maps maps, const __grid_constant__ Params
   if (warp == kWarpMma) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0 && leader) {
-      const uint32_t idesc_full = idesc_e4m3(BN, kPair ? 2 * kMmaM : kMmaM);
-      const uint32_t idesc_half = idesc_e4m3(BN / 2, kPair ? 2 * kMmaM : kMmaM);
+      const uint32_t idesc_full = kFp4 ? idesc_fp4(BN, kPair ? 2 * kMmaM : kMmaM) : idesc_e4m3(BN, kPair ? 2 * kMmaM : kMmaM);
+      const uint32_t idesc_half =
+          kFp4 ? idesc_fp4(BN / 2, kPair ? 2 * kMmaM : kMmaM) : idesc_e4m3(BN / 2, kPair ? 2 * kMmaM : kMmaM);
+      const uint32_t sfa = tmem_base + (uint32_t)p.sf_col, sfb = sfa + 16;  // (FP4 only)
       // descriptors of stage 0, k-step 0; later stages / sub-tiles / k-steps add
       // (byte offset >> 4) to the 14-bit start-address field (shared addresses < 2^18)
       // the descriptors' high words are constant; stages / sub-tiles / k-steps only move the
@@ -602,12 +649,17 @@ conv_tc_kernel(const __grid_constant__ Maps maps, const __grid_constant__ Params
             if (kk == kBK / 32 - 1) next_ready = mbar_test(b_full + 8 * s_next, ph_next);
             const uint32_t acc = (q > 0 || kk > 0) ? 1u : 0u;
             const uint64_t db = ((uint64_t)b_hi << 32) | (b_lo + 2 * kk);
-            if constexpr (kPair) {
+            if constexpr (kPair && kFp4) {
+              mma_fp4_pair(d0, ((uint64_t)a_hi << 32) | (a_lo + 2 * kk), db, idesc, sfa, sfb, acc);
+            } else if constexpr (kPair) {
               mma_e4m3_pair(d0, ((uint64_t)a_hi << 32) | (a_lo + 2 * kk), db, idesc, acc);
             } else {
 #pragma unroll
-              for (int j = 0; j < kSub; ++j)
-                mma_e4m3(d0 + j * BN, ((uint64_t)a_hi << 32) | (a_lo + j * (kSubA >> 4) + 2 * kk), db, idesc, acc);
+              for (int j = 0; j < kSub; ++j) {
+                const uint64_t da = ((uint64_t)a_hi << 32) | (a_lo + j * (kSubA >> 4) + 2 * kk);
+                if constexpr (kFp4) mma_fp4(d0 + j * BN, da, db, idesc, sfa, sfb, acc);
+                else mma_e4m3(d0 + j * BN, da, db, idesc, acc);
+              }
             }
           }
           if constexpr (kPair) mma_commit_pair_both(b_empty + 8 * s);
@@ -882,8 +934,8 @@ conv_tc_kernel(const __grid_constant__ Maps maps, const __grid_constant__ Params
           reg_fence32(vb);
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
-            const int32_t d1 = __float2int_rn(__uint_as_float(va[i]) * 262144.0f);
-            const int32_t d2 = (full || i < 16) ? __float2int_rn(__uint_as_float(vb[i]) * 262144.0f) : 0;
+            const int32_t d1 = __float2int_rn(__uint_as_float(va[i]) * kAccSc);
+            const int32_t d2 = (full || i < 16) ? __float2int_rn(__uint_as_float(vb[i]) * kAccSc) : 0;
             va[i] = (uint32_t)(d1 + 16 * d2);
           }
         }
@@ -902,91 +954,46 @@ conv_tc_kernel(const __grid_constant__ Maps maps, const __grid_constant__ Params
           m = ti.mt * BM + sub * 128 + quarter * 32 + lane;
           row_ok = m < jb.m_total;
         }
-        if (row_ok) {
-          uint8_t* yrow = ly.y[ti.job] + (int64_t)m * p.y_row_bytes;
+        if constexpr (kOStage) {
+          // (launched for int32 outputs without a skip only: mode 2)
+          // int32 outputs through this warp's staging block: each lane holds its row's 32
+          // values; stored back four rows at a time, so every warp store covers four whole
+          // 128-byte row segments instead of 32 scattered 16-byte pieces (cout % 4 == 0)
+          uint32_t* stg = reinterpret_cast<uint32_t*>(smem + p.off_ostage) + warp * (32 * kStageRow);
           const int ch0 = ti.col0 + g0;
-          if (mode == 1 && magic) {
-            // codes as byte-words: the chained image takes them as they are, the packed
-            // output a couple of shifts per 8 codes
-            uint32_t bw[8], gw[8];
-            magic_requant_bytes(v, epf + g0, qmax, bw);
-            switch (out_bits) {
-              case 2: pack_bytewords<2>(bw, gw); break;
-              case 3: pack_bytewords<3>(bw, gw); break;
-              case 4: pack_bytewords<4>(bw, gw); break;
-              default: pack_bytewords<8>(bw, gw); break;
-            }
-            store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
-            if (kFlat && ly.ws_out) chain_store_bytes(p, ly.ws_out, jb, oimg, oh, ow, ch0, bw);
-          } else if (mode == 1) {
-            uint32_t gw[8];
-            {
-              switch (out_bits) {
-                case 2: fast_requant_group<2>(v, epi, g0, qmax, gw); break;
-                case 3: fast_requant_group<3>(v, epi, g0, qmax, gw); break;
-                case 4: fast_requant_group<4>(v, epi, g0, qmax, gw); break;
-                default: fast_requant_group<8>(v, epi, g0, qmax, gw); break;
-              }
-            }
-            store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
-            if (kFlat && ly.ws_out) chain_store(p, ly.ws_out, jb, oimg, oh, ow, ch0, gw, out_bits);
-          } else if (mode == 2) {
-            int32_t* yr = reinterpret_cast<int32_t*>(yrow) + ch0;
-            const bool whole = ncols == 32 && ch0 + 32 <= p.cout;
-  #pragma unroll
-            for (int q = 0; q < 8; ++q) {
-              int32_t o[4];
-  #pragma unroll
-              for (int k = 0; k < 4; ++k) {
-                const float f = __uint_as_float(v[4 * q + k]);
-                o[k] = magic ? __float_as_int(__fmaf_rn(f, 262144.0f, kMagic)) + epf[g0 + 4 * q + k].x
-                             : add_sat(__float2int_rn(f * 262144.0f), epi[g0 + 4 * q + k].bias);
-              }
-              if (whole) {
-                reinterpret_cast<int4*>(yr)[q] = make_int4(o[0], o[1], o[2], o[3]);
-              } else {
-  #pragma unroll
-                for (int k = 0; k < 4; ++k)
-                  if (4 * q + k < ncols && ch0 + 4 * q + k < p.cout) yr[4 * q + k] = o[k];
-              }
-            }
-          } else {
-            const uint8_t* srow = nullptr;
-            if (kSkip && p.has_skip) {
-              int img, ho, wo;
-              if constexpr (kFlat) {
-                img = oimg; ho = oh; wo = ow;
-              } else {
-                const int hw = jb.ho * jb.wo;
-                img = m / hw;
-                const int rem = m - img * hw;
-                ho = rem / jb.wo; wo = rem - ho * jb.wo;
-              }
-              const int sh = p.upsample == 2 ? ho >> 1 : ho, sw = p.upsample == 2 ? wo >> 1 : wo;
-              srow = jb.skip + (((int64_t)img * jb.skip_h + sh) * jb.skip_w + sw) * p.skip_row_bytes;
-            }
-            int32_t oo[32];
-            if (kSkip && fast_skip && p.skip_bits <= 8) {
-              load_skip_group(p, srow, ch0, ncols, oo);   // skip codes, replaced by the results
-              fast_skip_group(v, epi + g0, oo, qmax, oo);
-            } else if (kSkip && fast_skip) {
-              load_skip_group(p, srow, ch0, ncols, oo);   // int32 skip, replaced by the results
-              fast_skip32_group(v, epi + g0, oo, qmax, oo);
-            } else {
-              general_group<kSkip, kSplit>(p, v, epi + g0, srow, ch0, ncols, oo);
-            }
-            if (out_bits == 32) {
-              int32_t* yr = reinterpret_cast<int32_t*>(yrow) + ch0;
 #pragma unroll
-              for (int i = 0; i < 32; ++i)
-                if (i < ncols && ch0 + i < p.cout) yr[i] = oo[i];
-            } else {
-              // clipped codes (< 2^out_bits) as byte-words, then the packed group
+          for (int q = 0; q < 8; ++q) {
+            int32_t o[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const float f = __uint_as_float(v[4 * q + k]);
+              o[k] = magic ? __float_as_int(__fmaf_rn(f, kAccSc, kMagic)) + epf[g0 + 4 * q + k].x
+                           : add_sat(__float2int_rn(f * kAccSc), epi[g0 + 4 * q + k].bias);
+            }
+            *reinterpret_cast<int4*>(stg + lane * kStageRow + 4 * q) = make_int4(o[0], o[1], o[2], o[3]);
+          }
+          __syncwarp();
+          const uint32_t rows_ok = __ballot_sync(0xffffffffu, row_ok);
+          const int nq = (ncols < p.cout - ch0 ? ncols : p.cout - ch0) >> 2;  // whole 16-byte pieces
+#pragma unroll
+          for (int r4 = 0; r4 < 8; ++r4) {
+            const int r = 4 * r4 + (lane >> 3), c4 = lane & 7;
+            const int mr = __shfl_sync(0xffffffffu, m, r);
+            if (((rows_ok >> r) & 1u) && c4 < nq) {
+              const int4 val = *reinterpret_cast<const int4*>(stg + r * kStageRow + 4 * c4);
+              *reinterpret_cast<int4*>(ly.y[ti.job] + (int64_t)mr * p.y_row_bytes + (int64_t)(ch0 + 4 * c4) * 4) = val;
+            }
+          }
+          __syncwarp();
+        } else {
+  if (row_ok) {
+            uint8_t* yrow = ly.y[ti.job] + (int64_t)m * p.y_row_bytes;
+            const int ch0 = ti.col0 + g0;
+            if (mode == 1 && magic) {
+              // codes as byte-words: the chained image takes them as they are, the packed
+              // output a couple of shifts per 8 codes
               uint32_t bw[8], gw[8];
-#pragma unroll
-              for (int j = 0; j < 8; ++j)
-                bw[j] = (uint32_t)oo[4 * j] | ((uint32_t)oo[4 * j + 1] << 8) | ((uint32_t)oo[4 * j + 2] << 16) |
-                        ((uint32_t)oo[4 * j + 3] << 24);
+              magic_requant_bytes(v, epf + g0, qmax, kAccSc, bw);
               switch (out_bits) {
                 case 2: pack_bytewords<2>(bw, gw); break;
                 case 3: pack_bytewords<3>(bw, gw); break;
@@ -994,7 +1001,85 @@ conv_tc_kernel(const __grid_constant__ Maps maps, const __grid_constant__ Params
                 default: pack_bytewords<8>(bw, gw); break;
               }
               store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
-              if (kFlat && ly.ws_out) chain_store_bytes(p, ly.ws_out, jb, oimg, oh, ow, ch0, bw);
+              if (kFlat && ly.ws_out) chain_store_bw(p, ly.ws_out, ly.ws_nib, jb, oimg, oh, ow, ch0, bw);
+            } else if (mode == 1) {
+              uint32_t gw[8];
+              {
+                switch (out_bits) {
+                  case 2: fast_requant_group<2>(v, epi, g0, qmax, kAccSc, gw); break;
+                  case 3: fast_requant_group<3>(v, epi, g0, qmax, kAccSc, gw); break;
+                  case 4: fast_requant_group<4>(v, epi, g0, qmax, kAccSc, gw); break;
+                  default: fast_requant_group<8>(v, epi, g0, qmax, kAccSc, gw); break;
+                }
+              }
+              store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
+              if (kFlat && ly.ws_out) chain_store(p, ly.ws_out, ly.ws_nib, jb, oimg, oh, ow, ch0, gw, out_bits);
+            } else if (mode == 2) {
+              int32_t* yr = reinterpret_cast<int32_t*>(yrow) + ch0;
+              const bool whole = ncols == 32 && ch0 + 32 <= p.cout;
+    #pragma unroll
+              for (int q = 0; q < 8; ++q) {
+                int32_t o[4];
+    #pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                  const float f = __uint_as_float(v[4 * q + k]);
+                  o[k] = magic ? __float_as_int(__fmaf_rn(f, kAccSc, kMagic)) + epf[g0 + 4 * q + k].x
+                               : add_sat(__float2int_rn(f * kAccSc), epi[g0 + 4 * q + k].bias);
+                }
+                if (whole) {
+                  reinterpret_cast<int4*>(yr)[q] = make_int4(o[0], o[1], o[2], o[3]);
+                } else {
+    #pragma unroll
+                  for (int k = 0; k < 4; ++k)
+                    if (4 * q + k < ncols && ch0 + 4 * q + k < p.cout) yr[4 * q + k] = o[k];
+                }
+              }
+            } else {
+              const uint8_t* srow = nullptr;
+              if (kSkip && p.has_skip) {
+                int img, ho, wo;
+                if constexpr (kFlat) {
+                  img = oimg; ho = oh; wo = ow;
+                } else {
+                  const int hw = jb.ho * jb.wo;
+                  img = m / hw;
+                  const int rem = m - img * hw;
+                  ho = rem / jb.wo; wo = rem - ho * jb.wo;
+                }
+                const int sh = p.upsample == 2 ? ho >> 1 : ho, sw = p.upsample == 2 ? wo >> 1 : wo;
+                srow = jb.skip + (((int64_t)img * jb.skip_h + sh) * jb.skip_w + sw) * p.skip_row_bytes;
+              }
+              int32_t oo[32];
+              if (kSkip && fast_skip && p.skip_bits <= 8) {
+                load_skip_group(p, srow, ch0, ncols, oo);   // skip codes, replaced by the results
+                fast_skip_group(v, epi + g0, oo, qmax, kAccSc, oo);
+              } else if (kSkip && fast_skip) {
+                load_skip_group(p, srow, ch0, ncols, oo);   // int32 skip, replaced by the results
+                fast_skip32_group(v, epi + g0, oo, qmax, kAccSc, oo);
+              } else {
+                general_group<kSkip, kSplit>(p, v, epi + g0, srow, ch0, ncols, kAccSc, oo);
+              }
+              if (out_bits == 32) {
+                int32_t* yr = reinterpret_cast<int32_t*>(yrow) + ch0;
+  #pragma unroll
+                for (int i = 0; i < 32; ++i)
+                  if (i < ncols && ch0 + i < p.cout) yr[i] = oo[i];
+              } else {
+                // clipped codes (< 2^out_bits) as byte-words, then the packed group
+                uint32_t bw[8], gw[8];
+  #pragma unroll
+                for (int j = 0; j < 8; ++j)
+                  bw[j] = (uint32_t)oo[4 * j] | ((uint32_t)oo[4 * j + 1] << 8) | ((uint32_t)oo[4 * j + 2] << 16) |
+                          ((uint32_t)oo[4 * j + 3] << 24);
+                switch (out_bits) {
+                  case 2: pack_bytewords<2>(bw, gw); break;
+                  case 3: pack_bytewords<3>(bw, gw); break;
+                  case 4: pack_bytewords<4>(bw, gw); break;
+                  default: pack_bytewords<8>(bw, gw); break;
+                }
+                store_group(yrow + (ch0 >> 5) * group_bytes(out_bits), gw, out_bits);
+                if (kFlat && ly.ws_out) chain_store_bw(p, ly.ws_out, ly.ws_nib, jb, oimg, oh, ow, ch0, bw);
+              }
             }
           }
         }
@@ -1200,6 +1285,41 @@ __global__ void __launch_bounds__(256) expand_kernel(const __grid_constant__ Exp
   }
 }
 
+// The zero-padded nibble image of 2-bit codes for the FP4 pipe: the first cin / 2 bytes of
+// workspace row r (rows cin bytes apart, as in the byte image) hold two codes per byte,
+// channel 2k in the low nibble of byte k, of input pixel (img, hp - pad, wp - pad), or zeros
+// in the border (code 0 is the E2M1 value 0). One thread
+// per 16 output bytes, i.e. one 32-channel packed group of 8 input bytes; consecutive threads
+// take consecutive groups of a row.
+__global__ void __launch_bounds__(256) expand_nib_kernel(const __grid_constant__ ExpandArgs a) {
+  grid_dep_wait();
+  if (threadIdx.x == 0) grid_dep_launch();
+  const int groups = a.cin >> 5;
+  const int64_t total = a.total_rows * groups;
+  for (int64_t e = (int64_t)blockIdx.x * 256 + threadIdx.x; e < total; e += (int64_t)gridDim.x * 256) {
+    const int row = (int)(e / groups), g = (int)(e - (int64_t)row * groups);
+    ExpandPos ps;
+    expand_locate(a, row, ps);
+    const ConvJobDev& jb = a.jobs[ps.job];
+    const int hi = ps.hr - a.pad, wi = ps.wc - a.pad;
+    uint32_t o[4] = {0u, 0u, 0u, 0u};
+    if (hi >= 0 && hi < jb.h && wi >= 0 && wi < jb.w) {
+      const uint2 v = __ldg(reinterpret_cast<const uint2*>(jb.x + ((size_t)(ps.img * jb.h + hi) * jb.w + wi) *
+                                                                   a.x_row_bytes) + g);
+#pragma unroll
+      for (int m = 0; m < 4; ++m) {
+        // output word m: channels 8m .. 8m + 7, the byte-words 2(m % 2) and 2(m % 2) + 1 of
+        // packed word m / 2 (byte-word j of a 2-bit word: channels 4j .. 4j + 3, one per byte)
+        const uint32_t wd = (m >> 1) ? v.y : v.x;
+        const int j0 = 2 * (m & 1);
+        const uint32_t b0 = (wd >> (2 * j0)) & 0x03030303u, b1 = (wd >> (2 * j0 + 2)) & 0x03030303u;
+        o[m] = __byte_perm(b0 | (b0 >> 4), b1 | (b1 >> 4), 0x6420);
+      }
+    }
+    *reinterpret_cast<uint4*>(a.ws + (size_t)row * a.cin + (size_t)g * 16) = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
 // ---------------------------------------------------------------- host side
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
@@ -1222,10 +1342,10 @@ static EncodeTiledFn get_encode_fn(std::string* err) {
 }
 
 template <int kXBits, bool kChunkInTap, bool kFlat, bool kPair = false, bool kSkip = true, bool kSplit = false,
-          int kBK = BK>
+          int kBK = BK, bool kFp4 = false, bool kOStage = false>
 static int launch_bits(const Params& prm, const Maps& maps, int grid, size_t smem, cudaStream_t stream,
                        std::string* err) {
-  auto kern = conv_tc_kernel<kXBits, kChunkInTap, kFlat, kPair, kSkip, kSplit, kBK>;
+  auto kern = conv_tc_kernel<kXBits, kChunkInTap, kFlat, kPair, kSkip, kSplit, kBK, kFp4, kOStage>;
   // The opt-in limit is raised to the device maximum, never lowered to this call's size:
   // a CUDA graph node captured earlier with a larger plan must stay launchable (a graph
   // node, or a tool relaunching it, is checked against the function's current limit).
@@ -1263,7 +1383,10 @@ static int launch_bits(const Params& prm, const Maps& maps, int grid, size_t sme
 
 bool conv_tc_uses_pair(const ConvArgs& a) {
   // every N tile width of the workspace path (BN is a multiple of 16, so each CTA's half of
-  // the weight tile is whole 8-row swizzle atoms and M = 256 MMAs take N = BN)
+  // the weight tile is whole 8-row swizzle atoms and M = 256 MMAs take N = BN), except narrow
+  // tiles on the FP4 pipe: the 256->84 output conv of the head measured 35.7 us on single
+  // CTAs against 39.4 us on pairs (same box, expansion included)
+  if (a.fp4 && a.bn <= 128) return false;
   return a.ws != nullptr && a.bn >= 16 && a.bn % 16 == 0 && tc::kSub == 1 && !a.no_pair;
 }
 
@@ -1321,9 +1444,17 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   }
   // K chunk width: 128 bytes of one tap, or on the workspace path with cin % 128 != 0 the 64
   // channels of one tap (cin % 64 == 0; 64-byte swizzled operand rows, two MMAs per chunk)
-  const int bk = (flat && a.cin % BK != 0) ? 64 : BK;
-  if (flat && (kSub != 1 || a.stride != 1 || a.cin % bk != 0 || rows > a.ws_rows || (a.split_w && bk != BK))) {
+  const bool fp4 = a.fp4 != 0;
+  // bytes per row of the image: one code per byte, or two (nibbles) on the FP4 pipe
+  const int img_row = fp4 ? a.cin / 2 : a.cin;
+  const int bk = (flat && img_row % BK != 0) ? 64 : BK;
+  if (flat && (kSub != 1 || a.stride != 1 || img_row % bk != 0 || rows > a.ws_rows || (a.split_w && bk != BK))) {
     *err = "conv_tc: workspace path needs stride 1, cin % 64 == 0 (128 for split weights) and a large enough workspace";
+    return 1;
+  }
+  if (fp4 && !(flat && bk == BK && a.x_bits == 2 && !a.split_w && a.a_planes <= 1 && a.zero_words == 0 && !a.ws_out &&
+               a.nlayers <= 1 && a.w_fp4)) {
+    *err = "conv_tc: the FP4 pipe takes 2-bit codes from a nibble image (cin % 256 == 0), one layer, no chained output";
     return 1;
   }
   if (tiles == 0) return 0;
@@ -1345,7 +1476,7 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   prm.total_tiles = nlayers * (prm.dp_tiles + 2 * (tiles - prm.dp_tiles));
   prm.nlayers = nlayers;
   prm.layer_tiles = prm.total_tiles / nlayers;
-  prm.num_kchunks = flat ? a.k_total / bk : a.k_pad / BK;
+  prm.num_kchunks = flat ? (fp4 ? a.k_total / 2 : a.k_total) / bk : a.k_pad / BK;
   prm.cin = a.cin; prm.cout = a.cout; prm.kh = a.kh; prm.kw = a.kw;
   prm.stride = a.stride; prm.pad = a.pad; prm.k_total = a.k_total;
   prm.out_bits = a.out_bits; prm.skip_bits = a.skip_bits;
@@ -1356,18 +1487,20 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
       ly.m0 = a.layer[l].m0; ly.shift = a.layer[l].shift; ly.bias = a.layer[l].bias;
       for (int j = 0; j < a.njobs; ++j) ly.y[j] = a.layer[l].y[j];
       ly.ws_out = a.layer[l].ws_out;
+      ly.ws_nib = a.layer[l].ws_nib;
     }
   } else {
     LayerDev& ly = prm.layers[0];
     ly.m0 = a.m0; ly.shift = a.shift; ly.bias = a.bias;
     for (int j = 0; j < a.njobs; ++j) ly.y[j] = a.jobs[j].y;
     ly.ws_out = a.ws_out;
+    ly.ws_nib = a.ws_out_nib;
   }
   prm.skip_c = a.skip_c; prm.skip_d = a.skip_d;
   prm.upsample = a.upsample; prm.scale_main = a.scale_main; prm.has_skip = a.has_skip;
   prm.bn = BN;
   prm.acc_small = a.acc_bound < (1LL << 22) ? 1 : 0;
-  prm.cin_chunks = a.cin / bk;
+  prm.cin_chunks = img_row / bk;
   prm.out_pad = a.out_pad;
   prm.a_planes = flat ? (a.a_planes > 1 ? a.a_planes : 1) : 1;
   prm.plane_rows = (int32_t)rows;
@@ -1395,7 +1528,11 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   const size_t bar_bytes = 8 * (2 * kMaxStages + 5) + 16;
   const size_t qtab_bytes = kQTab * sizeof(uint32_t);
   const size_t budget = 232448 - 1024;  // max dynamic smem per block minus alignment slack
-  int stages = (int)((budget - epi_bytes - bar_bytes - qtab_bytes) / stage_bytes);
+  // int32 outputs with cout % 4 == 0: per-warp staging blocks when at least 6 stages remain
+  const size_t ostage_bytes = (size_t)kEpiWarps * 32 * kStageRow * sizeof(uint32_t);
+  const bool ostage = flat && bk == BK && a.out_bits == 32 && a.cout % 4 == 0 && !a.has_skip && !a.split_w &&
+                      (budget - epi_bytes - bar_bytes - qtab_bytes - ostage_bytes) / stage_bytes >= 6;
+  int stages = (int)((budget - epi_bytes - bar_bytes - qtab_bytes - (ostage ? ostage_bytes : 0)) / stage_bytes);
   if (stages > kMaxStages) stages = kMaxStages;
   if (stages < 2) { *err = "conv_tc: shared memory plan does not fit"; return 2; }
   // The TMA issuers take K chunks round-robin and each waits on its stage's "empty"
@@ -1408,21 +1545,28 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   prm.off_epi = prm.off_b + (uint32_t)(stages * b_rows * bk);
   prm.off_bar = prm.off_epi + (uint32_t)epi_bytes;
   prm.off_qtab = prm.off_bar + (uint32_t)bar_bytes;
-  const size_t smem = 1024 + prm.off_qtab + qtab_bytes;
+  prm.off_ostage = ostage ? (uint32_t)((prm.off_qtab + qtab_bytes + 15) / 16 * 16) : 0u;
+  const size_t smem = 1024 + (ostage ? prm.off_ostage + ostage_bytes : prm.off_qtab + qtab_bytes);
+  // two buffers x kSub sub-tiles x BN fp32 columns (and, on the FP4 pipe, 32 columns of scales)
+  const int acc_cols = 2 * kSub * BN;
+  if (fp4 && acc_cols + 32 > 512) { *err = "conv_tc: FP4 tiles wider than 240 channels do not fit in TMEM"; return 2; }
   int cols = 32;
-  while (cols < 2 * kSub * BN) cols *= 2;  // two buffers x kSub sub-tiles x BN fp32 columns
+  while (cols < acc_cols + (fp4 ? 32 : 0)) cols *= 2;
   prm.tmem_cols = cols;
+  prm.sf_col = acc_cols;
 
   EncodeTiledFn enc = get_encode_fn(err);
   if (!enc) return 3;
   Maps maps{};
-  cuuint64_t gdim[2] = {(cuuint64_t)a.k_pad, (cuuint64_t)w_rows};
-  cuuint64_t gstride[1] = {(cuuint64_t)a.k_pad};
+  // weight rows: k_pad E4M3 bytes, or k_pad / 2 bytes of E2M1 nibbles on the FP4 pipe
+  const int w_row = fp4 ? a.k_pad / 2 : a.k_pad;
+  cuuint64_t gdim[2] = {(cuuint64_t)w_row, (cuuint64_t)w_rows};
+  cuuint64_t gstride[1] = {(cuuint64_t)w_row};
   cuuint32_t box[2] = {(cuuint32_t)bk, (cuuint32_t)b_rows};
   cuuint32_t estr[2] = {1, 1};
   const CUtensorMapSwizzle swz = bk == 64 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B;
   for (int l = 0; l < nlayers; ++l) {
-    const uint8_t* wl = nlayers > 1 ? a.layer[l].w_e4m3 : a.w_e4m3;
+    const uint8_t* wl = nlayers > 1 ? a.layer[l].w_e4m3 : (fp4 ? a.w_fp4 : a.w_e4m3);
     const CUresult r = enc(&maps.w[l], CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)wl, gdim, gstride, box, estr,
                            CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -1432,7 +1576,8 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   maps.wh = maps.w[0];
   if (prm.dp_tiles < prm.layer_tiles) {
     cuuint32_t box_h[2] = {(cuuint32_t)bk, (cuuint32_t)(b_rows / 2)};
-    const CUresult r = enc(&maps.wh, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)a.w_e4m3, gdim, gstride, box_h, estr,
+    const CUresult r = enc(&maps.wh, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)(fp4 ? a.w_fp4 : a.w_e4m3), gdim,
+                           gstride, box_h, estr,
                            CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) { *err = "cuTensorMapEncodeTiled (half) failed: " + std::to_string((int)r); return 3; }
@@ -1466,7 +1611,13 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
       cfg.attrs = attr;
       cfg.numAttrs = 1;
       cudaError_t e;
-      switch (a.x_bits) {
+      if (fp4) {
+        // nibble image: one thread per 16 output bytes, grid-strided
+        const int64_t chunks = ea.total_rows * (a.cin / 32);
+        const int64_t want = (chunks + 255) / 256;
+        cfg.gridDim = dim3((unsigned)(want < 4096 ? (want > 0 ? want : 1) : 4096));
+        e = cudaLaunchKernelEx(&cfg, expand_nib_kernel, ea);
+      } else switch (a.x_bits) {
         case 2: e = cudaLaunchKernelEx(&cfg, expand_kernel<2>, ea); break;
         case 3: e = cudaLaunchKernelEx(&cfg, expand_kernel<3>, ea); break;
         case 4: e = cudaLaunchKernelEx(&cfg, expand_kernel<4>, ea); break;
@@ -1479,7 +1630,8 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
     if (a.expand_only) return 0;
     // 2) tensor maps over the workspace (and, for chained layers in one launch, the second
     //    image) as [rows][cin] byte matrices with bk x 128 boxes
-    cuuint64_t gd[2] = {(cuuint64_t)a.cin, (cuuint64_t)rows * (cuuint64_t)prm.a_planes};
+    // (a nibble image keeps the byte image's row stride: cin bytes, the first cin / 2 used)
+    cuuint64_t gd[2] = {(cuuint64_t)img_row, (cuuint64_t)rows * (cuuint64_t)prm.a_planes};
     cuuint64_t gs[1] = {(cuuint64_t)a.cin};
     cuuint32_t bx[2] = {(cuuint32_t)bk, 128};
     for (int i = 0; i < (nlayers > 1 ? 2 : 1); ++i) {
@@ -1490,6 +1642,20 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
         *err = "cuTensorMapEncodeTiled (activations) failed: " + std::to_string((int)r2);
         return 3;
       }
+    }
+    if (ostage) {  // int32 outputs, no skip, 128-byte chunks (see the smem plan)
+      if (fp4)
+        return pair ? launch_bits<2, true, true, true, false, false, 128, true, true>(prm, maps, grid, smem, stream, err)
+                    : launch_bits<2, true, true, false, false, false, 128, true, true>(prm, maps, grid, smem, stream, err);
+      return pair ? launch_bits<2, true, true, true, false, false, 128, false, true>(prm, maps, grid, smem, stream, err)
+                  : launch_bits<2, true, true, false, false, false, 128, false, true>(prm, maps, grid, smem, stream, err);
+    }
+    if (fp4) {
+      if (pair)
+        return a.has_skip ? launch_bits<2, true, true, true, true, false, 128, true>(prm, maps, grid, smem, stream, err)
+                          : launch_bits<2, true, true, true, false, false, 128, true>(prm, maps, grid, smem, stream, err);
+      return a.has_skip ? launch_bits<2, true, true, false, true, false, 128, true>(prm, maps, grid, smem, stream, err)
+                        : launch_bits<2, true, true, false, false, false, 128, true>(prm, maps, grid, smem, stream, err);
     }
     if (a.split_w) {  // (no skip: the API keeps skips off the split form)
       if (pair) return launch_bits<2, true, true, true, false, true>(prm, maps, grid, smem, stream, err);

@@ -423,6 +423,32 @@ prepare_weights_kernel(const uint8_t* wp, int w_bits, int w_format, WeightGeom g
   }
 }
 
+// The E2M1 block of the prepared weights: byte b of row co holds weights k = 2b (low nibble)
+// and 2b + 1 (high nibble) as the E2M1 values w / 2: sign bit 3, magnitude code |w| for
+// |w| <= 4 (0, 0.5, 1, 1.5, 2). Padding rows and columns are 0.
+__global__ void __launch_bounds__(kThreads)
+prepare_fp4_kernel(const uint8_t* wp, int w_bits, int w_format, WeightGeom g, int64_t w_row_bytes, uint8_t* out) {
+  const int64_t row_bytes = g.k_pad / 2;
+  const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  if (t >= (int64_t)g.cout_pad * row_bytes) return;
+  const int64_t co = t / row_bytes, kb = t - co * row_bytes;
+  uint32_t byte = 0;
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int64_t k = 2 * kb + h;
+    int32_t w = 0;
+    if (co < g.cout && k < g.k_total) {
+      const int64_t tap = k / g.cin;
+      const int ch = (int)(k - tap * g.cin);
+      const uint8_t* row = wp + (co * g.kh * g.kw + tap) * w_row_bytes;
+      w = w_format == 0 ? read_code(row, ch, w_bits, true) : 2 * read_code(row, ch, w_bits, false) - ((1 << w_bits) - 1);
+    }
+    const uint32_t nib = (w < 0 ? 8u : 0u) | (uint32_t)(w < 0 ? -w : w);
+    byte |= nib << (4 * h);
+  }
+  out[g.fp4_offset + t] = (uint8_t)byte;
+}
+
 inline unsigned blocks_for(int64_t n) { return (unsigned)((n + kThreads - 1) / kThreads); }
 
 }  // namespace elt
@@ -504,7 +530,14 @@ int launch_prepare_weights(const uint8_t* w_packed, int32_t w_bits, int32_t w_fo
   const int64_t total = e4_rows * g.k_pad + (int64_t)g.cout * g.k_total;
   elt::prepare_weights_kernel<<<elt::blocks_for(total), elt::kThreads, 0, stream>>>(
       w_packed, w_bits, w_format, g, row_bytes_of(g.cin, w_bits), mode, out);
-  return check_launch("prepare_weights launch", err);
+  if (const int st = check_launch("prepare_weights launch", err)) return st;
+  if (fp4_weights(w_bits, w_format)) {
+    const int64_t n4 = (int64_t)g.cout_pad * (g.k_pad / 2);
+    elt::prepare_fp4_kernel<<<elt::blocks_for(n4), elt::kThreads, 0, stream>>>(
+        w_packed, w_bits, w_format, g, row_bytes_of(g.cin, w_bits), out);
+    return check_launch("prepare_weights (fp4) launch", err);
+  }
+  return 0;
 }
 
 }  // namespace aqd

@@ -75,9 +75,15 @@ struct ConvArgs {
     const int32_t* bias;
     uint8_t* y[kMaxJobs];
     uint8_t* ws_out;
+    int32_t ws_nib;
   } layer[kMaxLayers];
   uint8_t* ws2;
   uint32_t* dep;
+  // The FP4 pipe (2-bit codes, |w| <= 4, cin % 256 == 0): the workspace holds a nibble image
+  // (two codes per byte) and the weights come from the E2M1 block w_fp4.
+  int32_t fp4;
+  const uint8_t* w_fp4;
+  int32_t ws_out_nib;     // the chained output image holds two codes per byte (its reader is FP4)
 };
 // Tiles of one layer of a grouped workspace-path launch on CTA pairs with one N tile (the
 // per-layer length of a chained launch's counter array).
@@ -88,8 +94,17 @@ struct WeightGeom {
   int32_t cout, kh, kw, cin;
   int32_t k_total, k_pad, bn, cout_pad;
   int32_t split_rows;     // 2 * round_up(cout, 128): rows of the split (8-bit) weight layout
-  size_t e4m3_bytes, i16_offset, total_bytes;
+  size_t e4m3_bytes, i16_offset;
+  // [cout_pad][k_pad / 2] E2M1 nibbles (weight w as the value w / 2, |w| <= 4; weight k of a
+  // row in the low nibble of byte k / 2 for even k): the FP4 tensor-core B operand
+  size_t fp4_offset, fp4_bytes;
+  size_t total_bytes;
 };
+// Whether weights of this width and format are exact as E2M1 values w / 2 (|w| <= 4).
+inline bool fp4_weights(int32_t w_bits, int32_t w_format) {
+  const int max_abs = w_format == 0 ? (1 << (w_bits - 1)) : ((1 << w_bits) - 1);
+  return max_abs <= 4;
+}
 WeightGeom weight_geom(int32_t cout, int32_t kh, int32_t kw, int32_t cin);
 
 // 0 on success, else an aqd_status value; *err gets a message.

@@ -8,12 +8,21 @@ from paper_2007_06919_gb300 import synth
 
 pytestmark = pytest.mark.gpu
 
-TC, DIRECT, TC_NO_PAIR = 1, 2, 3
+TC, DIRECT, TC_NO_PAIR, TC_NO_FP4, TC_NO_PAIR_NO_FP4 = 1, 2, 3, 4, 5
+FP4 = 6  # reported path of the FP4 tensor-core pipe
 
 
 def ws_path(cout: int) -> int:
     """Path reported for the workspace-fed tensor-core kernel: it runs on CTA pairs (4)."""
     return 4
+
+
+def fp4_applies(xb, wb, fmt, cin, cout):
+    """Whether a workspace-path conv runs on the FP4 pipe: 2-bit codes, weights exact as E2M1
+    w / 2 (|w| <= 4), cin % 256 == 0, at most 240 channels per N tile."""
+    max_w = (1 << (wb - 1)) if fmt == 0 else (1 << wb) - 1
+    bn = (cout + 15) // 16 * 16 if cout <= 256 else 256
+    return xb == 2 and max_w <= 4 and cin % 256 == 0 and bn <= 240
 
 
 def _params(rng, levels, cout, out_bits, calib_std=None):
@@ -93,19 +102,23 @@ WS_CASES = [c for c in CASES if c[9] == 1 and c[6] % 64 == 0 and c[0] <= 4 and c
 
 @pytest.mark.parametrize("case", WS_CASES, ids=[str(i) for i in range(len(WS_CASES))])
 @pytest.mark.parametrize("pairs", [True, False])
-def test_conv_workspace_path_bit_exact(case, pairs):
+@pytest.mark.parametrize("fp4", [True, False])
+def test_conv_workspace_path_bit_exact(case, pairs, fp4):
     """The expanded-activation path (one expansion pass into a caller workspace, then TMA
-    tiles of the zero-padded byte image, junk columns dropped) gives the same bytes, on CTA
-    pairs (256-wide N tiles) and on single CTAs."""
+    tiles of the zero-padded byte or nibble image, junk columns dropped) gives the same
+    bytes, on CTA pairs (256-wide N tiles) and on single CTAs, on the E4M3 pipe and, where
+    it applies, on the FP4 one."""
     xb, wb, fmt, n, h, wd, cin, cout, k, stride, pad, ob = case
     rng = np.random.default_rng(hash(case) % 2 ** 32 + 1)
     x = synth.act_codes(rng, (n, h, wd, cin), xb)
     w = rng.integers(-(1 << (wb - 1)), 1 << (wb - 1), size=(cout, k, k, cin)).astype(np.int32)
     std = np.sqrt(k * k * cin * np.mean(np.arange(1 << xb) ** 2) * (1 << (2 * wb - 2)) / 3)
     m0, sh, b = _params(rng, 1, cout, ob if ob != 32 else 4, calib_std=std)
+    mode = {(True, True): TC, (True, False): TC_NO_FP4, (False, True): TC_NO_PAIR,
+            (False, False): TC_NO_PAIR_NO_FP4}[(pairs, fp4)]
     got, want, used = conv_pair(x, xb, w, wb, stride=stride, pad=pad, out_bits=ob, m0=m0, shift=sh, bias=b,
-                                path=TC if pairs else TC_NO_PAIR, workspace=True)
-    assert used == (ws_path(cout) if pairs else 3)
+                                path=mode, workspace=True)
+    assert used == (FP4 if fp4 and fp4_applies(xb, wb, fmt, cin, cout) else (ws_path(cout) if pairs else 3))
     assert_same(got, want, cout, ob, f"workspace case {case}")
 
 

@@ -160,7 +160,7 @@ def test_cls_and_box_as_one_conv_bit_exact():
     ys = [aqd.DTensor.empty(t.n, t.h, t.w, 84, 32) for t in xts]
     jobs = [(xs[l], ys[l], None, l) for l in range(5)]
     aqd.conv_int_grouped(jobs, W, 1, 1, rq=rq, workspace=aqd.workspace_for(jobs, W, 1, 1))
-    assert aqd.last_conv_path() == 4
+    assert aqd.last_conv_path() == 6  # 2-bit codes, 84 channels: the FP4 pipe
     torch.cuda.synchronize()
     for l in range(5):
         got = ys[l].data.cpu().numpy().view(np.int32).reshape(-1, 84)

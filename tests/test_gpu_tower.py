@@ -80,7 +80,7 @@ def test_full_head_tower_bit_exact(calibrated):
     t = Tower(synth.config2(calibrated=calibrated), 2)
     t.run()
     torch.cuda.synchronize()
-    assert aqd.last_conv_path() == 4
+    assert aqd.last_conv_path() == 6  # the 256->84 output conv on the FP4 pipe, from a nibble image
     assert aqd.device_status() == 0
     t.check(t.reference(), "full head")
 
@@ -88,7 +88,8 @@ def test_full_head_tower_bit_exact(calibrated):
 @pytest.mark.parametrize("bits", [2, 3, 4])
 def test_wide_levels_and_fallbacks_bit_exact(bits):
     """Level widths 300 and 600 (dependency windows of 5 and 7 tiles), a level narrower than a
-    tile, batch 2; then the same with the counters off and with CTA pairs off."""
+    tile, batch 2; then the same with the counters off, with CTA pairs off, and with the FP4
+    pipe off (the output conv then reads a byte image on the E4M3 pipe)."""
     levels = [(7, 300), (5, 600), (9, 20), (1, 3)]
     wl = synth.head_tower(60 + bits, 2, bits, levels=levels, calibrated=True)
     t = Tower(wl, bits, ntower=3)
@@ -97,11 +98,11 @@ def test_wide_levels_and_fallbacks_bit_exact(bits):
     torch.cuda.synchronize()
     assert aqd.device_status() == 0
     t.check(ref, "overlapped")
-    for mode in ("no sync", "no pairs"):
+    for mode in ("no sync", "no pairs", "no fp4"):
         for ys in t.ys:
             for y in ys:
                 y.data.fill_(0xEE)
-        old = aqd.set_conv_path(3 if mode == "no pairs" else 0)
+        old = aqd.set_conv_path({"no pairs": 3, "no fp4": 4}.get(mode, 0))
         try:
             t.run(sync=mode != "no sync")
         finally:

@@ -1635,9 +1635,11 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
     cuuint64_t gs[1] = {(cuuint64_t)a.cin};
     cuuint32_t bx[2] = {(cuuint32_t)bk, 128};
     for (int i = 0; i < (nlayers > 1 ? 2 : 1); ++i) {
+      // (a nibble image row uses 128 of every 256 bytes: fetch 128-byte lines from DRAM)
       const CUresult r2 = enc(&maps.a[i], CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)(i == 0 ? a.ws : a.ws2), gd, gs, bx,
                               estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
-                              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+                              fp4 ? CU_TENSOR_MAP_L2_PROMOTION_L2_128B : CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
       if (r2 != CUDA_SUCCESS) {
         *err = "cuTensorMapEncodeTiled (activations) failed: " + std::to_string((int)r2);
         return 3;

@@ -713,6 +713,8 @@ static aqd_status elementwise(const aqd_tensor* a, const aqd_tensor* b, const aq
   if (rq && (rq->levels <= 0 || level < 0 || level >= rq->levels)) return fail(AQD_ERR_INVALID, "level out of range");
   if (!rq && level != 0) return fail(AQD_ERR_INVALID, "level must be 0 without rq");
   EltArgs e{};
+  e.status = status_ptr(&err);
+  if (!e.status) return fail(AQD_ERR_CUDA, err);
   e.a = static_cast<const uint8_t*>(a->data); e.a_bits = a->bits; e.a_row_bytes = row_bytes_of(a->c, a->bits);
   e.y = static_cast<uint8_t*>(y->data); e.y_bits = y->bits; e.y_row_bytes = row_bytes_of(y->c, y->bits);
   e.n = a->n; e.h = a->h; e.w = a->w; e.c = a->c; e.level = level;

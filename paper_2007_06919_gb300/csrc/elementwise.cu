@@ -4,17 +4,22 @@
 //     skip through a nearest 2x upsample, the FPN top-down add),
 //   * max-pooling directly on codes (Sec. 3.2.4),
 //   * code packing / unpacking and the one-time weight preparation.
-// One thread handles one pixel's 32-channel group, so loads and stores are whole
-// packed groups (8/12/16/32 bytes, or 128 bytes of int32).
+// An int32 input on contiguous rows takes the staged kernel (bulk async copies of whole
+// pixel rows into shared memory, consumer warps with per-lane channel constants); other int32
+// inputs the lane kernel (kV channels per lane, direct loads); packed-code inputs the group
+// kernels (one thread per pixel's 32-channel group: whole packed groups per load and store).
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
 #include "common.cuh"
 #include "kernels.h"
+#include "tc_ptx.cuh"
 
 namespace aqd {
 namespace elt {
 
 constexpr int kThreads = 256;
+constexpr int kLanePix = 6;  // pixels per warp step of the element-wise lane kernel (table form)
 
 __device__ __forceinline__ void load_vals(const uint8_t* row, int bits, int c, int ch0, bool is_signed,
                                           int32_t v[32]) {
@@ -246,6 +251,524 @@ __global__ void __launch_bounds__(kThreads, 3) eltwise_group_kernel(const EltArg
   }
 }
 
+// Requant (Eq. 6 + Eq. 2) and the integer skip add (Eq. 7/8, then Eq. 2) of an int32 tensor
+// with kV consecutive channels per lane (c % (32 kV) == 0): lane l of a warp owns channels
+// 32 kV g + kV l .. + kV - 1 of one block g of 32 kV channels for the whole launch, so their
+// constants stay in registers, and the warp's load of one pixel's block is 128 kV contiguous
+// bytes (one 4 kV-byte load per lane). A packed skip code tensor gives each lane one 32-bit
+// word per pixel (its kV channels lie in one word). The packed output is assembled across
+// lanes: output word w of a 32-channel group holds its channels [w q, (w + 1) q), q = 32 / bits,
+// channel i at bit 8 (i % 4) + bits ((i % q) / 4); a lane's channels land in one word, so an OR
+// over the lanes of a word builds it and one of them stores it. Warps of one block take every
+// warps_per_block-th pixel, kPix per step with their loads issued first.
+//
+// Each block picks one of two exact forms of the epilogue once, from the constants of all c
+// channels:
+//  - table: every rescale has R = 31 + shift >= 33, where rhu(u M0, R) equals
+//    (mulhi(u, M0) + 2^(R-33)) >> (R-32); and, with a skip, the main path is not rescaled
+//    (Eq. 7 with the skip rescaled), the skip codes are at most 8 bits wide and the block's
+//    shared-memory table T[s][ch] = bias + rhu(s c, d) (built in int64 for every code s) fits
+//    int32. Then Eq. 6 + Eq. 7 is sat32(a + T[s][ch]), one saturating 32-bit add; without a
+//    skip it is sat32(a + bias). Table column of channel ch: ch + ch / 32, so the lanes of a
+//    warp, whose channels step by kV, read 32 distinct banks whatever their codes.
+//  - general: Eq. 6 -> Eq. 7 -> Eq. 2 in int64 exactly as defined (the shared epilogue).
+template <int kV>
+struct LaneVec;
+template <> struct LaneVec<1> { typedef int32_t T; };
+template <> struct LaneVec<2> { typedef int2 T; };
+template <> struct LaneVec<4> { typedef int4 T; };
+template <int kV>
+__device__ __forceinline__ void ld_lane(const void* p, int32_t (&v)[kV]) {
+  const typename LaneVec<kV>::T x = __ldg(reinterpret_cast<const typename LaneVec<kV>::T*>(p));
+  if constexpr (kV == 1) { v[0] = x; }
+  else if constexpr (kV == 2) { v[0] = x.x; v[1] = x.y; }
+  else { v[0] = x.x; v[1] = x.y; v[2] = x.z; v[3] = x.w; }
+}
+template <int kV>
+__device__ __forceinline__ void st_lane(void* p, const int32_t (&v)[kV]) {
+  if constexpr (kV == 1) *reinterpret_cast<int32_t*>(p) = v[0];
+  else if constexpr (kV == 2) *reinterpret_cast<int2*>(p) = make_int2(v[0], v[1]);
+  else *reinterpret_cast<int4*>(p) = make_int4(v[0], v[1], v[2], v[3]);
+}
+// sat32(x + y) of two int32 values
+__device__ __forceinline__ int32_t add_sat_s32(int32_t x, int32_t y) {
+  int32_t r;
+  asm("add.sat.s32 %0, %1, %2;" : "=r"(r) : "r"(x), "r"(y));
+  return r;
+}
+
+// Per-lane geometry shared by both forms.
+struct LaneGeo {
+  int64_t first, npix, stride;  // first pixel, pixel count, pixel stride of a step
+  int wpb, ch0, lane;
+  bool same_grid;
+};
+
+template <bool kSkip, int kSkipBits>
+__device__ __forceinline__ int64_t skip_pixel(const EltArgs& a, const LaneGeo& g, int64_t pix) {
+  if (g.same_grid) return pix;
+  const int64_t hw = (int64_t)a.h * a.w;
+  const int64_t img = pix / hw, rem = pix - img * hw;
+  const int hh = (int)(rem / a.w), ww = (int)(rem - (rem / a.w) * a.w);
+  return (img * a.b_h + hh / a.upsample) * a.b_w + ww / a.upsample;
+}
+
+// OR this lane's word contribution with the other lanes of its output word and store it
+template <int kOut, int kV>
+__device__ __forceinline__ void store_codes(const EltArgs& a, const LaneGeo& g, int64_t pix, uint32_t v) {
+  constexpr int q = 32 / kOut;
+  constexpr int span = (q / 4 * 4 + kV - 1) / kV;  // lanes per output word
+#pragma unroll
+  for (int off = 1; off < span; off <<= 1) v |= __shfl_xor_sync(0xffffffffu, v, off);
+  const int i0 = g.ch0 & 31;
+  if (pix < g.npix && g.lane % span == 0)
+    reinterpret_cast<uint32_t*>(a.y + pix * a.y_row_bytes + (g.ch0 >> 5) * group_bytes(kOut))[i0 / q] = v;
+}
+
+// bit position of channel i (of a 32-channel group) in its packed word
+template <int kBits>
+__device__ __forceinline__ int code_pos(int i) {
+  constexpr int q = 32 / kBits;
+  return 8 * (i & 3) + kBits * ((i % q) >> 2);
+}
+
+template <bool kSkip, int kOut, int kSkipBits, int kV>
+__device__ __forceinline__ void lane_fast(const EltArgs& a, const LaneGeo& g, const int32_t (&b)[kV],
+                                          const int32_t (&m0)[kV], const int32_t (&rnd)[kV],
+                                          const int32_t (&sh)[kV], const int32_t* tab, int tstride) {
+  constexpr int kPix = kLanePix;
+  const int i0 = g.ch0 & 31;
+  // channel i0 + k of a packed word sits at bit base + 8 k (kV divides 4 and i0): shift the
+  // word once per pixel instead of once per channel
+  const int sbase = kSkip && kSkipBits <= 8 ? code_pos<kSkip && kSkipBits <= 8 ? kSkipBits : 8>(i0) : 0;
+  const int obase = kOut != 32 ? code_pos<kOut != 32 ? kOut : 8>(i0) : 0;
+  for (int64_t p0 = g.first; p0 < g.npix; p0 += g.stride) {
+    int32_t av[kPix][kV];
+    uint32_t sw[kPix];
+#pragma unroll
+    for (int u = 0; u < kPix; ++u) {
+      const int64_t pix = p0 + (int64_t)u * g.wpb;
+#pragma unroll
+      for (int k = 0; k < kV; ++k) av[u][k] = 0;
+      sw[u] = 0;
+      if (pix >= g.npix) continue;
+      ld_lane<kV>(reinterpret_cast<const int32_t*>(a.a) + pix * a.c + g.ch0, av[u]);
+      if constexpr (kSkip && kSkipBits <= 8) {
+        const uint8_t* srow = a.b + skip_pixel<kSkip, kSkipBits>(a, g, pix) * a.b_row_bytes;
+        sw[u] = __ldg(reinterpret_cast<const uint32_t*>(srow + (g.ch0 >> 5) * group_bytes(kSkipBits)) +
+                      i0 / (32 / kSkipBits)) >> sbase;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kPix; ++u) {
+      const int64_t pix = p0 + (int64_t)u * g.wpb;
+      int32_t y[kV];
+      uint32_t v = 0;
+#pragma unroll
+      for (int k = 0; k < kV; ++k) {
+        int32_t bk = b[k];
+        if constexpr (kSkip && kSkipBits <= 8) {
+          const int s = (int)((sw[u] >> (8 * k)) & ((1u << kSkipBits) - 1u));
+          bk = tab[s * tstride + b[k]];  // b[k]: this channel's table column
+        }
+        const int32_t uu = add_sat_s32(av[u][k], bk);
+        if constexpr (kOut == 32) {
+          y[k] = uu;
+        } else {
+          y[k] = __vimin_s32_relu((__mulhi(uu, m0[k]) + rnd[k]) >> sh[k], (1 << kOut) - 1);
+          v |= (uint32_t)y[k] << (8 * k);
+        }
+      }
+      if constexpr (kOut == 32) {
+        if (pix < g.npix) st_lane<kV>(reinterpret_cast<int32_t*>(a.y + pix * a.y_row_bytes) + g.ch0, y);
+      } else {
+        store_codes<kOut, kV>(a, g, pix, v << obase);
+      }
+    }
+  }
+}
+
+// (not inlined: its int64 arithmetic would otherwise set the register budget of the table form)
+template <bool kSkip, int kOut, int kSkipBits, int kV>
+__device__ __noinline__ void lane_general(const EltArgs& a, const LaneGeo& g, const EpiChan (&ec)[kV]) {
+  constexpr int kPix = 2;
+  const int i0 = g.ch0 & 31;
+  for (int64_t p0 = g.first; p0 < g.npix; p0 += g.stride) {
+    int32_t av[kPix][kV], sv[kPix][kV];
+#pragma unroll
+    for (int u = 0; u < kPix; ++u) {
+      const int64_t pix = p0 + (int64_t)u * g.wpb;
+#pragma unroll
+      for (int k = 0; k < kV; ++k) { av[u][k] = 0; sv[u][k] = 0; }
+      if (pix >= g.npix) continue;
+      ld_lane<kV>(reinterpret_cast<const int32_t*>(a.a) + pix * a.c + g.ch0, av[u]);
+      if constexpr (kSkip) {
+        const uint8_t* srow = a.b + skip_pixel<kSkip, kSkipBits>(a, g, pix) * a.b_row_bytes;
+        if constexpr (kSkipBits == 32) {
+          ld_lane<kV>(reinterpret_cast<const int32_t*>(srow) + g.ch0, sv[u]);
+        } else {
+          const uint32_t w = __ldg(reinterpret_cast<const uint32_t*>(srow + (g.ch0 >> 5) * group_bytes(kSkipBits)) +
+                                   i0 / (32 / kSkipBits));
+#pragma unroll
+          for (int k = 0; k < kV; ++k)
+            sv[u][k] = (int32_t)((w >> code_pos<kSkipBits>(i0 + k)) & ((1u << kSkipBits) - 1u));
+        }
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kPix; ++u) {
+      const int64_t pix = p0 + (int64_t)u * g.wpb;
+      int32_t y[kV];
+      uint32_t v = 0;
+#pragma unroll
+      for (int k = 0; k < kV; ++k) {
+        y[k] = epilogue<kSkip>(av[u][k], sv[u][k], ec[k], a.scale_main, kOut);
+        if constexpr (kOut != 32) v |= (uint32_t)y[k] << code_pos<kOut>(i0 + k);
+      }
+      if constexpr (kOut == 32) {
+        if (pix < g.npix) st_lane<kV>(reinterpret_cast<int32_t*>(a.y + pix * a.y_row_bytes) + g.ch0, y);
+      } else {
+        store_codes<kOut, kV>(a, g, pix, v);
+      }
+    }
+  }
+}
+
+template <bool kSkip, int kOut, int kSkipBits, int kV>
+__global__ void __launch_bounds__(kThreads, 3)
+    eltwise_lane_kernel(const EltArgs a, int64_t npix, int warps_per_block, int tstride) {
+  extern __shared__ int32_t tab[];  // kSkip, tstride > 0: [2^kSkipBits][tstride] bias + rhu(s c, d)
+  LaneGeo g;
+  g.lane = threadIdx.x & 31;
+  const int blocks = a.c / (32 * kV);
+  const int wg = blockIdx.x * (kThreads / 32) + (threadIdx.x >> 5);
+  g.first = wg / blocks;
+  g.ch0 = 32 * kV * (wg % blocks) + kV * g.lane;
+  g.npix = npix;
+  g.wpb = warps_per_block;
+  g.same_grid = a.upsample == 1 && a.b_h == a.h && a.b_w == a.w;
+  const int64_t lv = (int64_t)a.level * a.c;
+  bool ok = true;
+  if constexpr (kOut != 32)
+    for (int ch = threadIdx.x; ch < a.c; ch += kThreads) ok = ok && __ldg(a.shift + lv + ch) >= 2;  // R >= 33
+  if constexpr (kSkip) {
+    if constexpr (kSkipBits <= 8) {
+      if (tstride > 0 && a.scale_main == 0) {
+        // one channel per thread: its constants once, then its 2^kSkipBits entries
+        for (int ch = threadIdx.x; ch < a.c; ch += kThreads) {
+          const int d = __ldg(a.skip_d + lv + ch);
+          const int64_t bias = a.bias ? __ldg(a.bias + lv + ch) : 0, cc = __ldg(a.skip_c + lv + ch);
+          ok = ok && d >= 0 && d <= 62;
+          const int dd = d >= 0 && d <= 62 ? d : 0;
+          for (int sc = 0; sc < (1 << kSkipBits); ++sc) {
+            const int64_t t = bias + rhu(sc * cc, dd);
+            ok = ok && t >= INT32_MIN && t <= INT32_MAX;
+            tab[sc * tstride + ch + (ch >> 5)] = (int32_t)t;
+          }
+        }
+      } else {
+        ok = false;
+      }
+    } else {
+      ok = false;
+    }
+  }
+  ok = __syncthreads_and(ok);
+  EpiChan ec[kV];
+#pragma unroll
+  for (int k = 0; k < kV; ++k) {
+    const int64_t idx = lv + g.ch0 + k;
+    ec[k].bias = a.bias ? __ldg(a.bias + idx) : 0;
+    ec[k].m0 = kOut != 32 ? __ldg(a.m0 + idx) : 0;
+    ec[k].r = kOut != 32 ? (int8_t)(31 + __ldg(a.shift + idx)) : 0;
+    ec[k].c = kSkip ? __ldg(a.skip_c + idx) : 0;
+    ec[k].d = kSkip ? __ldg(a.skip_d + idx) : 0;
+  }
+  if (ok) {
+    g.stride = (int64_t)kLanePix * g.wpb;
+    int32_t b[kV], m0[kV], rnd[kV], sh[kV];
+#pragma unroll
+    for (int k = 0; k < kV; ++k) {
+      const int ch = g.ch0 + k;
+      b[k] = kSkip ? ch + (ch >> 5) : ec[k].bias;
+      m0[k] = ec[k].m0;
+      sh[k] = kOut != 32 ? ec[k].r - 32 : 1;
+      rnd[k] = kOut != 32 ? 1 << (ec[k].r - 33) : 0;
+    }
+    lane_fast<kSkip, kOut, kSkipBits, kV>(a, g, b, m0, rnd, sh, tab, tstride);
+  } else {
+    g.stride = (int64_t)2 * g.wpb;
+    lane_general<kSkip, kOut, kSkipBits, kV>(a, g, ec);
+  }
+}
+
+// The same requant / skip add with its inputs staged through shared memory by the bulk-copy
+// engine: rows of consecutive pixels are contiguous in HBM (the int32 tensor, and the skip
+// tensor on the same grid), so one 1D bulk copy per operand fills a stage of kStagePix... pixels.
+// A producer warp (one thread) keeps `stages` stages in flight per block, so the bytes in
+// flight no longer depend on registers; 8 consumer warps take the filled stages in turn.
+// Warp w owns channel block w % cblocks (kV channels per lane, constants in registers) and
+// every (8 / cblocks)-th pixel of a stage. The epilogue is the table form above (exact when
+// the block's check passes) or, if not, the int64 general form on each pixel's lane group.
+// Every wait is bounded: a wait that runs out sets the status word to a timeout, raises the
+// block's abort flag and leaves; the producer then waits (bounded) for its copies in flight.
+struct StageGeo {
+  int P;                 // pixels per stage
+  int stages;
+  int64_t nchunks;       // ceil(npix / P)
+  uint32_t a_bytes;      // bytes of one stage's int32 rows (P * c * 4)
+  uint32_t s_bytes;      // bytes of one stage's skip rows (P * b_row_bytes, 0 without a skip)
+  uint32_t stage_bytes;  // a_bytes + s_bytes rounded to 128
+  uint32_t tab_bytes;    // skip table bytes rounded to 128
+};
+
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar,
+                                         uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;"
+      ::"r"(dst), "l"(src), "r"(bytes), "r"(bar), "l"(policy) : "memory");
+}
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+// one pixel of one lane group in the int64 general form (rare: constants the table cannot hold)
+template <bool kSkip, int kOut, int kSkipBits, int kV>
+__device__ __noinline__ void staged_general(const EltArgs& a, const int32_t* arow, const uint8_t* srow,
+                                            int ch0, int lane, int64_t pix) {
+  const int64_t lv = (int64_t)a.level * a.c;
+  const int i0 = ch0 & 31;
+  uint32_t v = 0;
+  int32_t y[kV];
+#pragma unroll
+  for (int k = 0; k < kV; ++k) {
+    EpiChan ec;
+    const int64_t idx = lv + ch0 + k;
+    ec.bias = a.bias ? __ldg(a.bias + idx) : 0;
+    ec.m0 = kOut != 32 ? __ldg(a.m0 + idx) : 0;
+    ec.r = kOut != 32 ? (int8_t)(31 + __ldg(a.shift + idx)) : 0;
+    ec.c = kSkip ? __ldg(a.skip_c + idx) : 0;
+    ec.d = kSkip ? __ldg(a.skip_d + idx) : 0;
+    int32_t sv = 0;
+    if constexpr (kSkip) {
+      const int i = i0 + k;
+      const uint32_t w = reinterpret_cast<const uint32_t*>(srow + (ch0 >> 5) * group_bytes(kSkipBits))[i / (32 / kSkipBits)];
+      sv = (int32_t)((w >> code_pos<kSkipBits>(i)) & ((1u << kSkipBits) - 1u));
+    }
+    y[k] = epilogue<kSkip>(arow[ch0 + k], sv, ec, a.scale_main, kOut);
+    if constexpr (kOut != 32) v |= (uint32_t)y[k] << code_pos<kOut>(i0 + k);
+  }
+  if constexpr (kOut == 32) {
+    st_lane<kV>(reinterpret_cast<int32_t*>(a.y + pix * a.y_row_bytes) + ch0, y);
+  } else {
+    constexpr int q = 32 / kOut;
+    constexpr int span = (q / 4 * 4 + kV - 1) / kV;
+#pragma unroll
+    for (int off = 1; off < span; off <<= 1) v |= __shfl_xor_sync(0xffffffffu, v, off);
+    if (lane % span == 0)
+      reinterpret_cast<uint32_t*>(a.y + pix * a.y_row_bytes + (ch0 >> 5) * group_bytes(kOut))[i0 / q] = v;
+  }
+}
+
+template <bool kSkip, int kOut, int kSkipBits, int kV>
+__global__ void __launch_bounds__(kThreads + 32, kSkip ? 2 : 3)  // the skip form: its table limits it to 2
+    eltwise_staged_kernel(const EltArgs a, int64_t npix, const StageGeo sg, int tstride) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  __shared__ uint64_t bars[2 * 8];  // full[s], empty[s], s < 8
+  __shared__ int abort_flag;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  int32_t* tab = reinterpret_cast<int32_t*>(smem);
+  uint8_t* stage0 = smem + sg.tab_bytes;
+  const uint32_t full0 = tc::smem_u32(&bars[0]), empty0 = tc::smem_u32(&bars[8]);
+  if (tid == 0) {
+    abort_flag = 0;
+    for (int s = 0; s < sg.stages; ++s) {
+      tc::mbar_init(full0 + 8 * s, 1);
+      tc::mbar_init(empty0 + 8 * s, kThreads / 32);
+    }
+    tc::fence_barrier_init();
+  }
+  // the block's form (table fits / every R >= 33) and its skip table, as in the lane kernel
+  const int64_t lv = (int64_t)a.level * a.c;
+  bool ok = true, small = true;  // small: every table entry within [-2^30, 2^30]
+  if (tid < kThreads) {
+    if constexpr (kOut != 32)
+      for (int ch = tid; ch < a.c; ch += kThreads) ok = ok && __ldg(a.shift + lv + ch) >= 2;
+    if constexpr (kSkip) {
+      if (tstride > 0 && a.scale_main == 0) {
+        for (int ch = tid; ch < a.c; ch += kThreads) {
+          const int d = __ldg(a.skip_d + lv + ch);
+          const int64_t bias = a.bias ? __ldg(a.bias + lv + ch) : 0, cc = __ldg(a.skip_c + lv + ch);
+          ok = ok && d >= 0 && d <= 62;
+          const int dd = d >= 0 && d <= 62 ? d : 0;
+          for (int sc = 0; sc < (1 << kSkipBits); ++sc) {
+            const int64_t t = bias + rhu(sc * cc, dd);
+            ok = ok && t >= INT32_MIN && t <= INT32_MAX;
+            small = small && t >= -(1LL << 30) && t <= (1LL << 30);
+            tab[sc * tstride + ch + (ch >> 5)] = (int32_t)t;
+          }
+        }
+      } else {
+        ok = false;
+      }
+    }
+  }
+  ok = __syncthreads_and(ok);
+  small = __syncthreads_and(small);
+
+  if (warp == kThreads / 32) {
+    // producer: thread 0 of the last warp issues the stage copies
+    if (lane != 0) return;
+    const uint64_t pol = policy_evict_first();
+    int it = 0;
+    bool live = true;
+    for (int64_t j = blockIdx.x; j < sg.nchunks && live; j += gridDim.x, ++it) {
+      const int s = it % sg.stages;
+      if (it >= sg.stages && !tc::mbar_wait(empty0 + 8 * s, ((it / sg.stages) - 1) & 1, &abort_flag)) {
+        tc::fail(&abort_flag, a.status);
+        live = false;
+        break;
+      }
+      const int64_t p0 = j * sg.P;
+      const int np = (int)(npix - p0 < sg.P ? npix - p0 : sg.P);
+      const uint32_t ab = (uint32_t)np * (uint32_t)a.c * 4u;
+      const uint32_t sb = kSkip ? (uint32_t)np * (uint32_t)a.b_row_bytes : 0u;
+      const uint32_t dst = tc::smem_u32(stage0 + (size_t)s * sg.stage_bytes);
+      tc::mbar_arrive_expect_tx(full0 + 8 * s, ab + sb);
+      bulk_g2s(dst, a.a + p0 * a.c * 4, ab, full0 + 8 * s, pol);
+      if constexpr (kSkip) bulk_g2s(dst + sg.a_bytes, a.b + p0 * a.b_row_bytes, sb, full0 + 8 * s, pol);
+    }
+    // before leaving, the copies still in flight (the last `stages` chunks) land: bounded
+    const int issued = it;
+    for (int k = issued - sg.stages > 0 ? issued - sg.stages : 0; k < issued; ++k) {
+      const int s = k % sg.stages;
+      if (!tc::mbar_wait(full0 + 8 * s, (k / sg.stages) & 1, &abort_flag)) break;
+    }
+    return;
+  }
+
+  // consumers
+  const int cblocks = a.c / (32 * kV);
+  const int cb = warp % cblocks, pg = warp / cblocks, pgs = (kThreads / 32) / cblocks;
+  const int ch0 = 32 * kV * cb + kV * lane;
+  const int i0 = ch0 & 31;
+  // b: the bias (no skip) or the channel's table column (skip)
+  int32_t b[kV], m0[kV], rnd[kV], sh[kV];
+#pragma unroll
+  for (int k = 0; k < kV; ++k) {
+    const int ch = ch0 + k;
+    const int64_t idx = lv + ch;
+    const int r = kOut != 32 ? 31 + __ldg(a.shift + idx) : 33;
+    b[k] = kSkip ? ch + (ch >> 5) : (a.bias ? __ldg(a.bias + idx) : 0);
+    m0[k] = kOut != 32 ? __ldg(a.m0 + idx) : 0;
+    sh[k] = r - 32;
+    rnd[k] = r >= 33 ? 1 << (r - 33) : 0;
+  }
+  const int sbase = kSkip ? code_pos<kSkip ? kSkipBits : 8>(i0) : 0;
+  const int obase = kOut != 32 ? code_pos<kOut != 32 ? kOut : 8>(i0) : 0;
+  int it = 0;
+  for (int64_t j = blockIdx.x; j < sg.nchunks; j += gridDim.x, ++it) {
+    const int s = it % sg.stages;
+    if (!tc::mbar_wait(full0 + 8 * s, (it / sg.stages) & 1, &abort_flag)) {
+      tc::fail(&abort_flag, a.status);
+      return;
+    }
+    const int64_t p0 = j * sg.P;
+    const int np = (int)(npix - p0 < sg.P ? npix - p0 : sg.P);
+    const uint8_t* st = stage0 + (size_t)s * sg.stage_bytes;
+    if (!ok) {
+      for (int p = pg; p < np; p += pgs)
+        staged_general<kSkip, kOut, kSkipBits, kV>(a, reinterpret_cast<const int32_t*>(st) + (size_t)p * a.c,
+                                                   st + sg.a_bytes + (size_t)p * a.b_row_bytes, ch0, lane, p0 + p);
+    } else {
+      // two pixels per step (the second clamped to the last one and its store predicated off)
+      // so their chains interleave
+      for (int p = pg; p < np; p += 2 * pgs) {
+        const int pp[2] = {p, p + pgs < np ? p + pgs : np - 1};
+        int32_t av[2][kV];
+        uint32_t sw[2] = {0, 0};
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const int32_t* arow = reinterpret_cast<const int32_t*>(st) + pp[u] * a.c;
+          if constexpr (kV == 4) {
+            const int4 x = *reinterpret_cast<const int4*>(arow + ch0);
+            av[u][0] = x.x; av[u][1] = x.y; av[u][2] = x.z; av[u][3] = x.w;
+          } else if constexpr (kV == 2) {
+            const int2 x = *reinterpret_cast<const int2*>(arow + ch0);
+            av[u][0] = x.x; av[u][1] = x.y;
+          } else {
+            av[u][0] = arow[ch0];
+          }
+          if constexpr (kSkip)
+            sw[u] = reinterpret_cast<const uint32_t*>(st + sg.a_bytes + pp[u] * (int)a.b_row_bytes +
+                                                      (ch0 >> 5) * group_bytes(kSkipBits))[i0 / (32 / kSkipBits)] >> sbase;
+        }
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const bool live = u == 0 || p + pgs < np;
+          uint8_t* yrow = a.y + (p0 + pp[u]) * a.y_row_bytes;
+          int32_t y[kV];
+          uint32_t v = 0;
+          int32_t us[kV];
+          if constexpr (kSkip) {
+            // codes: masked once, then byte k of the word is channel k's code
+            const uint32_t swm = sw[u] & (((1u << kSkipBits) - 1u) * 0x01010101u);
+            int32_t t[kV];
+            int32_t f = 0;  // sign bit set iff some a is outside [-2^30, 2^30)
+#pragma unroll
+            for (int k = 0; k < kV; ++k) {
+              const uint32_t code = k == 0 ? (swm & 0xffu) : (k == 3 ? swm >> 24 : __byte_perm(swm, 0u, 0x4440u + k));
+              t[k] = tab[(int)code * tstride + b[k]];
+              f |= av[u][k] + (1 << 30);
+            }
+            if (small && f >= 0) {
+              // |a| <= 2^30 and |t| <= 2^30: the sum cannot leave int32
+#pragma unroll
+              for (int k = 0; k < kV; ++k) us[k] = av[u][k] + t[k];
+            } else {
+              // sat32(a + t): the wrapped sum, replaced by the bound of a's sign where a and t
+              // have one sign and the sum the other
+#pragma unroll
+              for (int k = 0; k < kV; ++k) {
+                const int32_t w = (int32_t)((uint32_t)av[u][k] + (uint32_t)t[k]);
+                us[k] = ((w ^ av[u][k]) & (w ^ t[k])) < 0 ? (av[u][k] >> 31) ^ INT32_MAX : w;
+              }
+            }
+          } else {
+#pragma unroll
+            for (int k = 0; k < kV; ++k) us[k] = add_sat_s32(av[u][k], b[k]);
+          }
+#pragma unroll
+          for (int k = 0; k < kV; ++k) {
+            const int32_t uu = us[k];
+            if constexpr (kOut == 32) {
+              y[k] = uu;
+            } else {
+              y[k] = __vimin_s32_relu((__mulhi(uu, m0[k]) + rnd[k]) >> sh[k], (1 << kOut) - 1);
+              v += (uint32_t)y[k] << (8 * k);
+            }
+          }
+          if constexpr (kOut == 32) {
+            if (live) st_lane<kV>(reinterpret_cast<int32_t*>(yrow) + ch0, y);
+          } else {
+            constexpr int q = 32 / kOut;
+            constexpr int span = (q / 4 * 4 + kV - 1) / kV;
+            v <<= obase;
+#pragma unroll
+            for (int off = 1; off < span; off <<= 1) v |= __shfl_xor_sync(0xffffffffu, v, off);
+            if (live && lane % span == 0)
+              reinterpret_cast<uint32_t*>(yrow + (ch0 >> 5) * group_bytes(kOut))[i0 / q] = v;
+          }
+        }
+      }
+    }
+    __syncwarp();
+    if (lane == 0) tc::mbar_arrive(empty0 + 8 * s);
+  }
+}
+
 __global__ void __launch_bounds__(kThreads) maxpool_kernel(const PoolArgs a) {
   const int groups = (a.c + 31) / 32;
   const int64_t total = (int64_t)a.n * a.ho * a.wo * groups;
@@ -276,15 +799,27 @@ __global__ void __launch_bounds__(kThreads) maxpool_kernel(const PoolArgs a) {
 }
 
 // Max-pool on packed codes of 2, 4 or 8 bits (Sec. 3.2.4: max-pooling commutes with the
-// monotone quantizer, so it runs on the codes). In these layouts every byte holds 8/bits
-// codes at bit offsets 0, bits, 2 bits, ..., each of a different channel, so the per-channel
-// maximum is a byte-wise maximum (__vmaxu4) of each bit plane. One thread owns kVec words of
-// one output pixel's row; window taps outside the input are skipped (codes are >= 0 and the
-// padding is smaller than the window, so every window holds a tap).
-template <int kBits, int kVec>
+// monotone quantizer, so it runs on the codes). Codes sit in aligned kBits-bit fields of each
+// 32-bit word, so the word's bits (w >> s) & M, M = (2^kBits - 1) * 0x00010001, for
+// s = 0, kBits, ..., 16 - kBits, are 16 / kBits "planes" of two codes each, one at the bottom
+// of each 16-bit half. OR-ed with 0x3C00 per half, a plane is a pair of normal half-precision
+// numbers 1 + code / 2^10, which order like the codes, so one native packed-half maximum
+// (__hmax2) takes the maximum of two channels per plane. One thread owns kVec words of one
+// output pixel's row. A window tap outside the input is replaced by the nearest row / column
+// inside it: the padding is smaller than the window, so that tap lies in the same window, and
+// a maximum taken twice is the same maximum. With kK = 3 (the network's 3x3 pools) the 9 taps
+// are unrolled and their loads issued together; kK = 0 loops over a.k.
+template <int kBits>
+__device__ __forceinline__ __half2 code_plane(uint32_t w, int s) {
+  constexpr uint32_t kM = ((1u << kBits) - 1u) * 0x00010001u;
+  const uint32_t x = ((w >> s) & kM) | 0x3C003C00u;
+  return *reinterpret_cast<const __half2*>(&x);
+}
+
+template <int kBits, int kVec, int kK>
 __global__ void __launch_bounds__(kThreads) maxpool_packed_kernel(const PoolArgs a) {
-  constexpr int kPlanes = 8 / kBits;
-  constexpr uint32_t kMask = kBits == 8 ? 0xFFFFFFFFu : (kBits == 4 ? 0x0F0F0F0Fu : 0x03030303u);
+  constexpr int kPlanes = 16 / kBits;
+  constexpr uint32_t kM = ((1u << kBits) - 1u) * 0x00010001u;
   const int64_t units = a.row_bytes / (4 * kVec);
   const int64_t total = (int64_t)a.n * a.ho * a.wo * units;
   const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
@@ -295,17 +830,21 @@ __global__ void __launch_bounds__(kThreads) maxpool_packed_kernel(const PoolArgs
   const int img = (int)(pix / hw);
   const int rem = (int)(pix - (int64_t)img * hw);
   const int oh = rem / a.wo, ow = rem - oh * a.wo;
-  uint32_t acc[kVec][kPlanes];
+  __half2 acc[kVec][kPlanes];
+  {
+    const uint32_t one = 0x3C003C00u;  // code 0 in both halves: codes are >= 0
 #pragma unroll
-  for (int v = 0; v < kVec; ++v)
+    for (int v = 0; v < kVec; ++v)
 #pragma unroll
-    for (int j = 0; j < kPlanes; ++j) acc[v][j] = 0u;
-  for (int r = 0; r < a.k; ++r) {
-    const int hi = oh * a.stride - a.pad + r;
-    if (hi < 0 || hi >= a.h) continue;
-    for (int s = 0; s < a.k; ++s) {
-      const int wi = ow * a.stride - a.pad + s;
-      if (wi < 0 || wi >= a.w) continue;
+      for (int j = 0; j < kPlanes; ++j) acc[v][j] = *reinterpret_cast<const __half2*>(&one);
+  }
+  const int k = kK > 0 ? kK : a.k;
+#pragma unroll
+  for (int r = 0; r < (kK > 0 ? kK : k); ++r) {
+    const int hi = min(max(oh * a.stride - a.pad + r, 0), a.h - 1);
+#pragma unroll
+    for (int s = 0; s < (kK > 0 ? kK : k); ++s) {
+      const int wi = min(max(ow * a.stride - a.pad + s, 0), a.w - 1);
       const uint32_t* src = reinterpret_cast<const uint32_t*>(
           a.x + (((int64_t)img * a.h + hi) * a.w + wi) * a.row_bytes) + u * kVec;
       uint32_t w[kVec];
@@ -319,7 +858,7 @@ __global__ void __launch_bounds__(kThreads) maxpool_packed_kernel(const PoolArgs
 #pragma unroll
       for (int v = 0; v < kVec; ++v)
 #pragma unroll
-        for (int j = 0; j < kPlanes; ++j) acc[v][j] = __vmaxu4(acc[v][j], (w[v] >> (kBits * j)) & kMask);
+        for (int j = 0; j < kPlanes; ++j) acc[v][j] = __hmax2(acc[v][j], code_plane<kBits>(w[v], kBits * j));
     }
   }
   uint32_t o[kVec];
@@ -327,7 +866,7 @@ __global__ void __launch_bounds__(kThreads) maxpool_packed_kernel(const PoolArgs
   for (int v = 0; v < kVec; ++v) {
     o[v] = 0u;
 #pragma unroll
-    for (int j = 0; j < kPlanes; ++j) o[v] |= acc[v][j] << (kBits * j);
+    for (int j = 0; j < kPlanes; ++j) o[v] |= (*reinterpret_cast<const uint32_t*>(&acc[v][j]) & kM) << (kBits * j);
   }
   uint32_t* dst = reinterpret_cast<uint32_t*>(a.y + pix * a.row_bytes) + u * kVec;
   if constexpr (kVec == 4) {
@@ -459,9 +998,141 @@ static int check_launch(const char* what, std::string* err) {
   return 0;
 }
 
+// kV channels per lane: int32 input, c % (32 kV) == 0, 2/4/8/32-bit output, 2/4/8/32-bit skip.
+// One wave of blocks (the resident count per SM for this kernel and table size, times the SMs),
+// each building its table once; the warp count a multiple of the channel-block count (warps of
+// one channel block take every warps_per_block-th pixel).
+template <bool kSkip, int kOut, int kSkipBits, int kV>
+static void launch_lane_k(const EltArgs& a, int ts, int sms, cudaStream_t stream) {
+  auto kern = elt::eltwise_lane_kernel<kSkip, kOut, kSkipBits, kV>;
+  const size_t smem = ts > 0 ? ((size_t)ts << kSkipBits) * sizeof(int32_t) : 0;
+  int occ = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, elt::kThreads, smem) != cudaSuccess || occ < 1) occ = 1;
+  const int cblocks = a.c / (32 * kV);
+  const int64_t npix = (int64_t)a.n * a.h * a.w;
+  int g = cblocks, w = elt::kThreads / 32;  // blocks must be a multiple of cblocks / gcd(cblocks, 8)
+  while (w) { const int t = g % w; g = w; w = t; }
+  const int64_t unit = cblocks / g;
+  int64_t blocks = (int64_t)sms * occ;
+  const int64_t need = (npix * cblocks + 7) / 8;  // one pixel per warp at most
+  if (blocks > need) blocks = need;
+  blocks = blocks / unit * unit;
+  if (blocks < unit) blocks = unit;
+  const int wpb = (int)(blocks * (elt::kThreads / 32) / cblocks);
+  kern<<<(unsigned)blocks, elt::kThreads, smem, stream>>>(a, npix, wpb, ts);
+}
+template <bool kSkip, int kSkipBits, int kV>
+static bool launch_lane_v(const EltArgs& a, int ts, int sms, cudaStream_t stream) {
+  switch (a.y_bits) {
+    case 2: launch_lane_k<kSkip, 2, kSkipBits, kV>(a, ts, sms, stream); return true;
+    case 4: launch_lane_k<kSkip, 4, kSkipBits, kV>(a, ts, sms, stream); return true;
+    case 8: launch_lane_k<kSkip, 8, kSkipBits, kV>(a, ts, sms, stream); return true;
+    case 32: launch_lane_k<kSkip, 32, kSkipBits, kV>(a, ts, sms, stream); return true;
+    default: return false;
+  }
+}
+template <bool kSkip, int kSkipBits>
+static bool launch_lane(const EltArgs& a, int sms, cudaStream_t stream) {
+  // the skip table's row stride: c columns plus one per 32 channels, rounded to 32 banks; none
+  // when the main path is rescaled, the skip is int32 or the table would pass 48 KB
+  int ts = 0;
+  if (kSkip && kSkipBits <= 8 && a.scale_main == 0) {
+    ts = (a.c + a.c / 32 + 31) / 32 * 32;
+    if (((size_t)ts << kSkipBits) * sizeof(int32_t) > 48 * 1024) ts = 0;
+  }
+  const int v = a.c % 128 == 0 ? 4 : (a.c % 64 == 0 ? 2 : 1);  // channels per lane
+  if (v == 4) return launch_lane_v<kSkip, kSkipBits, 4>(a, ts, sms, stream);
+  if (v == 2) return launch_lane_v<kSkip, kSkipBits, 2>(a, ts, sms, stream);
+  return launch_lane_v<kSkip, kSkipBits, 1>(a, ts, sms, stream);
+}
+
+// The staged kernel: one wave of blocks, 2 stages of about 32 KB of int32 rows each.
+template <bool kSkip, int kOut, int kSkipBits, int kV>
+static void launch_staged_k(const EltArgs& a, int ts, int sms, cudaStream_t stream) {
+  auto kern = elt::eltwise_staged_kernel<kSkip, kOut, kSkipBits, kV>;
+  const int64_t npix = (int64_t)a.n * a.h * a.w;
+  const int row = a.c * 4;
+  elt::StageGeo g{};
+  g.P = 32768 / row > 0 ? 32768 / row : 1;  // measured: fewer, larger stages beat more, smaller ones
+  g.stages = 2;
+  g.nchunks = (npix + g.P - 1) / g.P;
+  g.a_bytes = (uint32_t)g.P * (uint32_t)row;
+  g.s_bytes = kSkip ? (uint32_t)g.P * (uint32_t)a.b_row_bytes : 0u;
+  g.stage_bytes = (g.a_bytes + g.s_bytes + 127u) / 128u * 128u;
+  g.tab_bytes = ts > 0 ? (uint32_t)((((size_t)ts << kSkipBits) * sizeof(int32_t) + 127) / 128 * 128) : 0u;
+  const size_t smem = g.tab_bytes + (size_t)g.stages * g.stage_bytes;
+  cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  int occ = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, elt::kThreads + 32, smem) != cudaSuccess || occ < 1)
+    occ = 1;
+  int64_t blocks = (int64_t)sms * occ;
+  if (blocks > g.nchunks) blocks = g.nchunks;
+  kern<<<(unsigned)blocks, elt::kThreads + 32, smem, stream>>>(a, npix, g, ts);
+}
+template <bool kSkip, int kSkipBits, int kV>
+static bool launch_staged_v(const EltArgs& a, int ts, int sms, cudaStream_t stream) {
+  switch (a.y_bits) {
+    case 2: launch_staged_k<kSkip, 2, kSkipBits, kV>(a, ts, sms, stream); return true;
+    case 4: launch_staged_k<kSkip, 4, kSkipBits, kV>(a, ts, sms, stream); return true;
+    case 8: launch_staged_k<kSkip, 8, kSkipBits, kV>(a, ts, sms, stream); return true;
+    case 32: launch_staged_k<kSkip, 32, kSkipBits, kV>(a, ts, sms, stream); return true;
+    default: return false;
+  }
+}
+// Whether the staged kernel takes these arguments: contiguous int32 rows (and skip rows on the
+// same grid, 2/4/8-bit, whole 16-byte rows) at 16-byte aligned addresses, and a channel-block
+// count that divides the 8 consumer warps.
+static bool staged_applies(const EltArgs& a) {
+  if (a.a_bits != 32 || a.c % 32 != 0 || a.a_row_bytes != (int64_t)a.c * 4 || a.y_bits == 3) return false;
+  if ((uintptr_t)a.a % 16 != 0) return false;
+  const int v = a.c % 128 == 0 ? 4 : (a.c % 64 == 0 ? 2 : 1);
+  const int cblocks = a.c / (32 * v);
+  if (cblocks != 1 && cblocks != 2 && cblocks != 4 && cblocks != 8) return false;
+  if (a.has_skip) {
+    if (a.b_bits != 2 && a.b_bits != 4 && a.b_bits != 8) return false;
+    if (!(a.upsample == 1 && a.b_h == a.h && a.b_w == a.w)) return false;
+    if (a.b_row_bytes % 16 != 0 || (uintptr_t)a.b % 16 != 0) return false;
+  }
+  return true;
+}
+template <bool kSkip, int kSkipBits>
+static bool launch_staged(const EltArgs& a, int sms, cudaStream_t stream) {
+  int ts = 0;
+  if (kSkip && a.scale_main == 0) {
+    ts = (a.c + a.c / 32 + 31) / 32 * 32;
+    if (((size_t)ts << kSkipBits) * sizeof(int32_t) > 48 * 1024) ts = 0;
+  }
+  const int v = a.c % 128 == 0 ? 4 : (a.c % 64 == 0 ? 2 : 1);
+  if (v == 4) return launch_staged_v<kSkip, kSkipBits, 4>(a, ts, sms, stream);
+  if (v == 2) return launch_staged_v<kSkip, kSkipBits, 2>(a, ts, sms, stream);
+  return launch_staged_v<kSkip, kSkipBits, 1>(a, ts, sms, stream);
+}
+
 int launch_elementwise(const EltArgs& a, cudaStream_t stream, std::string* err) {
   const int64_t total = (int64_t)a.n * a.h * a.w * ((a.c + 31) / 32);
   if (total == 0) return 0;
+  const bool lane_ok = a.a_bits == 32 && a.c % 32 == 0 && a.y_bits != 3 &&
+                       (!a.has_skip || a.b_bits == 2 || a.b_bits == 4 || a.b_bits == 8 || a.b_bits == 32);
+  if (lane_ok) {
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (sms <= 0) sms = 152;
+    bool ok = false;
+    if (staged_applies(a)) {
+      if (!a.has_skip) ok = launch_staged<false, 0>(a, sms, stream);
+      else if (a.b_bits == 2) ok = launch_staged<true, 2>(a, sms, stream);
+      else if (a.b_bits == 4) ok = launch_staged<true, 4>(a, sms, stream);
+      else ok = launch_staged<true, 8>(a, sms, stream);
+      if (ok) return check_launch("eltwise launch", err);
+    }
+    if (!a.has_skip) ok = launch_lane<false, 0>(a, sms, stream);
+    else if (a.b_bits == 2) ok = launch_lane<true, 2>(a, sms, stream);
+    else if (a.b_bits == 4) ok = launch_lane<true, 4>(a, sms, stream);
+    else if (a.b_bits == 8) ok = launch_lane<true, 8>(a, sms, stream);
+    else ok = launch_lane<true, 32>(a, sms, stream);
+    if (ok) return check_launch("eltwise launch", err);
+  }
   if (a.c <= elt::kTabChannels && a.c % 32 == 0) {
     // enough blocks for every SM several times over; each block stages the constants once
     int dev = 0, sms = 0;
@@ -487,15 +1158,26 @@ int launch_maxpool(const PoolArgs& a, cudaStream_t stream, std::string* err) {
     const bool v4 = a.row_bytes % 16 == 0;
     const int64_t total = pixels * (a.row_bytes / (v4 ? 16 : 4));
     const int blocks = elt::blocks_for(total);
-    if (a.bits == 2) {
-      if (v4) elt::maxpool_packed_kernel<2, 4><<<blocks, elt::kThreads, 0, stream>>>(a);
-      else elt::maxpool_packed_kernel<2, 1><<<blocks, elt::kThreads, 0, stream>>>(a);
+    if (a.k == 3) {
+      if (a.bits == 2) {
+        if (v4) elt::maxpool_packed_kernel<2, 4, 3><<<blocks, elt::kThreads, 0, stream>>>(a);
+        else elt::maxpool_packed_kernel<2, 1, 3><<<blocks, elt::kThreads, 0, stream>>>(a);
+      } else if (a.bits == 4) {
+        if (v4) elt::maxpool_packed_kernel<4, 4, 3><<<blocks, elt::kThreads, 0, stream>>>(a);
+        else elt::maxpool_packed_kernel<4, 1, 3><<<blocks, elt::kThreads, 0, stream>>>(a);
+      } else {
+        if (v4) elt::maxpool_packed_kernel<8, 4, 3><<<blocks, elt::kThreads, 0, stream>>>(a);
+        else elt::maxpool_packed_kernel<8, 1, 3><<<blocks, elt::kThreads, 0, stream>>>(a);
+      }
+    } else if (a.bits == 2) {
+      if (v4) elt::maxpool_packed_kernel<2, 4, 0><<<blocks, elt::kThreads, 0, stream>>>(a);
+      else elt::maxpool_packed_kernel<2, 1, 0><<<blocks, elt::kThreads, 0, stream>>>(a);
     } else if (a.bits == 4) {
-      if (v4) elt::maxpool_packed_kernel<4, 4><<<blocks, elt::kThreads, 0, stream>>>(a);
-      else elt::maxpool_packed_kernel<4, 1><<<blocks, elt::kThreads, 0, stream>>>(a);
+      if (v4) elt::maxpool_packed_kernel<4, 4, 0><<<blocks, elt::kThreads, 0, stream>>>(a);
+      else elt::maxpool_packed_kernel<4, 1, 0><<<blocks, elt::kThreads, 0, stream>>>(a);
     } else {
-      if (v4) elt::maxpool_packed_kernel<8, 4><<<blocks, elt::kThreads, 0, stream>>>(a);
-      else elt::maxpool_packed_kernel<8, 1><<<blocks, elt::kThreads, 0, stream>>>(a);
+      if (v4) elt::maxpool_packed_kernel<8, 4, 0><<<blocks, elt::kThreads, 0, stream>>>(a);
+      else elt::maxpool_packed_kernel<8, 1, 0><<<blocks, elt::kThreads, 0, stream>>>(a);
     }
     return check_launch("maxpool launch", err);
   }

@@ -141,6 +141,7 @@ struct EltArgs {
   const int32_t* skip_c;
   const int8_t* skip_d;
   int32_t upsample, scale_main, has_skip, level;
+  uint32_t* status;       // device status word (bounded waits of the staged kernel)
 };
 int launch_elementwise(const EltArgs& a, cudaStream_t stream, std::string* err);
 

@@ -122,6 +122,51 @@ def test_residual_add_int32_spans(with_rq, mirror):
     assert_same(Y.data.cpu().numpy().reshape(ref.packed.shape), ref.packed, c, out_bits, "residual spans")
 
 
+@pytest.mark.parametrize("c,b_bits,out_bits,wide", [(256, 2, 2, True), (256, 4, 4, True), (256, 8, 32, True),
+                                                     (128, 4, 8, False), (128, 4, 8, True), (64, 4, 2, False),
+                                                     (96, 8, 4, True), (32, 2, 2, False)])
+def test_residual_add_int32_lane_forms(c, b_bits, out_bits, wide):
+    """The int32 skip add's two exact forms side by side: channels 0 .. c/2 - 1 take skip
+    constants at the edge of the 32-bit form (s c + 2^(d-1) at the widest code s equal to
+    2^31 - 1, and a bias whose sum with rhu(s c, d) reaches +-(2^31 - 1) exactly), the other
+    half one channel with a skip multiplier too wide for it (its warp runs the int64 form);
+    accumulators at the int32 extremes saturate Eq. 6's sum. 4, 2 and 1 channels per lane."""
+    rng = np.random.default_rng(c * 7 + b_bits + out_bits)
+    n, h, w = 2, 19, 23
+    a = rng.integers(-(1 << 31), 1 << 31, size=(n, h, w, c), dtype=np.int64).astype(np.int32)
+    a[0, 0, :3, :] = np.array([2 ** 31 - 1, -2 ** 31, 0], dtype=np.int64)[:, None].astype(np.int32)
+    b = synth.act_codes(rng, (n, h, w, c), b_bits)
+    b[0, 0, :2, :] = (1 << b_bits) - 1
+    smax = (1 << b_bits) - 1
+    dd = rng.integers(0, 12, size=(1, c)).astype(np.int8)
+    half = np.where(dd > 0, 1 << np.maximum(dd.astype(np.int64) - 1, 0), 0)
+    cc = np.zeros((1, c), dtype=np.int64)
+    bias = rng.integers(-(1 << 20), 1 << 20, size=(1, c)).astype(np.int64)
+    for j in range(c // 2):
+        if j % 2 == 0:   # s c + half = 2^31 - 1 at s = smax, bias + rhu = 2^31 - 1
+            cc[0, j] = (2 ** 31 - 1 - half[0, j]) // smax
+            bias[0, j] = 2 ** 31 - 1 - ((smax * cc[0, j] + half[0, j]) >> int(dd[0, j]))
+        else:            # s c + half >= -2^31, bias + rhu = -2^31
+            cc[0, j] = -((2 ** 31 + half[0, j]) // smax)
+            bias[0, j] = -2 ** 31 - ((smax * cc[0, j] + half[0, j]) >> int(dd[0, j]))
+    cc[0, c // 2:] = rng.integers(-(1 << 12), 1 << 12, size=c - c // 2)
+    if wide:
+        cc[0, c - 1] = 2 ** 31 - 1   # too wide for the 32-bit form: this channel's warp takes int64
+    cc, bias = cc.astype(np.int32), bias.astype(np.int32)
+    m0 = rng.integers(1 << 30, 1 << 31, size=(1, c), dtype=np.int64).astype(np.int32)
+    sh = rng.integers(20, 28, size=(1, c)).astype(np.int8)
+    kw = dict(m0=m0, shift=sh, bias=bias) if out_bits != 32 else dict(bias=bias)
+    at, bt = oracle.CodeTensor.from_codes(a, 32), oracle.CodeTensor.from_codes(b, b_bits)
+    ref = oracle.residual_add(at, bt, cc, dd, upsample=1, scale_a=0, out_bits=out_bits, **kw)
+    Y = aqd.DTensor.empty(n, h, w, c, out_bits)
+    Y.data.fill_(0xA5)
+    rq = aqd.RequantParams.from_numpy(m0, sh, bias) if out_bits != 32 else aqd.RequantParams.from_numpy(None, None, bias)
+    aqd.residual_add_int(to_device(at), to_device(bt), aqd.SkipParams.from_numpy(cc, dd), Y, rq=rq)
+    torch.cuda.synchronize()
+    assert aqd.device_status() == 0
+    assert_same(Y.data.cpu().numpy().reshape(ref.packed.shape), ref.packed, c, out_bits, "residual lane forms")
+
+
 @pytest.mark.parametrize("c,a_bits,b_bits,out_bits", [(160, 4, 32, 2), (96, 8, 2, 32), (256, 3, 4, 4)])
 def test_residual_add_packed_main_operand(c, a_bits, b_bits, out_bits):
     """The skip add with packed codes as the main operand (their bytes staged through shared

@@ -218,6 +218,43 @@ def int8_library_peak(timeout_s: float = 120.0) -> dict:
         return {"tops": None, "unavailable": type(e).__name__}
 
 
+def detector_rate(dev, stream, flush, replays: int = 8) -> dict:
+    """The whole integer detector (integer ResNet-18 + FPN P3-P7 + shared RetinaNet head,
+    4-bit codes, 8-bit RGB input) at batch 8, 800x1344, as one captured graph of its forward
+    pass: median device time of `replays` replays, L2 flushed before each."""
+    import torch
+    from paper_2007_06919_gb300 import aqd, synth
+    from paper_2007_06919_gb300.detector import IntDetector
+    wl = synth.config3()
+    nb, (hh, ww) = wl.extra["batch"], wl.extra["hw"]
+    with torch.cuda.stream(stream):
+        net = IntDetector(wl.extra["layers"], (nb, hh, ww, 3, 8), device=dev)
+        net.tensors["image"].data.copy_(aqd.DTensor.from_codes(torch.from_numpy(wl.inputs[0]).to(dev), 8).data)
+        for _ in range(3):
+            net.forward(stream=stream)
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        net.forward(stream=stream)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(replays)]
+    with torch.cuda.stream(stream):
+        for a, b in ev:
+            flush.fill_(1)
+            a.record(stream)
+            g.replay()
+            b.record(stream)
+    stream.synchronize()
+    assert aqd.device_status(stream) == 0
+    ms = statistics.median(a.elapsed_time(b) for a, b in ev)
+    out = {"value": nb / (ms * 1e-3), "unit": "images/s", "ms_per_batch": ms, "batch": nb,
+           "input": f"{hh}x{ww} 8-bit RGB codes (seeded synthetic)", "tops": net.ops / (ms * 1e-3) / 1e12,
+           "launches_per_batch": net.launches, "replays": replays, "l2": "flushed before every replay",
+           "network": "integer ResNet-18 + FPN P3-P7 + shared RetinaNet head, 4-bit codes, random-init weights"}
+    del g, net
+    torch.cuda.empty_cache()
+    return out
+
+
 def max_over_ranks(x: float, device) -> float:
     """The largest x over all ranks (the job's time is its slowest replica's)."""
     import torch
@@ -489,6 +526,15 @@ def run_sweep(args):
         nb = n * (h * w + 200 * 336) * aqd.row_bytes(c, 4)
         emit("eltwise_maxpool3x3s2_4bit_8x400x672x64", ms, 0, nb, frac_hbm=nb / (ms * 1e-3) / 1e9 / hbm,
              hbm_peak_gbs=hbm)
+        # the same pool fused into the expansion pass of a 3x3 64->64 conv over its output (what
+        # the detector runs): reads the 4-bit input, writes the pooled codes and the byte image
+        Wp = aqd.ConvWeights(torch.from_numpy(rng.integers(-2, 2, size=(64, 3, 3, c)).astype(np.int32)).to(dev), 2)
+        pj = [(P4, aqd.DTensor.empty(n, 200, 336, 64, 4, device=dev), None, 0)]
+        wsp = torch.empty(aqd.conv_workspace_bytes(pj, Wp, 1, 1), dtype=torch.uint8, device=dev)
+        ms = timed(lambda: aqd.maxpool_expand(X4, 3, 2, 1, P4, Wp, 1, 1, wsp, stream=stream))
+        nb = n * h * w * aqd.row_bytes(c, 4) + n * 200 * 336 * aqd.row_bytes(c, 4) + wsp.numel()
+        emit("eltwise_maxpool3x3s2_expand_4bit_8x400x672x64", ms, 0, nb, frac_hbm=nb / (ms * 1e-3) / 1e9 / hbm,
+             hbm_peak_gbs=hbm, bytes_note="input + pooled codes + the conv's zero-padded byte image")
 
     # config 4: first tower layer of the head at batch 16, 2/3/4/8-bit
     for bits in ((2, 3, 4, 8) if want in ("all", "config4") else ()):
@@ -527,6 +573,8 @@ def main():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-detector", action="store_true",
+                    help="skip the whole-detector images/s measurement (batch 8, 800x1344)")
     ap.add_argument("--sweep", nargs="?", const="all", default=None, choices=["all", "config0", "config1", "config3", "config4", "eltwise"],
                     help="measure the other workloads (several lines)")
     args = ap.parse_args()
@@ -760,6 +808,8 @@ def main():
         line["cpu_baseline"] = {"value": ops_c / t_c / 1e12, "unit": "TOPS", "cores": omp_threads(),
                                 "kind": "oracle", "sample": "one full step (4 tower layers + cls + box, all "
                                 f"5 levels, batch 2): {ops_c / 1e9:.1f} GOP in {t_c:.1f} s"}
+    if rank == 0 and world == 1 and not args.no_detector:
+        line["detector_images_per_s"] = detector_rate(dev, stream, flush)
     if rank == 0 and world == 1:
         # A library comparison, not a tensor peak: the INT8 GEMM that torch ships
         # (torch._int_mm) measured here, beside the tower conv's rate. sm_103a's tcgen05 has

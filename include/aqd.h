@@ -330,6 +330,21 @@ aqd_status aqd_residual_add_int(const aqd_tensor* a, const aqd_tensor* b,
 aqd_status aqd_maxpool_codes(const aqd_tensor* x, int32_t k, int32_t stride, int32_t pad,
                              aqd_tensor* y, aqd_stream_t stream);
 
+/* Sec. 3.2.4's max-pool fused with the first step of the workspace path of the convolution
+ * that reads its output (the stem's 3x3 stride-2 pool feeding the first residual stage):
+ * y = aqd_maxpool_codes(x, k, stride, pad) is written as packed codes (for any other reader,
+ * e.g. a skip), and in the same pass `workspace` receives the zero-padded byte image that
+ * aqd_conv_expand_input would write for the single job {x = y} of weights w with conv_stride
+ * and conv_pad. A following aqd_conv_int_grouped_expanded of that job then reads it, so the
+ * pooled map is never read back for its expansion and no separate pooling launch runs.
+ * The pool must be 3x3 with stride 2 on 2- or 4-bit codes (else AQD_ERR_UNSUPPORTED);
+ * x and y: same n, c and bits, y the pooled shape, distinct storage. The workspace path must apply to that convolution and the workspace
+ * hold aqd_conv_workspace_bytes of it: otherwise AQD_ERR_UNSUPPORTED (AQD_ERR_INVALID for a
+ * NULL workspace or bad shapes). Results are the bytes the two separate calls produce. */
+aqd_status aqd_maxpool_expand(const aqd_tensor* x, int32_t k, int32_t stride, int32_t pad, aqd_tensor* y,
+                              const aqd_conv_weights* w, int32_t conv_stride, int32_t conv_pad,
+                              void* workspace, size_t ws_bytes, aqd_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -57,7 +57,7 @@ EXPORTS = ["aqd_row_bytes", "aqd_quantize_multiplier", "aqd_status_string", "aqd
            "aqd_unpack_codes", "aqd_conv_weights_bytes", "aqd_conv_prepare_weights", "aqd_conv_int",
            "aqd_conv_int_grouped", "aqd_conv_workspace_bytes", "aqd_conv_expand_input",
            "aqd_conv_int_grouped_expanded", "aqd_conv_int_grouped_chain", "aqd_requant", "aqd_residual_add_int",
-           "aqd_maxpool_codes", "aqd_conv_int_static_workspace", "aqd_selftest_wait_timeout",
+           "aqd_maxpool_codes", "aqd_maxpool_expand", "aqd_conv_int_static_workspace", "aqd_selftest_wait_timeout",
            "aqd_conv_tower_sync_bytes", "aqd_conv_int_grouped_tower"]
 
 _lib = None
@@ -123,10 +123,12 @@ def load(build_if_missing: bool = True):
     L.aqd_residual_add_int.argtypes = [ctypes.POINTER(_Tensor), ctypes.POINTER(_Tensor), ctypes.POINTER(_Skip),
                                        ctypes.POINTER(_Requant), i32, ctypes.POINTER(_Tensor), vp]
     L.aqd_maxpool_codes.argtypes = [ctypes.POINTER(_Tensor), i32, i32, i32, ctypes.POINTER(_Tensor), vp]
+    L.aqd_maxpool_expand.argtypes = [ctypes.POINTER(_Tensor), i32, i32, i32, ctypes.POINTER(_Tensor),
+                                     ctypes.POINTER(_Weights), i32, i32, vp, ctypes.c_size_t, vp]
     for name in ("aqd_quantize_multiplier", "aqd_device_status", "aqd_pack_codes", "aqd_unpack_codes",
                  "aqd_conv_prepare_weights", "aqd_conv_int", "aqd_conv_int_grouped", "aqd_conv_expand_input",
                  "aqd_conv_int_grouped_expanded", "aqd_conv_int_grouped_chain", "aqd_requant",
-                 "aqd_residual_add_int", "aqd_maxpool_codes"):
+                 "aqd_residual_add_int", "aqd_maxpool_codes", "aqd_maxpool_expand"):
         getattr(L, name).restype = c_int
     _lib = L
     return L
@@ -464,6 +466,17 @@ def maxpool_codes(x: DTensor, k: int, stride: int, pad: int, y: DTensor, stream=
     xc, yc = x.ct(), y.ct()
     _check(load().aqd_maxpool_codes(ctypes.byref(xc), k, stride, pad, ctypes.byref(yc), _stream(stream)),
            "aqd_maxpool_codes")
+    return y
+
+
+def maxpool_expand(x: DTensor, k: int, stride: int, pad: int, y: DTensor, w: ConvWeights, conv_stride: int,
+                   conv_pad: int, workspace: torch.Tensor, stream=None) -> DTensor:
+    """maxpool_codes(x) -> y fused with conv_expand_input([(y, ...)], w, conv_stride, conv_pad,
+    workspace): one pass writes y and the byte image of y for that convolution."""
+    xc, yc = x.ct(), y.ct()
+    wsp, wsb = _ws(workspace)
+    _check(load().aqd_maxpool_expand(ctypes.byref(xc), k, stride, pad, ctypes.byref(yc), ctypes.byref(w.desc),
+                                     conv_stride, conv_pad, wsp, wsb, _stream(stream)), "aqd_maxpool_expand")
     return y
 
 

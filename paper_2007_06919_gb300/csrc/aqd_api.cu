@@ -767,6 +767,47 @@ aqd_status aqd_maxpool_codes(const aqd_tensor* x, int32_t k, int32_t stride, int
   return st ? fail((aqd_status)st, err) : AQD_OK;
 }
 
+aqd_status aqd_maxpool_expand(const aqd_tensor* x, int32_t k, int32_t stride, int32_t pad, aqd_tensor* y,
+                              const aqd_conv_weights* w, int32_t conv_stride, int32_t conv_pad, void* workspace,
+                              size_t ws_bytes, aqd_stream_t stream) {
+  std::string err;
+  if (!check_tensor(x, false, "x", &err)) return fail(AQD_ERR_INVALID, err);
+  if (!check_tensor(y, false, "y", &err)) return fail(AQD_ERR_INVALID, err);
+  if (k <= 0 || stride <= 0 || pad < 0 || pad >= k) return fail(AQD_ERR_INVALID, "need k > 0, stride > 0, 0 <= pad < k");
+  if (x->h + 2 * pad < k || x->w + 2 * pad < k) return fail(AQD_ERR_INVALID, "window larger than the padded input");
+  const int ho = (x->h + 2 * pad - k) / stride + 1, wo = (x->w + 2 * pad - k) / stride + 1;
+  if (y->n != x->n || y->h != ho || y->w != wo || y->c != x->c || y->bits != x->bits)
+    return fail(AQD_ERR_INVALID, "y shape does not match the pooled output");
+  if (x->data == y->data) return fail(AQD_ERR_INVALID, "x and y must not share storage");
+  if (!workspace) return fail(AQD_ERR_INVALID, "the workspace must not be NULL");
+  if ((x->bits != 2 && x->bits != 4) || k != 3 || stride != 2)
+    return fail(AQD_ERR_UNSUPPORTED, "the fused max-pool takes a 3x3 stride-2 pool on 2- or 4-bit codes");
+  // the expansion of the job {x = y} for the convolution (only its input matters)
+  aqd_conv_job job{};
+  job.x = *y;
+  job.y.n = y->n;
+  job.y.h = w && conv_stride > 0 && conv_pad >= 0 ? (y->h + 2 * conv_pad - w->kh) / conv_stride + 1 : 0;
+  job.y.w = w && conv_stride > 0 && conv_pad >= 0 ? (y->w + 2 * conv_pad - w->kw) / conv_stride + 1 : 0;
+  job.y.c = w ? w->cout : 0;
+  job.y.bits = 32;
+  job.y.data = workspace;  // any non-null aligned pointer; never dereferenced
+  // validates the convolution and its workspace (the image geometry: one job, rows of cin bytes
+  // from the workspace start, padding conv_pad)
+  ConvPlan plan;
+  const aqd_status s = plan_grouped(&job, 1, w, conv_stride, conv_pad, nullptr, nullptr, workspace, ws_bytes,
+                                    kStageExpandOnly, nullptr, true, &plan);
+  if (s != AQD_OK) return s;
+  if (plan.path != 1 || plan.a.a_planes != 1 || plan.a.fp4 || plan.a.cin != y->c || plan.a.jobs[0].row_off != 0)
+    return fail(AQD_ERR_UNSUPPORTED, "the convolution does not read a one-plane byte image");
+  PoolArgs p{};
+  p.x = static_cast<const uint8_t*>(x->data); p.y = static_cast<uint8_t*>(y->data);
+  p.n = x->n; p.h = x->h; p.w = x->w; p.c = x->c; p.bits = x->bits; p.ho = ho; p.wo = wo;
+  p.k = k; p.stride = stride; p.pad = pad; p.row_bytes = row_bytes_of(x->c, x->bits);
+  const int st = launch_maxpool_expand(p, static_cast<uint8_t*>(workspace), conv_pad,
+                                       static_cast<cudaStream_t>(stream), &err);
+  return st ? fail((aqd_status)st, err) : AQD_OK;
+}
+
 }  // extern "C"
 
 // ---------------------------------------------------------------- static workspace

@@ -49,6 +49,55 @@ __device__ __forceinline__ int32_t epilogue(int64_t acc, int64_t skip, const Epi
   return (int32_t)(v < 0 ? 0 : (v > hi ? hi : v));
 }
 
+// ---------------------------------------------------------------- maxima of packed codes
+
+// Max-pooling on codes (Sec. 3.2.4). Codes of 2, 4 or 8 bits sit in aligned kBits-bit fields of
+// each 32-bit word, so w & (M << kBits j), M = (2^kBits - 1) * 0x00010001, j < 16 / kBits, are
+// 16 / kBits planes of two codes each, one per 16-bit half, in place: as unsigned 16-bit
+// numbers they order like the codes, so a packed 16-bit maximum (three inputs at a time) is
+// the maximum of two channels, and the maxima of all planes OR back into one word. The top
+// plane needs no mask before the maximum: unsigned 16-bit halves order first by their top
+// field, so the maximum of the raw halves carries the maximum top code (masked once at the
+// end). PoolAcc holds the planes of one word.
+template <int kBits>
+struct PoolAcc {
+  static constexpr int kPlanes = 16 / kBits;
+  static constexpr uint32_t kM = ((1u << kBits) - 1u) * 0x00010001u;
+  static constexpr uint32_t kTop = kM << (kBits * (kPlanes - 1));
+  uint32_t p[kPlanes];
+  static __device__ __forceinline__ uint32_t plane(uint32_t w, int j) {
+    return j == kPlanes - 1 ? w : w & (kM << (kBits * j));
+  }
+  __device__ __forceinline__ void init() {
+#pragma unroll
+    for (int j = 0; j < kPlanes; ++j) p[j] = 0u;  // codes are >= 0
+  }
+  __device__ __forceinline__ void add(uint32_t w) {
+#pragma unroll
+    for (int j = 0; j < kPlanes; ++j) p[j] = __vimax3_u16x2(p[j], plane(w, j), 0u);
+  }
+  __device__ __forceinline__ void add2(uint32_t w0, uint32_t w1) {
+#pragma unroll
+    for (int j = 0; j < kPlanes; ++j) p[j] = __vimax3_u16x2(p[j], plane(w0, j), plane(w1, j));
+  }
+  // the maximum of three words' planes (replaces the contents)
+  __device__ __forceinline__ void set3(uint32_t w0, uint32_t w1, uint32_t w2) {
+#pragma unroll
+    for (int j = 0; j < kPlanes; ++j) p[j] = __vimax3_u16x2(plane(w0, j), plane(w1, j), plane(w2, j));
+  }
+  // this = max(this, a, b), plane by plane
+  __device__ __forceinline__ void max3(const PoolAcc& a, const PoolAcc& b) {
+#pragma unroll
+    for (int j = 0; j < kPlanes; ++j) p[j] = __vimax3_u16x2(p[j], a.p[j], b.p[j]);
+  }
+  __device__ __forceinline__ uint32_t word() const {
+    uint32_t o = p[kPlanes - 1] & kTop;
+#pragma unroll
+    for (int j = 0; j < kPlanes - 1; ++j) o |= p[j];
+    return o;
+  }
+};
+
 // ---------------------------------------------------------------- packed layout
 // A group = 32 consecutive channels of one pixel row: 4*bits bytes for bits 2/3/4/8.
 // bits 2/4/8: word w holds channels [w*q, (w+1)*q), q = 32/bits, channel i of the word

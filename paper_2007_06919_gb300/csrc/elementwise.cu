@@ -8,7 +8,6 @@
 // pixel rows into shared memory, consumer warps with per-lane channel constants); other int32
 // inputs the lane kernel (kV channels per lane, direct loads); packed-code inputs the group
 // kernels (one thread per pixel's 32-channel group: whole packed groups per load and store).
-#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
 #include "common.cuh"
@@ -799,81 +798,204 @@ __global__ void __launch_bounds__(kThreads) maxpool_kernel(const PoolArgs a) {
 }
 
 // Max-pool on packed codes of 2, 4 or 8 bits (Sec. 3.2.4: max-pooling commutes with the
-// monotone quantizer, so it runs on the codes). Codes sit in aligned kBits-bit fields of each
-// 32-bit word, so the word's bits (w >> s) & M, M = (2^kBits - 1) * 0x00010001, for
-// s = 0, kBits, ..., 16 - kBits, are 16 / kBits "planes" of two codes each, one at the bottom
-// of each 16-bit half. OR-ed with 0x3C00 per half, a plane is a pair of normal half-precision
-// numbers 1 + code / 2^10, which order like the codes, so one native packed-half maximum
-// (__hmax2) takes the maximum of two channels per plane. One thread owns kVec words of one
-// output pixel's row. A window tap outside the input is replaced by the nearest row / column
-// inside it: the padding is smaller than the window, so that tap lies in the same window, and
-// a maximum taken twice is the same maximum. With kK = 3 (the network's 3x3 pools) the 9 taps
-// are unrolled and their loads issued together; kK = 0 loops over a.k.
-template <int kBits>
-__device__ __forceinline__ __half2 code_plane(uint32_t w, int s) {
-  constexpr uint32_t kM = ((1u << kBits) - 1u) * 0x00010001u;
-  const uint32_t x = ((w >> s) & kM) | 0x3C003C00u;
-  return *reinterpret_cast<const __half2*>(&x);
-}
-
+// monotone quantizer, so it runs on the codes), word by word with PoolAcc's packed 16-bit
+// maxima. One thread owns kVec words of one output pixel's row. A window tap outside the input
+// is replaced by the nearest row / column inside it: the padding is smaller than the window,
+// so that tap lies in the same window, and a maximum taken twice is the same maximum. With
+// kK = 3 (the network's 3x3 pools) the 9 taps are unrolled and their loads issued together;
+// kK = 0 loops over a.k.
+// Grid: z = image, y = output row, x = the row's (output pixel, unit) pairs, unit fastest
+// (ushift = log2 of the units per pixel when that is a power of two, else -1).
 template <int kBits, int kVec, int kK>
-__global__ void __launch_bounds__(kThreads) maxpool_packed_kernel(const PoolArgs a) {
-  constexpr int kPlanes = 16 / kBits;
-  constexpr uint32_t kM = ((1u << kBits) - 1u) * 0x00010001u;
-  const int64_t units = a.row_bytes / (4 * kVec);
-  const int64_t total = (int64_t)a.n * a.ho * a.wo * units;
-  const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
-  if (t >= total) return;
-  const int64_t pix = t / units;
-  const int u = (int)(t - pix * units);
-  const int hw = a.ho * a.wo;
-  const int img = (int)(pix / hw);
-  const int rem = (int)(pix - (int64_t)img * hw);
-  const int oh = rem / a.wo, ow = rem - oh * a.wo;
-  __half2 acc[kVec][kPlanes];
-  {
-    const uint32_t one = 0x3C003C00u;  // code 0 in both halves: codes are >= 0
+__global__ void __launch_bounds__(kThreads) maxpool_packed_kernel(const PoolArgs a, int ushift) {
+  const int units = (int)(a.row_bytes / (4 * kVec));
+  const int x = blockIdx.x * kThreads + threadIdx.x;
+  const int ow = ushift >= 0 ? x >> ushift : x / units;
+  const int u = x - ow * units;
+  if (ow >= a.wo) return;
+  const int oh = blockIdx.y, img = blockIdx.z;
+  const int64_t pix = ((int64_t)img * a.ho + oh) * a.wo + ow;
+  PoolAcc<kBits> acc[kVec];
 #pragma unroll
-    for (int v = 0; v < kVec; ++v)
-#pragma unroll
-      for (int j = 0; j < kPlanes; ++j) acc[v][j] = *reinterpret_cast<const __half2*>(&one);
-  }
+  for (int v = 0; v < kVec; ++v) acc[v].init();
   const int k = kK > 0 ? kK : a.k;
-#pragma unroll
-  for (int r = 0; r < (kK > 0 ? kK : k); ++r) {
+  // the window's taps in row-major order, two per maximum (an odd last one alone)
+  auto tap = [&](int t, uint32_t (&w)[kVec]) {
+    const int r = t / k, s = t - r * k;
     const int hi = min(max(oh * a.stride - a.pad + r, 0), a.h - 1);
+    const int wi = min(max(ow * a.stride - a.pad + s, 0), a.w - 1);
+    const uint32_t* src = reinterpret_cast<const uint32_t*>(
+        a.x + (((int64_t)img * a.h + hi) * a.w + wi) * a.row_bytes) + u * kVec;
+    if constexpr (kVec == 4) {
+      const uint4 q = __ldg(reinterpret_cast<const uint4*>(src));
+      w[0] = q.x; w[1] = q.y; w[2] = q.z; w[3] = q.w;
+    } else {
 #pragma unroll
-    for (int s = 0; s < (kK > 0 ? kK : k); ++s) {
-      const int wi = min(max(ow * a.stride - a.pad + s, 0), a.w - 1);
-      const uint32_t* src = reinterpret_cast<const uint32_t*>(
-          a.x + (((int64_t)img * a.h + hi) * a.w + wi) * a.row_bytes) + u * kVec;
-      uint32_t w[kVec];
-      if constexpr (kVec == 4) {
-        const uint4 q = __ldg(reinterpret_cast<const uint4*>(src));
-        w[0] = q.x; w[1] = q.y; w[2] = q.z; w[3] = q.w;
-      } else {
-#pragma unroll
-        for (int v = 0; v < kVec; ++v) w[v] = __ldg(src + v);
-      }
-#pragma unroll
-      for (int v = 0; v < kVec; ++v)
-#pragma unroll
-        for (int j = 0; j < kPlanes; ++j) acc[v][j] = __hmax2(acc[v][j], code_plane<kBits>(w[v], kBits * j));
+      for (int v = 0; v < kVec; ++v) w[v] = __ldg(src + v);
     }
+  };
+  const int taps = k * k;
+#pragma unroll
+  for (int t = 0; t + 1 < (kK > 0 ? kK * kK : taps); t += 2) {
+    uint32_t w0[kVec], w1[kVec];
+    tap(t, w0);
+    tap(t + 1, w1);
+#pragma unroll
+    for (int v = 0; v < kVec; ++v) acc[v].add2(w0[v], w1[v]);
+  }
+  if (taps & 1) {
+    uint32_t w0[kVec];
+    tap(taps - 1, w0);
+#pragma unroll
+    for (int v = 0; v < kVec; ++v) acc[v].add(w0[v]);
   }
   uint32_t o[kVec];
 #pragma unroll
-  for (int v = 0; v < kVec; ++v) {
-    o[v] = 0u;
-#pragma unroll
-    for (int j = 0; j < kPlanes; ++j) o[v] |= (*reinterpret_cast<const uint32_t*>(&acc[v][j]) & kM) << (kBits * j);
-  }
+  for (int v = 0; v < kVec; ++v) o[v] = acc[v].word();
   uint32_t* dst = reinterpret_cast<uint32_t*>(a.y + pix * a.row_bytes) + u * kVec;
   if constexpr (kVec == 4) {
     *reinterpret_cast<uint4*>(dst) = make_uint4(o[0], o[1], o[2], o[3]);
   } else {
 #pragma unroll
     for (int v = 0; v < kVec; ++v) dst[v] = o[v];
+  }
+}
+
+// The 3x3 stride-2 max-pool (the stem's) on packed codes, two horizontally adjacent outputs
+// per thread: their windows share the middle column, so 5 columns x 3 rows of taps serve both.
+// Per column the three rows' maximum first (one three-input maximum per plane), then each
+// output's three columns. Taps outside the input are clamped inside, as above. Thread x of
+// grid row (img, oh) takes output pair x >> ushift (x / units when the units per pixel are not
+// a power of two), unit x - pair * units; false past the row's end.
+template <int kBits, int kVec>
+__device__ __forceinline__ bool pool3s2_pair(const PoolArgs& a, int ushift, int img, int oh, int x, int& ow, int& u,
+                                             uint32_t (&oa)[kVec], uint32_t (&ob)[kVec]) {
+  const int units = (int)(a.row_bytes / (4 * kVec));
+  const int op = ushift >= 0 ? x >> ushift : x / units;  // output pair: columns 2 op, 2 op + 1
+  u = x - op * units;
+  ow = 2 * op;
+  if (ow >= a.wo) return false;
+  const uint8_t* rows[3];
+#pragma unroll
+  for (int r = 0; r < 3; ++r)
+    rows[r] = a.x + ((int64_t)img * a.h + min(max(2 * oh - a.pad + r, 0), a.h - 1)) * a.w * a.row_bytes +
+              (int64_t)u * kVec * 4;
+  auto column = [&](int c, PoolAcc<kBits> (&m)[kVec]) {
+    const int64_t off = (int64_t)min(max(2 * ow - a.pad + c, 0), a.w - 1) * a.row_bytes;
+    uint32_t w[3][kVec];
+#pragma unroll
+    for (int r = 0; r < 3; ++r) {
+      const uint32_t* src = reinterpret_cast<const uint32_t*>(rows[r] + off);
+      if constexpr (kVec == 4) {
+        const uint4 q = __ldg(reinterpret_cast<const uint4*>(src));
+        w[r][0] = q.x; w[r][1] = q.y; w[r][2] = q.z; w[r][3] = q.w;
+      } else {
+#pragma unroll
+        for (int v = 0; v < kVec; ++v) w[r][v] = __ldg(src + v);
+      }
+    }
+#pragma unroll
+    for (int v = 0; v < kVec; ++v) m[v].set3(w[0][v], w[1][v], w[2][v]);
+  };
+  PoolAcc<kBits> A[kVec], B[kVec], c1[kVec], c3[kVec];
+  column(0, A);
+  column(1, c1);
+  column(2, B);
+#pragma unroll
+  for (int v = 0; v < kVec; ++v) A[v].max3(c1[v], B[v]);  // A = max(col 0, col 1, col 2); B = col 2
+  column(3, c3);
+  column(4, c1);
+#pragma unroll
+  for (int v = 0; v < kVec; ++v) B[v].max3(c3[v], c1[v]);  // B = max(col 2, col 3, col 4)
+#pragma unroll
+  for (int v = 0; v < kVec; ++v) { oa[v] = A[v].word(); ob[v] = B[v].word(); }
+  return true;
+}
+
+template <int kVec>
+__device__ __forceinline__ void store_words(uint8_t* p, const uint32_t (&o)[kVec]) {
+  if constexpr (kVec == 4) {
+    *reinterpret_cast<uint4*>(p) = make_uint4(o[0], o[1], o[2], o[3]);
+  } else {
+#pragma unroll
+    for (int v = 0; v < kVec; ++v) reinterpret_cast<uint32_t*>(p)[v] = o[v];
+  }
+}
+
+// Grid: z = image, y = output row, x = the row's (output pair, unit) pairs, unit fastest.
+// (3 blocks per SM: measured faster than the unconstrained register count, and than 4)
+template <int kBits, int kVec>
+__global__ void __launch_bounds__(kThreads, kBits == 2 ? 2 : 3) maxpool3s2_pair_kernel(const PoolArgs a, int ushift) {
+  int ow, u;
+  uint32_t oa[kVec], ob[kVec];
+  const int img = blockIdx.z, oh = blockIdx.y;
+  if (!pool3s2_pair<kBits, kVec>(a, ushift, img, oh, blockIdx.x * kThreads + threadIdx.x, ow, u, oa, ob)) return;
+  uint8_t* dst = a.y + (((int64_t)img * a.ho + oh) * a.wo + ow) * a.row_bytes + (int64_t)u * kVec * 4;
+  store_words<kVec>(dst, oa);
+  if (ow + 1 < a.wo) store_words<kVec>(dst + a.row_bytes, ob);
+}
+
+// The byte image of one packed unit (kVec words of 2- or 4-bit codes): one byte per code, in
+// channel order (channel i of a word at bit 8 (i % 4) + bits ((i % q) / 4), q = 32 / bits, so
+// the word's bit planes (w >> bits j) & 0x0303.. / 0x0F0F.. hold channels 4 j .. 4 j + 3).
+template <int kBits, int kVec>
+__device__ __forceinline__ void store_code_bytes(uint8_t* p, const uint32_t (&o)[kVec]) {
+  constexpr int kPl = 8 / kBits;                     // byte planes per word
+  constexpr uint32_t kB = kBits == 2 ? 0x03030303u : 0x0F0F0F0Fu;
+#pragma unroll
+  for (int v = 0; v < kVec; ++v) {
+    uint32_t b[kPl];
+#pragma unroll
+    for (int j = 0; j < kPl; ++j) b[j] = (o[v] >> (kBits * j)) & kB;
+    if constexpr (kPl == 4) *reinterpret_cast<uint4*>(p + 16 * v) = make_uint4(b[0], b[1], b[2], b[3]);
+    else *reinterpret_cast<uint2*>(p + 8 * v) = make_uint2(b[0], b[1]);
+  }
+}
+
+// Max-pool (3x3, stride 2) fused with the expansion of its output for a convolution with
+// padding cpad: writes the pooled codes to a.y and their zero-padded byte image (rows of c
+// bytes; image row (img (ho + 2 cpad) + oh + cpad) (wo + 2 cpad) + ow + cpad) to ws. Grid row
+// y = ho of each image writes the image's border pixels (zeros), spread over its x threads.
+template <int kBits, int kVec>
+__global__ void __launch_bounds__(kThreads, kBits == 2 ? 2 : 3)
+    maxpool3s2_expand_kernel(const PoolArgs a, int ushift, uint8_t* ws, int cpad) {
+  const int img = blockIdx.z, oh = blockIdx.y;
+  const int hp = a.ho + 2 * cpad, wp = a.wo + 2 * cpad;
+  const int64_t ibase = (int64_t)img * hp * wp;
+  constexpr int kUnitBytes = kVec * 4 * 8 / kBits;  // byte-image bytes of one packed unit
+  if (oh == a.ho) {
+    // border: cpad rows on top and bottom (wp pixels each), cpad columns left and right
+    const int units = (int)(a.row_bytes / (4 * kVec));
+    const int nb = 2 * cpad * wp + 2 * cpad * a.ho;
+    const int64_t items = (int64_t)nb * units;
+    for (int64_t e = (int64_t)blockIdx.x * kThreads + threadIdx.x; e < items; e += (int64_t)gridDim.x * kThreads) {
+      const int b = (int)(e / units), uu = (int)(e - (int64_t)b * units);
+      int r, cidx;
+      if (b < 2 * cpad * wp) {
+        const int t = b / wp;
+        r = t < cpad ? t : a.ho + t;  // rows 0 .. cpad - 1, then ho + cpad .. ho + 2 cpad - 1
+        cidx = b - t * wp;
+      } else {
+        const int b2 = b - 2 * cpad * wp, t = b2 / (2 * cpad), s2 = b2 - t * 2 * cpad;
+        r = cpad + t;
+        cidx = s2 < cpad ? s2 : a.wo + s2;
+      }
+      uint8_t* p = ws + ((ibase + (int64_t)r * wp + cidx) * a.c) + (int64_t)uu * kUnitBytes;
+#pragma unroll
+      for (int k = 0; k < kUnitBytes; k += 16) *reinterpret_cast<uint4*>(p + k) = make_uint4(0u, 0u, 0u, 0u);
+    }
+    return;
+  }
+  int ow, u;
+  uint32_t oa[kVec], ob[kVec];
+  if (!pool3s2_pair<kBits, kVec>(a, ushift, img, oh, blockIdx.x * kThreads + threadIdx.x, ow, u, oa, ob)) return;
+  uint8_t* dst = a.y + (((int64_t)img * a.ho + oh) * a.wo + ow) * a.row_bytes + (int64_t)u * kVec * 4;
+  uint8_t* img_row = ws + ((ibase + (int64_t)(oh + cpad) * wp + ow + cpad) * a.c) + (int64_t)u * kUnitBytes;
+  store_words<kVec>(dst, oa);
+  store_code_bytes<kBits, kVec>(img_row, oa);
+  if (ow + 1 < a.wo) {
+    store_words<kVec>(dst + a.row_bytes, ob);
+    store_code_bytes<kBits, kVec>(img_row + a.c, ob);
   }
 }
 
@@ -1156,34 +1278,73 @@ int launch_maxpool(const PoolArgs& a, cudaStream_t stream, std::string* err) {
   // packed 2/4/8-bit rows: bit-plane maxima on whole words (16-byte units when the row allows)
   if ((a.bits == 2 || a.bits == 4 || a.bits == 8) && a.row_bytes % 4 == 0) {
     const bool v4 = a.row_bytes % 16 == 0;
-    const int64_t total = pixels * (a.row_bytes / (v4 ? 16 : 4));
-    const int blocks = elt::blocks_for(total);
-    if (a.k == 3) {
+    const int units = (int)(a.row_bytes / (v4 ? 16 : 4));
+    int ushift = -1;
+    for (int sft = 0; sft < 31; ++sft)
+      if ((1 << sft) == units) ushift = sft;
+    if ((int64_t)a.wo * units >= (1LL << 31) || a.ho > 65535 || a.n > 65535) {
+      *err = "maxpool: output too large for the packed kernel's grid";
+      return 1;
+    }
+    const dim3 blocks((unsigned)elt::blocks_for((int64_t)a.wo * units), (unsigned)a.ho, (unsigned)a.n);
+    if (a.k == 3 && a.stride == 2) {
+      const dim3 pblocks((unsigned)elt::blocks_for((int64_t)((a.wo + 1) / 2) * units), (unsigned)a.ho, (unsigned)a.n);
       if (a.bits == 2) {
-        if (v4) elt::maxpool_packed_kernel<2, 4, 3><<<blocks, elt::kThreads, 0, stream>>>(a);
-        else elt::maxpool_packed_kernel<2, 1, 3><<<blocks, elt::kThreads, 0, stream>>>(a);
+        if (v4) elt::maxpool3s2_pair_kernel<2, 4><<<pblocks, elt::kThreads, 0, stream>>>(a, ushift);
+        else elt::maxpool3s2_pair_kernel<2, 1><<<pblocks, elt::kThreads, 0, stream>>>(a, ushift);
       } else if (a.bits == 4) {
-        if (v4) elt::maxpool_packed_kernel<4, 4, 3><<<blocks, elt::kThreads, 0, stream>>>(a);
-        else elt::maxpool_packed_kernel<4, 1, 3><<<blocks, elt::kThreads, 0, stream>>>(a);
+        if (v4) elt::maxpool3s2_pair_kernel<4, 4><<<pblocks, elt::kThreads, 0, stream>>>(a, ushift);
+        else elt::maxpool3s2_pair_kernel<4, 1><<<pblocks, elt::kThreads, 0, stream>>>(a, ushift);
       } else {
-        if (v4) elt::maxpool_packed_kernel<8, 4, 3><<<blocks, elt::kThreads, 0, stream>>>(a);
-        else elt::maxpool_packed_kernel<8, 1, 3><<<blocks, elt::kThreads, 0, stream>>>(a);
+        if (v4) elt::maxpool3s2_pair_kernel<8, 4><<<pblocks, elt::kThreads, 0, stream>>>(a, ushift);
+        else elt::maxpool3s2_pair_kernel<8, 1><<<pblocks, elt::kThreads, 0, stream>>>(a, ushift);
+      }
+    } else if (a.k == 3) {
+      if (a.bits == 2) {
+        if (v4) elt::maxpool_packed_kernel<2, 4, 3><<<blocks, elt::kThreads, 0, stream>>>(a, ushift);
+        else elt::maxpool_packed_kernel<2, 1, 3><<<blocks, elt::kThreads, 0, stream>>>(a, ushift);
+      } else if (a.bits == 4) {
+        if (v4) elt::maxpool_packed_kernel<4, 4, 3><<<blocks, elt::kThreads, 0, stream>>>(a, ushift);
+        else elt::maxpool_packed_kernel<4, 1, 3><<<blocks, elt::kThreads, 0, stream>>>(a, ushift);
+      } else {
+        if (v4) elt::maxpool_packed_kernel<8, 4, 3><<<blocks, elt::kThreads, 0, stream>>>(a, ushift);
+        else elt::maxpool_packed_kernel<8, 1, 3><<<blocks, elt::kThreads, 0, stream>>>(a, ushift);
       }
     } else if (a.bits == 2) {
-      if (v4) elt::maxpool_packed_kernel<2, 4, 0><<<blocks, elt::kThreads, 0, stream>>>(a);
-      else elt::maxpool_packed_kernel<2, 1, 0><<<blocks, elt::kThreads, 0, stream>>>(a);
+      if (v4) elt::maxpool_packed_kernel<2, 4, 0><<<blocks, elt::kThreads, 0, stream>>>(a, ushift);
+      else elt::maxpool_packed_kernel<2, 1, 0><<<blocks, elt::kThreads, 0, stream>>>(a, ushift);
     } else if (a.bits == 4) {
-      if (v4) elt::maxpool_packed_kernel<4, 4, 0><<<blocks, elt::kThreads, 0, stream>>>(a);
-      else elt::maxpool_packed_kernel<4, 1, 0><<<blocks, elt::kThreads, 0, stream>>>(a);
+      if (v4) elt::maxpool_packed_kernel<4, 4, 0><<<blocks, elt::kThreads, 0, stream>>>(a, ushift);
+      else elt::maxpool_packed_kernel<4, 1, 0><<<blocks, elt::kThreads, 0, stream>>>(a, ushift);
     } else {
-      if (v4) elt::maxpool_packed_kernel<8, 4, 0><<<blocks, elt::kThreads, 0, stream>>>(a);
-      else elt::maxpool_packed_kernel<8, 1, 0><<<blocks, elt::kThreads, 0, stream>>>(a);
+      if (v4) elt::maxpool_packed_kernel<8, 4, 0><<<blocks, elt::kThreads, 0, stream>>>(a, ushift);
+      else elt::maxpool_packed_kernel<8, 1, 0><<<blocks, elt::kThreads, 0, stream>>>(a, ushift);
     }
     return check_launch("maxpool launch", err);
   }
   const int64_t total = pixels * ((a.c + 31) / 32);
   elt::maxpool_kernel<<<elt::blocks_for(total), elt::kThreads, 0, stream>>>(a);
   return check_launch("maxpool launch", err);
+}
+
+int launch_maxpool_expand(const PoolArgs& a, uint8_t* ws, int32_t cpad, cudaStream_t stream, std::string* err) {
+  if (a.k != 3 || a.stride != 2 || (a.bits != 2 && a.bits != 4) || a.row_bytes % 16 != 0 || a.c % 16 != 0) {
+    *err = "maxpool_expand: needs a 3x3 stride-2 pool on 2- or 4-bit codes with 16-byte rows";
+    return 2;
+  }
+  if (a.n == 0 || a.ho == 0 || a.wo == 0) return 0;
+  const int units = (int)(a.row_bytes / 16);
+  int ushift = -1;
+  for (int sft = 0; sft < 31; ++sft)
+    if ((1 << sft) == units) ushift = sft;
+  if ((int64_t)((a.wo + 1) / 2) * units >= (1LL << 31) || a.ho + 1 > 65535 || a.n > 65535) {
+    *err = "maxpool_expand: output too large for the kernel's grid";
+    return 1;
+  }
+  const dim3 blocks((unsigned)elt::blocks_for((int64_t)((a.wo + 1) / 2) * units), (unsigned)(a.ho + 1), (unsigned)a.n);
+  if (a.bits == 2) elt::maxpool3s2_expand_kernel<2, 4><<<blocks, elt::kThreads, 0, stream>>>(a, ushift, ws, cpad);
+  else elt::maxpool3s2_expand_kernel<4, 4><<<blocks, elt::kThreads, 0, stream>>>(a, ushift, ws, cpad);
+  return check_launch("maxpool_expand launch", err);
 }
 
 int launch_pack(const int32_t* codes, int64_t rows, int32_t c, int32_t bits, uint8_t* out,

@@ -152,6 +152,9 @@ struct PoolArgs {
   int64_t row_bytes;
 };
 int launch_maxpool(const PoolArgs& a, cudaStream_t stream, std::string* err);
+// 3x3 stride-2 max-pool on 2-/4-bit codes fused with the zero-padded byte image (padding
+// cpad, rows of a.c bytes, one image after another from ws) of its output
+int launch_maxpool_expand(const PoolArgs& a, uint8_t* ws, int32_t cpad, cudaStream_t stream, std::string* err);
 
 // the bounded-wait self-test (selftest.cu): out receives 5 int64 values
 int launch_wait_selftest(uint32_t* status, int64_t* out, cudaStream_t stream, std::string* err);

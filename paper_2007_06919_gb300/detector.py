@@ -8,12 +8,16 @@ the FPN's nearest-2x top-down maps) are added in the conv epilogue (Eq. 7). Outp
 and one shared expanded-activation workspace are allocated once, up front, so the whole
 forward pass can be captured in a CUDA graph.
 
-Two launch-level fusions, neither of which changes any output value:
+Three launch-level fusions, none of which changes any output value:
 - the classification (256->80) and box (256->4) convs read the same tower output, so they run
   as one 256->84 conv with concatenated weight rows and biases (``fuse_heads``);
 - a stride-1 conv whose only consumer is a stride-1 conv on the workspace path writes that
   consumer's zero-padded byte image in its epilogue (``chain``), so the consumer skips the
-  expansion pass. The head tower uses it: the image of tower layer i is the input of i+1.
+  expansion pass. The head tower uses it: the image of tower layer i is the input of i+1;
+- a max-pool on codes whose output the next conv reads on the workspace path (the stem's
+  3x3 stride-2 pool and the first residual stage) runs inside that conv's expansion pass
+  (``fuse_pool``, aqd_maxpool_expand): the pooled codes are still written for the stage's
+  skip, but not read back for the expansion, and the pool launch disappears.
 """
 from __future__ import annotations
 
@@ -38,6 +42,7 @@ class _ConvPlan:
     reads_image: bool = False   # input image already written by the producer (chained)
     chain_to: "_ConvPlan | None" = None
     image: int = 0         # which of the two chain images this conv reads (when reads_image)
+    pool: object = None    # the max-pool layer fused into this conv's expansion pass
 
 
 def _aligned(nbytes: int, device) -> torch.Tensor:
@@ -54,7 +59,8 @@ class IntDetector:
     named "image". The caller writes the input codes into ``self.tensors["image"]`` (or passes
     a DTensor of that shape to ``forward``)."""
 
-    def __init__(self, layers, image_shape, device="cuda", fuse_heads: bool = True, chain: bool = True):
+    def __init__(self, layers, image_shape, device="cuda", fuse_heads: bool = True, chain: bool = True,
+                 fuse_pool: bool = True):
         self.device = torch.device(device)
         n, h, w, c, bits = image_shape
         self.tensors: dict[str, aqd.DTensor] = {"image": aqd.DTensor.empty(n, h, w, c, bits, device=self.device)}
@@ -93,6 +99,8 @@ class IntDetector:
             self.steps.append(("conv", _ConvPlan(ly, W, rq, sp, jobs, cv.stride, cv.pad, wsb)))
         if chain:
             self._plan_chains(layers)
+        if fuse_pool:
+            self._plan_pool_fusion()
         self.workspace = _aligned(ws_max, self.device) if ws_max else None
         # byte images of chained convs, two per geometry (conv i writes the one conv i+1 reads);
         # their zero borders are written here once and never touched again
@@ -101,7 +109,7 @@ class IntDetector:
             if k == "conv" and p.reads_image and self._image_key(p) not in self.images:
                 self.images[self._image_key(p)] = [_aligned(p.ws_bytes, self.device) for _ in range(2)]
         self.launches = sum(1 + (1 if (k == "conv" and p.ws_bytes and not p.reads_image) else 0)
-                            for k, p in self.steps)
+                            for k, p in self.steps) - sum(1 for k, p in self.steps if k == "conv" and p.pool)
 
     # -------------------------------------------------------------- planning
 
@@ -156,6 +164,17 @@ class IntDetector:
             if p.chain_to is not None:
                 p.chain_to.image = 1 - p.image if p.reads_image else 0
 
+    def _plan_pool_fusion(self):
+        """Marks max-pools whose output is the single input of the next step, a conv on the
+        workspace path that expands its own input (not chained), with 2-, 4- or 8-bit codes:
+        that conv's expansion pass computes the pool (aqd_maxpool_expand)."""
+        for (k0, ly), (k1, p) in zip(self.steps, self.steps[1:]):
+            if (k0 == "pool" and k1 == "conv" and p.ws_bytes and not p.reads_image
+                    and list(p.layer.src) == [ly.dst[0]] and self.tensors[ly.dst[0]].bits in (2, 4, 8)):
+                p.pool = ly
+        fused = {id(p.pool) for k, p in self.steps if k == "conv" and p.pool is not None}
+        self.steps = [(k, p) for k, p in self.steps if not (k == "pool" and id(p) in fused)]
+
     @staticmethod
     def _image_key(p: _ConvPlan):
         return (tuple((x.n, x.h, x.w, x.c) for x, _, _, _ in p.jobs), p.pad, p.ws_bytes)
@@ -176,14 +195,18 @@ class IntDetector:
                 src_ws = self.images[self._image_key(p)][p.image]
             else:
                 src_ws = self.workspace[:p.ws_bytes] if p.ws_bytes else None
+            if p.pool is not None:
+                k, s, pd = p.pool.pool
+                aqd.maxpool_expand(T[p.pool.src[0]], k, s, pd, T[p.pool.dst[0]], p.w, p.stride, p.pad, src_ws,
+                                   stream=stream)
             if p.chain_to is not None:
                 nxt = p.chain_to
-                if not p.reads_image:
+                if not p.reads_image and p.pool is None:
                     aqd.conv_expand_input(p.jobs, p.w, p.stride, p.pad, src_ws, stream=stream)
                 aqd.conv_int_grouped_chain(p.jobs, p.w, p.stride, p.pad, rq=p.rq, sp=p.sp, workspace=src_ws,
                                            next_pad=nxt.pad, next_workspace=self.images[self._image_key(nxt)][nxt.image],
                                            stream=stream)
-            elif p.reads_image:
+            elif p.reads_image or p.pool is not None:
                 aqd.conv_int_grouped_expanded(p.jobs, p.w, p.stride, p.pad, rq=p.rq, sp=p.sp, workspace=src_ws,
                                               stream=stream)
             else:

@@ -50,7 +50,7 @@ def test_detector_reduced_size_bit_exact(size, chain, fuse):
     import torch
     import oracle
     from paper_2007_06919_gb300 import aqd
-    wl, layers, img, net = _build(*size, chain=chain, fuse_heads=fuse)
+    wl, layers, img, net = _build(*size, chain=chain, fuse_heads=fuse, fuse_pool=fuse)
     net.forward()
     torch.cuda.synchronize()
     assert aqd.device_status() == 0
@@ -76,6 +76,9 @@ def test_detector_plan_uses_fast_paths():
     chained = [p.layer.name for k, p in net.steps if k == "conv" and p.chain_to is not None]
     for i in range(4):
         assert f"head.tower{i}" in chained
+    # the stem's max-pool runs in the first residual stage's expansion pass
+    assert not [p for k, p in net.steps if k == "pool"]
+    assert [p.pool.name for k, p in net.steps if k == "conv" and p.pool is not None] == ["pool"]
     assert set(net.fused) == {f"cls.{l}+box.{l}" for l in range(5)}
     ops = 0
     for ly in layers:

@@ -195,7 +195,8 @@ def test_residual_add_packed_main_operand(c, a_bits, b_bits, out_bits):
 # rows; 8-bit 4 ch), and the generic kernel (8-bit 3 ch, 3-bit)
 @pytest.mark.parametrize("bits,c,k,stride,pad", [(4, 64, 3, 2, 1), (2, 256, 3, 2, 1), (8, 3, 2, 2, 0),
                                                   (3, 32, 3, 1, 1), (2, 32, 3, 1, 1), (8, 32, 3, 2, 1),
-                                                  (8, 4, 2, 2, 0), (4, 96, 3, 2, 0)])
+                                                  (8, 4, 2, 2, 0), (4, 96, 3, 2, 0), (4, 64, 3, 2, 2),
+                                                  (2, 64, 3, 2, 1)])
 def test_maxpool_matches_oracle(bits, c, k, stride, pad):
     rng = np.random.default_rng(bits + c)
     x = synth.act_codes(rng, (2, 41, 67, c), bits)

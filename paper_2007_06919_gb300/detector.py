@@ -165,12 +165,13 @@ class IntDetector:
                 p.chain_to.image = 1 - p.image if p.reads_image else 0
 
     def _plan_pool_fusion(self):
-        """Marks max-pools whose output is the single input of the next step, a conv on the
-        workspace path that expands its own input (not chained), with 2-, 4- or 8-bit codes:
+        """Marks 3x3 stride-2 max-pools on 2- or 4-bit codes whose output is the single input of
+        the next step, a conv on the workspace path that expands its own input (not chained):
         that conv's expansion pass computes the pool (aqd_maxpool_expand)."""
         for (k0, ly), (k1, p) in zip(self.steps, self.steps[1:]):
             if (k0 == "pool" and k1 == "conv" and p.ws_bytes and not p.reads_image
-                    and list(p.layer.src) == [ly.dst[0]] and self.tensors[ly.dst[0]].bits in (2, 4, 8)):
+                    and tuple(ly.pool[:2]) == (3, 2) and list(p.layer.src) == [ly.dst[0]]
+                    and self.tensors[ly.dst[0]].bits in (2, 4)):
                 p.pool = ly
         fused = {id(p.pool) for k, p in self.steps if k == "conv" and p.pool is not None}
         self.steps = [(k, p) for k, p in self.steps if not (k == "pool" and id(p) in fused)]

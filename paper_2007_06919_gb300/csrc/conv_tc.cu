@@ -267,7 +267,7 @@ template <bool kSkip, bool kIntAcc = false>
 __device__ __forceinline__ void general_group(const Params& p, const uint32_t* v, const EpiChan* ep,
                                               const uint8_t* srow, int ch0, int ncols, float sc, int32_t (&out)[32]) {
   int32_t sk[32];
-  if (kSkip && p.has_skip) load_skip_group(p, srow, ch0, ncols, sk);
+  if (kSkip) load_skip_group(p, srow, ch0, ncols, sk);
   else {
 #pragma unroll
     for (int i = 0; i < 32; ++i) sk[i] = 0;
@@ -278,7 +278,7 @@ __device__ __forceinline__ void general_group(const Params& p, const uint32_t* v
     const int64_t acc = kIntAcc ? (int64_t)(int32_t)v[i]
                                 : (int64_t)__float2int_rn(__uint_as_float(v[i]) * sc);
     const EpiChan ec = ep[i];
-    out[i] = (kSkip && p.has_skip) ? epilogue<true>(acc, sk[i], ec, p.scale_main, p.out_bits)
+    out[i] = kSkip ? epilogue<true>(acc, sk[i], ec, p.scale_main, p.out_bits)
                         : epilogue<false>(acc, 0, ec, p.scale_main, p.out_bits);
   }
 }
@@ -870,7 +870,7 @@ conv_tc_kernel(const __grid_constant__ Maps maps, const __grid_constant__ Params
               if (r >= 33 && sb) { ef.y = ec.m0; ef.z = 1 << (r - 33); ef.w = r - 32; }
               else fq = 0;
             }
-            if (p.has_skip) { ec.c = p.skip_c[idx]; ec.d = p.skip_d[idx]; }
+            if (kSkip) { ec.c = p.skip_c[idx]; ec.d = p.skip_d[idx]; }
           }
           epi[col] = ec;
           reinterpret_cast<int4*>(epi + 256)[col] = ef;
@@ -880,7 +880,7 @@ conv_tc_kernel(const __grid_constant__ Maps maps, const __grid_constant__ Params
         // 32-bit skip path (fast_skip_group): default direction, code skips, d >= 8 everywhere
         // (int32 skips: 64-bit product, any d >= 1)
         int fsk = 0;
-        if (kSkip && p.has_skip && p.scale_main == 0 && out_bits != 32 && fq && sbias) {
+        if (kSkip && p.scale_main == 0 && out_bits != 32 && fq && sbias) {
           const int dmin = p.skip_bits <= 8 ? 8 : 1;
           int okd = 1;
           for (int col = et; col < TBN; col += kEpiThreads)
@@ -892,7 +892,9 @@ conv_tc_kernel(const __grid_constant__ Maps maps, const __grid_constant__ Params
       }
       const int fast_req = flags & 1, small_bias = (flags >> 1) & 1, fast_skip = (flags >> 2) & 1;
       // 0: general int64 epilogue; 1: fast requant to codes; 2: int32 output, no skip
-      const int mode = (kSplit || p.has_skip) ? 0 : (out_bits == 32 ? 2 : (fast_req ? 1 : 0));
+      // (kSkip: the skip instantiation runs exactly the calls with a skip, so its mode is 0 at
+      // compile time and it carries no code or registers of the other modes)
+      const int mode = (kSplit || kSkip) ? 0 : (out_bits == 32 ? 2 : (fast_req ? 1 : 0));
       const bool magic = p.acc_small && (mode == 2 ? small_bias : fast_req);
       const uint32_t buf = lt & 1;
       if (!mbar_wait(b_tfull + 8 * buf, (lt >> 1) & 1, abort_flag)) { ok = false; break; }
@@ -1036,7 +1038,7 @@ conv_tc_kernel(const __grid_constant__ Maps maps, const __grid_constant__ Params
               }
             } else {
               const uint8_t* srow = nullptr;
-              if (kSkip && p.has_skip) {
+              if (kSkip) {
                 int img, ho, wo;
                 if constexpr (kFlat) {
                   img = oimg; ho = oh; wo = ow;

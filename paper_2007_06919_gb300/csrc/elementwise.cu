@@ -1183,7 +1183,16 @@ static void launch_staged_k(const EltArgs& a, int ts, int sms, cudaStream_t stre
   g.stage_bytes = (g.a_bytes + g.s_bytes + 127u) / 128u * 128u;
   g.tab_bytes = ts > 0 ? (uint32_t)((((size_t)ts << kSkipBits) * sizeof(int32_t) + 127) / 128 * 128) : 0u;
   const size_t smem = g.tab_bytes + (size_t)g.stages * g.stage_bytes;
-  cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  // the dynamic limit goes to the device maximum (less the kernel's static barriers), never to
+  // this call's size: a graph node captured earlier with a larger table must stay launchable
+  // after a smaller call
+  int dev = 0, optin = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  cudaFuncAttributes fa{};
+  cudaFuncGetAttributes(&fa, kern);
+  const int maxdyn = optin - (int)fa.sharedSizeBytes;
+  cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, maxdyn > (int)smem ? maxdyn : (int)smem);
   int occ = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, elt::kThreads + 32, smem) != cudaSuccess || occ < 1)
     occ = 1;

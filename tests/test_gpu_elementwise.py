@@ -210,3 +210,39 @@ def test_maxpool_matches_oracle(bits, c, k, stride, pad):
 
 def test_device_status_is_clean():
     assert aqd.device_status() == 0
+
+
+def test_staged_graph_replays_after_a_smaller_call():
+    """A CUDA graph holding the staged skip add with a 256-channel table (the larger shared
+    memory plan) still replays, bit-exact, after an eager call of the same kernel with a
+    128-channel table: its shared-memory limit is never lowered below an earlier capture's."""
+    rng = np.random.default_rng(314)
+
+    def case(c, n=2, h=21, w=33):
+        a = rng.integers(-30000, 30000, size=(n, h, w, c)).astype(np.int32)
+        b = synth.act_codes(rng, (n, h, w, c), 4)
+        m0, sh, bias = synth.requant_params(rng, 1, c, calib_std=20000.0, out_bits=2)
+        cc, dd = synth.skip_params(rng, 1, c, sh)
+        at, bt = oracle.CodeTensor.from_codes(a, 32), oracle.CodeTensor.from_codes(b, 4)
+        ref = oracle.residual_add(at, bt, cc, dd, out_bits=2, m0=m0, shift=sh, bias=bias)
+        args = (to_device(at), to_device(bt), aqd.SkipParams.from_numpy(cc, dd), aqd.DTensor.empty(n, h, w, c, 2),
+                aqd.RequantParams.from_numpy(m0, sh, bias))
+        return args, ref
+
+    (a1, b1, s1, y1, r1), ref1 = case(256)
+    (a2, b2, s2, y2, r2), ref2 = case(128)
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):
+        aqd.residual_add_int(a1, b1, s1, y1, rq=r1, stream=stream)
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        aqd.residual_add_int(a1, b1, s1, y1, rq=r1, stream=stream)
+    aqd.residual_add_int(a2, b2, s2, y2, rq=r2)
+    torch.cuda.synchronize()
+    y1.data.fill_(0xA5)
+    g.replay()
+    torch.cuda.synchronize()
+    assert aqd.device_status() == 0
+    assert_same(y1.data.cpu().numpy().reshape(ref1.packed.shape), ref1.packed, 256, 2, "graph replay")
+    assert_same(y2.data.cpu().numpy().reshape(ref2.packed.shape), ref2.packed, 128, 2, "smaller call")

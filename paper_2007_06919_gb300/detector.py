@@ -108,8 +108,10 @@ class IntDetector:
         for k, p in self.steps:
             if k == "conv" and p.reads_image and self._image_key(p) not in self.images:
                 self.images[self._image_key(p)] = [_aligned(p.ws_bytes, self.device) for _ in range(2)]
+        # a conv that expands its own input is two launches (with a fused pool the expansion
+        # launch is the pool's, whose own step is gone)
         self.launches = sum(1 + (1 if (k == "conv" and p.ws_bytes and not p.reads_image) else 0)
-                            for k, p in self.steps) - sum(1 for k, p in self.steps if k == "conv" and p.pool)
+                            for k, p in self.steps)
 
     # -------------------------------------------------------------- planning
 

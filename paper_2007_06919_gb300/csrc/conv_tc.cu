@@ -110,6 +110,8 @@ struct Params {
   int32_t acc_small;  // |acc| < 2^22 guaranteed by K * max|x| * max|w|
   int32_t cin_chunks; // cin / 128 (flat path)
   int32_t dp_tiles;   // tiles [0, dp_tiles) are bn wide; later ones are the two bn/2 halves
+  int32_t contig;     // each CTA takes one contiguous range of tiles (single CTAs, one layer,
+                      // no half tiles) instead of every gridDim-th tile
                       // of the remaining full tiles (the last, partial wave)
   uint32_t off_b, off_epi, off_bar, off_qtab;
   uint32_t off_ostage;  // int32 outputs: per-warp staging blocks for row-contiguous stores (0: none)
@@ -604,8 +606,19 @@ conv_tc_kernel(const __grid_constant__ Maps maps, const __grid_constant__ Params
   if (threadIdx.x == 0) grid_dep_launch();
 
   const int nk = p.num_kchunks * p.a_planes;  // K chunks, over every plane of the image
-  const int first_tile = kPair ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
-  const int tile_stride = kPair ? (int)(gridDim.x >> 1) : (int)gridDim.x;
+  // This CTA's tiles: every tile_stride-th from first_tile, or (contig) the range
+  // [first_tile, tile_end) of a balanced split of the tiles over the grid, so that a CTA's
+  // consecutive tiles are neighbours (one level's table, adjacent rows in L2)
+  int first_tile = kPair ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+  int tile_stride = kPair ? (int)(gridDim.x >> 1) : (int)gridDim.x;
+  int tile_end = p.total_tiles;
+  if (!kPair && p.contig) {
+    const int q = p.total_tiles / (int)gridDim.x, r = p.total_tiles % (int)gridDim.x;
+    const int b = (int)blockIdx.x;
+    first_tile = b * q + (b < r ? b : r);
+    tile_end = first_tile + q + (b < r ? 1 : 0);
+    tile_stride = 1;
+  }
 
   if (warp == kWarpMma) {
     // ------------------------------------------------------------ MMA issuer
@@ -624,7 +637,7 @@ conv_tc_kernel(const __grid_constant__ Maps maps, const __grid_constant__ Params
       uint32_t it = 0, lt = 0, s = 0, ph = 0;
       bool ok = true;
       bool next_ready = false;  // the stage after the current one is known to be full
-      for (int t = first_tile; t < p.total_tiles && ok; t += tile_stride, ++lt) {
+      for (int t = first_tile; t < tile_end && ok; t += tile_stride, ++lt) {
         const uint32_t buf = lt & 1;
         // (half-width tiles are counted within a layer; a launch of several layers has none)
         const int t_in_layer = p.nlayers > 1 ? t - (t / p.layer_tiles) * p.layer_tiles : t;
@@ -685,7 +698,7 @@ conv_tc_kernel(const __grid_constant__ Maps maps, const __grid_constant__ Params
     if (lane == 0) {
       uint32_t it = 0, s = 0, ph = 0;
       bool ok = true;
-      for (int t = first_tile; t < p.total_tiles && ok; t += tile_stride) {
+      for (int t = first_tile; t < tile_end && ok; t += tile_stride) {
         const TileInfo ti = tile_info(p, t);
         // per tile: the first workspace row of this CTA's A rows (flat path) and the image width
         int row0 = 0, wp = 0;
@@ -755,7 +768,7 @@ conv_tc_kernel(const __grid_constant__ Maps maps, const __grid_constant__ Params
     const int sub = row >> 7, r7 = row & 7;
     uint8_t* arow = smem + sub * kSubA + (row & 127) * BK;
     int my_tiles = 0;
-    for (int t = first_tile; t < p.total_tiles; t += tile_stride) ++my_tiles;
+    for (int t = first_tile; t < tile_end; t += tile_stride) ++my_tiles;
     const int total = my_tiles * nk;
 
     RowCursor<kXBits> rc{};
@@ -836,7 +849,7 @@ conv_tc_kernel(const __grid_constant__ Maps maps, const __grid_constant__ Params
     // without table loads or barriers
     long long cur_key = -1;  // (level, first channel, width) of the tables
     int flags = 0;           // bit 0: 32-bit requant form, 1: |bias| <= 2^30, 2: 32-bit skip form
-    for (int t = first_tile; t < p.total_tiles; t += tile_stride, ++lt) {
+    for (int t = first_tile; t < tile_end; t += tile_stride, ++lt) {
       const TileInfo ti = tile_info(p, t);
       const ConvJobDev& jb = p.jobs[ti.job];
       // this tile's output channels that exist (a last N tile may reach past cout; packed
@@ -1476,6 +1489,9 @@ int launch_conv_tc(const ConvArgs& a, cudaStream_t stream, std::string* err) {
   // (a launch of several layers has no half-width tiles: every layer keeps the same tiles)
   prm.dp_tiles = nlayers > 1 ? tiles : split_start(tiles, pair ? sms / 2 : sms, BN, a.split_w != 0);
   prm.total_tiles = nlayers * (prm.dp_tiles + 2 * (tiles - prm.dp_tiles));
+  // contiguous tile ranges for single-CTA launches of one layer on the workspace path with no
+  // half tiles (the FP4 output conv): neighbouring tiles share a level's tables and halo rows
+  prm.contig = (!pair && flat && nlayers <= 1 && prm.dp_tiles == tiles) ? 1 : 0;
   prm.nlayers = nlayers;
   prm.layer_tiles = prm.total_tiles / nlayers;
   prm.num_kchunks = flat ? (fp4 ? a.k_total / 2 : a.k_total) / bk : a.k_pad / BK;

@@ -37,9 +37,9 @@ METRIC = "int-only conv TOPS & % of INT8 tensor peak; detector-head images/s at 
 # DRAM bytes (read + write) of one chained tower-layer conv_tc launch, from an ncu capture
 # (dram__bytes_read.sum + dram__bytes_write.sum) of the build of conv_tc.cu whose SHA-256
 # prefix is recorded beside it; reported as null when the source differs from that build.
-TOWER_CONV_TRAFFIC = {"bytes": 15763712, "conv_tc_sha256": "b0eacf921e1801d4",
+TOWER_CONV_TRAFFIC = {"bytes": 15791872, "conv_tc_sha256": "27b166ea8ac326ff",
                       "profile": "profiles/conv_tc_retina_head_800x1333_b2_2bit_full.md (dram__bytes_read.sum "
-                                 "15.05 MB + dram__bytes_write.sum 0.72 MB, one fused tower launch)"}
+                                 "15.04 MB + dram__bytes_write.sum 0.75 MB, one fused tower launch)"}
 KTOWERS = 4  # chained 4-layer towers per timed kernel graph, each on its own workspaces
 WORKLOAD = "retina_head_800x1333_b2_2bit"
 

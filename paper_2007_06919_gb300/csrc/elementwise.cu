@@ -503,8 +503,9 @@ __global__ void __launch_bounds__(kThreads, 3)
 
 // The same requant / skip add with its inputs staged through shared memory by the bulk-copy
 // engine: rows of consecutive pixels are contiguous in HBM (the int32 tensor, and the skip
-// tensor on the same grid), so one 1D bulk copy per operand fills a stage of kStagePix... pixels.
-// A producer warp (one thread) keeps `stages` stages in flight per block, so the bytes in
+// tensor on the same grid), so one 1D bulk copy per operand fills a stage of P pixels (about
+// 32 KB of int32 rows, StageGeo). A producer warp (one thread) keeps `stages` stages in flight
+// per block, so the bytes in
 // flight no longer depend on registers; 8 consumer warps take the filled stages in turn.
 // Warp w owns channel block w % cblocks (kV channels per lane, constants in registers) and
 // every (8 / cblocks)-th pixel of a stage. The epilogue is the table form above (exact when

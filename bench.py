@@ -538,6 +538,35 @@ def run_sweep(args):
         emit("eltwise_maxpool3x3s2_expand_4bit_8x400x672x64", ms, 0, nb, frac_hbm=nb / (ms * 1e-3) / 1e9 / hbm,
              hbm_peak_gbs=hbm, bytes_note="input + pooled codes + the conv's zero-padded byte image")
 
+    # the training-side steps (Sec. 3.1.2, Sec. 3.2.2), HBM-bound: Eq. 2 fake quantization of a
+    # 16x100x168x256 float32 activation tensor (4 B read, 4 B value + 1 B code written per
+    # element), its STE backward (x and gy read, gx written: 12 B per element, plus the
+    # interval's gradient), and the multi-level BN batch statistics of the five FPN levels at
+    # batch 16, 256 channels (4 B read per element)
+    if want in ("all", "train"):
+        hbm = peaks["hbm_gbs"]
+        rng = np.random.default_rng(6)
+        n = 16 * 100 * 168 * 256
+        x = torch.from_numpy(rng.normal(1.0, 1.2, size=n).astype(np.float32)).to(dev)
+        gy = torch.from_numpy(rng.normal(0, 1, size=n).astype(np.float32)).to(dev)
+        y = torch.empty_like(x)
+        codes = torch.empty(n, dtype=torch.uint8, device=dev)
+        gx = torch.empty_like(x)
+        ms = timed(lambda: aqd.fake_quant(x, 2.5, 4, y=y, codes=codes, stream=stream))
+        emit("train_fake_quant_eq2_4bit_16x100x168x256", ms, 0, 9 * n, frac_hbm=9 * n / (ms * 1e-3) / 1e9 / hbm,
+             hbm_peak_gbs=hbm)
+        ms = timed(lambda: aqd.fake_quant_backward(x, gy, 2.5, 4, gx=gx, stream=stream))
+        emit("train_fake_quant_eq2_backward_4bit_16x100x168x256", ms, 0, 12 * n,
+             frac_hbm=12 * n / (ms * 1e-3) / 1e9 / hbm, hbm_peak_gbs=hbm)
+        del x, gy, y, codes, gx
+        zs = [torch.from_numpy(rng.normal(0.5, 2.0, size=(16, h, w, 256)).astype(np.float32)).to(dev)
+              for h, w in [(100, 168), (50, 84), (25, 42), (13, 21), (7, 11)]]
+        nb = 4 * sum(z.numel() for z in zs)
+        ms = timed(lambda: aqd.bn_level_stats(zs, stream=stream))
+        emit("train_bn_level_stats_5_levels_b16_256ch", ms, 0, nb, frac_hbm=nb / (ms * 1e-3) / 1e9 / hbm,
+             hbm_peak_gbs=hbm)
+        del zs
+
     # config 4: first tower layer of the head at batch 16, 2/3/4/8-bit
     for bits in ((2, 3, 4, 8) if want in ("all", "config4") else ()):
         wl = synth.config4(bits)
@@ -577,7 +606,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-detector", action="store_true",
                     help="skip the whole-detector images/s measurement (batch 8, 800x1344)")
-    ap.add_argument("--sweep", nargs="?", const="all", default=None, choices=["all", "config0", "config1", "config3", "config4", "eltwise"],
+    ap.add_argument("--sweep", nargs="?", const="all", default=None, choices=["all", "config0", "config1", "config3", "config4", "eltwise", "train"],
                     help="measure the other workloads (several lines)")
     args = ap.parse_args()
     if args.impl == "reference":

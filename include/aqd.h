@@ -311,6 +311,42 @@ aqd_status aqd_conv_int_static_workspace(const aqd_tensor* x, const aqd_conv_wei
                                          const aqd_tensor* skip, const aqd_skip_params* sp, aqd_tensor* y,
                                          aqd_stream_t stream);
 
+/* ---- training side (Sec. 3.1.2, Sec. 3.2.2) --------------------------------------- */
+
+/* The quantizers with learnable intervals. weight = 0: Eq. 2 on activations,
+ *   eta = round(clip(x / nu, 0, 1) (2^b - 1)), y = eta nu / (2^b - 1);
+ * weight = 1: Eq. 3 on weights,
+ *   eta = round((clip(w / nu, -1, 1) + 1) / 2 (2^b - 1)), y = (2 eta / (2^b - 1) - 1) nu.
+ * "round" is half-up. Every code is decided in float32 in that order (one correctly rounded
+ * division x / nu, the clip, the products, floor(v + 0.5); no fused multiply-add), so a float32
+ * restatement of the equations gives the same codes and values. x, y: n float32 (device,
+ * 4-byte aligned; 16-byte alignment takes vector loads); codes: n uint8 codes eta or NULL;
+ * y may be NULL when codes is given. bits 1..8, nu > 0. */
+aqd_status aqd_fake_quant(const float* x, int64_t n, float nu, int32_t bits, int32_t weight, float* y,
+                          uint8_t* codes, aqd_stream_t stream);
+
+/* The Straight-Through Estimator backward of aqd_fake_quant (the rounding's derivative taken
+ * as 1). gx = gy where the value lies inside the clip range (0 < x / nu < 1 for Eq. 2,
+ * -1 < w / nu < 1 for Eq. 3), else 0 (gx may be NULL). *gnu (one device float64) =
+ * sum of gy * d y / d nu with d y / d nu = eta / Q - x / nu inside, 1 above, 0 below (Eq. 2) and
+ * 2 eta / Q - 1 - w / nu inside, 1 above, -1 below (Eq. 3), Q = 2^b - 1: float32 within runs of
+ * a thread, float64 across threads, a fixed order across blocks (deterministic).
+ * workspace: aqd_fake_quant_backward_workspace_bytes() bytes, 8-byte aligned. */
+size_t aqd_fake_quant_backward_workspace_bytes(void);
+aqd_status aqd_fake_quant_backward(const float* x, const float* gy, int64_t n, float nu, int32_t bits, int32_t weight,
+                                   float* gx, double* gnu, void* workspace, size_t ws_bytes, aqd_stream_t stream);
+
+/* Batch statistics of the multi-level BN (Sec. 3.2.2, Fig. 3: one BN per FPN level over a
+ * shared head) during training: for level l, the per-channel mean and biased variance of the
+ * float32 tensor z[l] ([pixels[l]][c], channels last, device) over all its pixels, written as
+ * float64 mean[l][c], var[l][c] (device). z and pixels are host arrays of `levels` (1..8)
+ * entries. Sums are shifted by the level's first pixel, float32 over runs of 32 pixels and
+ * float64 beyond. workspace: aqd_bn_level_stats_workspace_bytes(levels, c) bytes (0 for
+ * invalid arguments), 8-byte aligned. */
+size_t aqd_bn_level_stats_workspace_bytes(int32_t levels, int32_t c);
+aqd_status aqd_bn_level_stats(const float* const* z, const int64_t* pixels, int32_t levels, int32_t c, double* mean,
+                              double* var, void* workspace, size_t ws_bytes, aqd_stream_t stream);
+
 /* ---- elementwise ------------------------------------------------------------------ */
 
 /* y = requant(sat32(acc + bias)) per channel at `level`: Eq. 6 + Eq. 2 on an int32

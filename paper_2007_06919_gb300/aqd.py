@@ -58,7 +58,9 @@ EXPORTS = ["aqd_row_bytes", "aqd_quantize_multiplier", "aqd_status_string", "aqd
            "aqd_conv_int_grouped", "aqd_conv_workspace_bytes", "aqd_conv_expand_input",
            "aqd_conv_int_grouped_expanded", "aqd_conv_int_grouped_chain", "aqd_requant", "aqd_residual_add_int",
            "aqd_maxpool_codes", "aqd_maxpool_expand", "aqd_conv_int_static_workspace", "aqd_selftest_wait_timeout",
-           "aqd_conv_tower_sync_bytes", "aqd_conv_int_grouped_tower"]
+           "aqd_conv_tower_sync_bytes", "aqd_conv_int_grouped_tower", "aqd_fake_quant",
+           "aqd_fake_quant_backward_workspace_bytes", "aqd_fake_quant_backward",
+           "aqd_bn_level_stats_workspace_bytes", "aqd_bn_level_stats"]
 
 _lib = None
 
@@ -125,10 +127,19 @@ def load(build_if_missing: bool = True):
     L.aqd_maxpool_codes.argtypes = [ctypes.POINTER(_Tensor), i32, i32, i32, ctypes.POINTER(_Tensor), vp]
     L.aqd_maxpool_expand.argtypes = [ctypes.POINTER(_Tensor), i32, i32, i32, ctypes.POINTER(_Tensor),
                                      ctypes.POINTER(_Weights), i32, i32, vp, ctypes.c_size_t, vp]
+    f32, i64, sz = ctypes.c_float, ctypes.c_int64, ctypes.c_size_t
+    L.aqd_fake_quant.argtypes = [vp, i64, f32, i32, i32, vp, vp, vp]
+    L.aqd_fake_quant_backward_workspace_bytes.restype = sz
+    L.aqd_fake_quant_backward_workspace_bytes.argtypes = []
+    L.aqd_fake_quant_backward.argtypes = [vp, vp, i64, f32, i32, i32, vp, vp, vp, sz, vp]
+    L.aqd_bn_level_stats_workspace_bytes.restype = sz
+    L.aqd_bn_level_stats_workspace_bytes.argtypes = [i32, i32]
+    L.aqd_bn_level_stats.argtypes = [ctypes.POINTER(vp), ctypes.POINTER(i64), i32, i32, vp, vp, vp, sz, vp]
     for name in ("aqd_quantize_multiplier", "aqd_device_status", "aqd_pack_codes", "aqd_unpack_codes",
                  "aqd_conv_prepare_weights", "aqd_conv_int", "aqd_conv_int_grouped", "aqd_conv_expand_input",
                  "aqd_conv_int_grouped_expanded", "aqd_conv_int_grouped_chain", "aqd_requant",
-                 "aqd_residual_add_int", "aqd_maxpool_codes", "aqd_maxpool_expand"):
+                 "aqd_residual_add_int", "aqd_maxpool_codes", "aqd_maxpool_expand", "aqd_fake_quant",
+                 "aqd_fake_quant_backward", "aqd_bn_level_stats"):
         getattr(L, name).restype = c_int
     _lib = L
     return L
@@ -478,6 +489,55 @@ def maxpool_expand(x: DTensor, k: int, stride: int, pad: int, y: DTensor, w: Con
     _check(load().aqd_maxpool_expand(ctypes.byref(xc), k, stride, pad, ctypes.byref(yc), ctypes.byref(w.desc),
                                      conv_stride, conv_pad, wsp, wsb, _stream(stream)), "aqd_maxpool_expand")
     return y
+
+
+def _f32(t: torch.Tensor | None):
+    if t is None:
+        return None
+    if t.dtype != torch.float32 or not t.is_cuda or not t.is_contiguous():
+        raise ValueError("expected a contiguous float32 CUDA tensor")
+    return t.data_ptr()
+
+
+def fake_quant(x: torch.Tensor, nu: float, bits: int, *, weight: bool = False, y: torch.Tensor | None = None,
+               codes: torch.Tensor | None = None, stream=None):
+    """Eq. 2 (weight=False) / Eq. 3 (weight=True) on a float32 tensor: returns (y, codes), the
+    fake-quantized values and the uint8 codes (allocated when not given)."""
+    y = torch.empty_like(x) if y is None else y
+    codes = torch.empty(x.shape, dtype=torch.uint8, device=x.device) if codes is None else codes
+    _check(load().aqd_fake_quant(_f32(x), x.numel(), float(nu), bits, int(weight), _f32(y), codes.data_ptr(),
+                                 _stream(stream)), "aqd_fake_quant")
+    return y, codes
+
+
+def fake_quant_backward(x: torch.Tensor, gy: torch.Tensor, nu: float, bits: int, *, weight: bool = False,
+                        gx: torch.Tensor | None = None, stream=None):
+    """The STE backward of fake_quant: returns (gx, gnu) with gnu a one-element float64 CUDA
+    tensor (the interval's gradient)."""
+    gx = torch.empty_like(x) if gx is None else gx
+    gnu = torch.empty(1, dtype=torch.float64, device=x.device)
+    ws = torch.empty(int(load().aqd_fake_quant_backward_workspace_bytes()), dtype=torch.uint8, device=x.device)
+    _check(load().aqd_fake_quant_backward(_f32(x), _f32(gy), x.numel(), float(nu), bits, int(weight), _f32(gx),
+                                          gnu.data_ptr(), ws.data_ptr(), ws.numel(), _stream(stream)),
+           "aqd_fake_quant_backward")
+    return gx, gnu
+
+
+def bn_level_stats(zs, stream=None):
+    """Per-level batch mean and biased variance (float64 [levels, c]) of float32 CUDA tensors
+    with channels last (Sec. 3.2.2's multi-level BN)."""
+    c = zs[0].shape[-1]
+    dev = zs[0].device
+    nlev = len(zs)
+    ptrs = (ctypes.c_void_p * nlev)(*[_f32(z) for z in zs])
+    pix = (ctypes.c_int64 * nlev)(*[z.numel() // c for z in zs])
+    mean = torch.empty((nlev, c), dtype=torch.float64, device=dev)
+    var = torch.empty((nlev, c), dtype=torch.float64, device=dev)
+    wsb = int(load().aqd_bn_level_stats_workspace_bytes(nlev, c))
+    ws = torch.empty(max(wsb, 8), dtype=torch.uint8, device=dev)
+    _check(load().aqd_bn_level_stats(ptrs, pix, nlev, c, mean.data_ptr(), var.data_ptr(), ws.data_ptr(), ws.numel(),
+                                     _stream(stream)), "aqd_bn_level_stats")
+    return mean, var
 
 
 def device_status(stream=None) -> int:

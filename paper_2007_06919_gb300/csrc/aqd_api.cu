@@ -808,6 +808,68 @@ aqd_status aqd_maxpool_expand(const aqd_tensor* x, int32_t k, int32_t stride, in
   return st ? fail((aqd_status)st, err) : AQD_OK;
 }
 
+// ---------------------------------------------------------------- training-side steps
+
+static constexpr int32_t kFqParts = 1024;  // float64 block partials of the interval's gradient
+
+size_t aqd_fake_quant_backward_workspace_bytes(void) { return (size_t)kFqParts * sizeof(double); }
+
+static bool fq_args_ok(int64_t n, float nu, int32_t bits, int32_t weight, std::string* err) {
+  if (n < 0) { *err = "n must be >= 0"; return false; }
+  if (!(nu > 0.0f) || !std::isfinite(nu)) { *err = "nu must be a positive finite interval"; return false; }
+  if (bits < 1 || bits > 8) { *err = "bits must be 1..8"; return false; }
+  if (weight != 0 && weight != 1) { *err = "weight must be 0 (Eq. 2) or 1 (Eq. 3)"; return false; }
+  return true;
+}
+
+aqd_status aqd_fake_quant(const float* x, int64_t n, float nu, int32_t bits, int32_t weight, float* y,
+                          uint8_t* codes, aqd_stream_t stream) {
+  std::string err;
+  if (!fq_args_ok(n, nu, bits, weight, &err)) return fail(AQD_ERR_INVALID, err);
+  if (n > 0 && (!x || (!y && !codes))) return fail(AQD_ERR_INVALID, "x and at least one of y, codes are required");
+  if (((uintptr_t)x | (uintptr_t)y) % 4 != 0) return fail(AQD_ERR_INVALID, "x and y must be 4-byte aligned");
+  const int st = launch_fake_quant(x, n, nu, bits, weight != 0, y, codes, static_cast<cudaStream_t>(stream), &err);
+  return st ? fail((aqd_status)st, err) : AQD_OK;
+}
+
+aqd_status aqd_fake_quant_backward(const float* x, const float* gy, int64_t n, float nu, int32_t bits, int32_t weight,
+                                   float* gx, double* gnu, void* workspace, size_t ws_bytes, aqd_stream_t stream) {
+  std::string err;
+  if (!fq_args_ok(n, nu, bits, weight, &err)) return fail(AQD_ERR_INVALID, err);
+  if (!gnu) return fail(AQD_ERR_INVALID, "gnu is required");
+  if (n > 0 && (!x || !gy)) return fail(AQD_ERR_INVALID, "x and gy are required");
+  if (((uintptr_t)x | (uintptr_t)gy | (uintptr_t)gx) % 4 != 0)
+    return fail(AQD_ERR_INVALID, "x, gy and gx must be 4-byte aligned");
+  if (!workspace || ws_bytes < aqd_fake_quant_backward_workspace_bytes() || (uintptr_t)workspace % 8 != 0)
+    return fail(AQD_ERR_INVALID, "workspace: aqd_fake_quant_backward_workspace_bytes() bytes, 8-byte aligned");
+  const int st = launch_fake_quant_backward(x, gy, n, nu, bits, weight != 0, gx, gnu, static_cast<double*>(workspace),
+                                            kFqParts, static_cast<cudaStream_t>(stream), &err);
+  return st ? fail((aqd_status)st, err) : AQD_OK;
+}
+
+size_t aqd_bn_level_stats_workspace_bytes(int32_t levels, int32_t c) {
+  if (levels <= 0 || levels > kMaxJobs || c <= 0) return 0;
+  return (size_t)2 * bn_stats_blocks(levels) * c * sizeof(double);
+}
+
+aqd_status aqd_bn_level_stats(const float* const* z, const int64_t* pixels, int32_t levels, int32_t c, double* mean,
+                              double* var, void* workspace, size_t ws_bytes, aqd_stream_t stream) {
+  std::string err;
+  if (levels <= 0 || levels > kMaxJobs) return fail(AQD_ERR_INVALID, "levels must be 1..8");
+  if (c <= 0) return fail(AQD_ERR_INVALID, "c must be > 0");
+  if (!z || !pixels || !mean || !var) return fail(AQD_ERR_INVALID, "z, pixels, mean and var are required");
+  for (int l = 0; l < levels; ++l) {
+    if (pixels[l] < 0) return fail(AQD_ERR_INVALID, "pixels must be >= 0");
+    if (pixels[l] > 0 && (!z[l] || (uintptr_t)z[l] % 4 != 0)) return fail(AQD_ERR_INVALID, "z[l] must be 4-byte aligned");
+  }
+  const size_t need = aqd_bn_level_stats_workspace_bytes(levels, c);
+  if (!workspace || ws_bytes < need || (uintptr_t)workspace % 8 != 0)
+    return fail(AQD_ERR_INVALID, "workspace: aqd_bn_level_stats_workspace_bytes() bytes, 8-byte aligned");
+  const int st = launch_bn_level_stats(z, pixels, levels, c, mean, var, static_cast<double*>(workspace),
+                                       static_cast<cudaStream_t>(stream), &err);
+  return st ? fail((aqd_status)st, err) : AQD_OK;
+}
+
 }  // extern "C"
 
 // ---------------------------------------------------------------- static workspace

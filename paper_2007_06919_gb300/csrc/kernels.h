@@ -156,6 +156,18 @@ int launch_maxpool(const PoolArgs& a, cudaStream_t stream, std::string* err);
 // cpad, rows of a.c bytes, one image after another from ws) of its output
 int launch_maxpool_expand(const PoolArgs& a, uint8_t* ws, int32_t cpad, cudaStream_t stream, std::string* err);
 
+// training-side steps (train.cu): Eq. 2 / Eq. 3 fake quantization (weight: Eq. 3), its STE
+// backward (gnu: one float64, the interval's gradient; partial: max_parts float64), and the
+// per-level batch statistics (work: bn_stats_work_doubles(levels, c) float64)
+int launch_fake_quant(const float* x, int64_t n, float nu, int32_t bits, bool weight, float* y, uint8_t* codes,
+                      cudaStream_t stream, std::string* err);
+int launch_fake_quant_backward(const float* x, const float* gy, int64_t n, float nu, int32_t bits, bool weight,
+                               float* gx, double* gnu, double* partial, int32_t max_parts, cudaStream_t stream,
+                               std::string* err);
+int bn_stats_blocks(int32_t levels);
+int launch_bn_level_stats(const float* const* z, const int64_t* pixels, int32_t levels, int32_t c, double* mean,
+                          double* var, double* work, cudaStream_t stream, std::string* err);
+
 // the bounded-wait self-test (selftest.cu): out receives 5 int64 values
 int launch_wait_selftest(uint32_t* status, int64_t* out, cudaStream_t stream, std::string* err);
 

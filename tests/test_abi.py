@@ -144,3 +144,31 @@ def test_workspace_bytes_host_logic(lib):
 def test_set_conv_path_rejects_unknown(lib):
     assert lib.aqd_set_conv_path(7) == -1
     assert lib.aqd_set_conv_path(0) in (0, 1, 2)
+
+
+def test_training_entry_points_validate_before_any_launch(lib):
+    """The training-side entries refuse bad arguments on the host (AQD_ERR_INVALID = 1, no
+    CUDA call made); the workspace queries are pure host arithmetic."""
+    f32 = ctypes.c_float
+    assert lib.aqd_fake_quant_backward_workspace_bytes() >= 8 * 512
+    assert lib.aqd_bn_level_stats_workspace_bytes(0, 256) == 0
+    assert lib.aqd_bn_level_stats_workspace_bytes(9, 256) == 0
+    assert lib.aqd_bn_level_stats_workspace_bytes(5, 0) == 0
+    assert lib.aqd_bn_level_stats_workspace_bytes(5, 256) > 0
+    fake = ctypes.c_void_p(0x1000)  # never dereferenced: the calls fail before any launch
+    for nu, bits, weight in ((0.0, 2, 0), (-1.0, 2, 0), (float("nan"), 2, 0), (float("inf"), 4, 1),
+                             (1.0, 0, 0), (1.0, 9, 0), (1.0, 4, 2)):
+        assert lib.aqd_fake_quant(fake, 16, f32(nu), bits, weight, fake, None, None) == 1
+        assert lib.aqd_fake_quant_backward(fake, fake, 16, f32(nu), bits, weight, fake, fake, fake, 8192, None) == 1
+    assert lib.aqd_fake_quant(fake, -1, f32(1.0), 2, 0, fake, None, None) == 1
+    assert lib.aqd_fake_quant(fake, 16, f32(1.0), 2, 0, None, None, None) == 1          # no output
+    assert lib.aqd_fake_quant(ctypes.c_void_p(0x1002), 16, f32(1.0), 2, 0, fake, None, None) == 1  # misaligned
+    assert lib.aqd_fake_quant_backward(fake, fake, 16, f32(1.0), 2, 0, fake, None, fake, 8192, None) == 1  # no gnu
+    assert lib.aqd_fake_quant_backward(fake, fake, 16, f32(1.0), 2, 0, fake, fake, fake, 8, None) == 1  # small ws
+    ptrs = (ctypes.c_void_p * 1)(fake)
+    pix = (ctypes.c_int64 * 1)(10)
+    assert lib.aqd_bn_level_stats(ptrs, pix, 0, 4, fake, fake, fake, 1 << 20, None) == 1   # levels
+    assert lib.aqd_bn_level_stats(ptrs, pix, 1, 0, fake, fake, fake, 1 << 20, None) == 1   # channels
+    assert lib.aqd_bn_level_stats(ptrs, pix, 1, 4, fake, fake, fake, 8, None) == 1         # workspace
+    neg = (ctypes.c_int64 * 1)(-1)
+    assert lib.aqd_bn_level_stats(ptrs, neg, 1, 4, fake, fake, fake, 1 << 20, None) == 1   # pixels
